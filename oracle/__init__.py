@@ -1,0 +1,156 @@
+"""Plain CPU oracle for the exact LLM output head -- TEST INFRASTRUCTURE ONLY.
+
+Only ``tests/``, ``__graft_entry__.smoke()`` and the ``cpu_baseline`` and
+``--impl reference`` legs of ``bench.py`` may import this package.  The CUDA
+path (``paper_2608_27460_gb300``) never imports it, and this package imports
+nothing from that path: the two share no code.
+
+The arithmetic lives in ``oracle.c`` (plain C, fp64, no blocking); this module
+only builds it with gcc and marshals numpy arrays through ctypes.
+
+  * :func:`logits`  -- z = W_out h, z_i = <w_i, h> in fp64      (Section 3)
+  * :func:`topk`    -- exhaustive MIPS: full sort by (z desc, index asc),
+                       first k rows                               (Sections 2, 3)
+  * :func:`scatter` -- sparse full-vocabulary tensor, -inf except the k
+                       retrieved logits at their indices          (Section 3)
+
+Parity of :func:`topk` against the paper cannot be pinned to printed values
+(the paper prints no worked example); it is pinned instead to hand-worked
+cases, exact rational brute force, Cauchy-Schwarz planted cases, library
+argmax/sort special cases and the sparse-softmax identity (tests/test_oracle_*).
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import threading
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "oracle.c")
+_LIB = os.path.join(_HERE, "liboracle.so")
+_lock = threading.Lock()
+_lib = None
+
+
+def build(force: bool = False, src: str = _SRC, out: str = _LIB) -> str:
+    """Compile oracle.c (or another C file with the same exports) with gcc."""
+    if force or not os.path.exists(out) or os.path.getmtime(out) < os.path.getmtime(src):
+        tmp = out + f".tmp{os.getpid()}"
+        cmd = ["gcc", "-O2", "-fopenmp", "-ffp-contract=off", "-fPIC", "-shared",
+               src, "-o", tmp, "-lm"]
+        subprocess.run(cmd, check=True)
+        os.replace(tmp, out)
+    return out
+
+
+def _ptr(a: np.ndarray) -> int:
+    return a.ctypes.data
+
+
+def _check_inputs(W_bits: np.ndarray, h: np.ndarray):
+    if W_bits.dtype != np.uint16 or W_bits.ndim != 2:
+        raise TypeError("W_bits must be a 2-D uint16 array of bf16 bit patterns")
+    if h.dtype != np.float32:
+        raise TypeError("h must be float32")
+    W_bits = np.ascontiguousarray(W_bits)
+    h = np.ascontiguousarray(h.reshape(-1, W_bits.shape[1]))
+    return W_bits, h
+
+
+class OracleLib:
+    """ctypes marshalling around one compiled copy of the oracle."""
+
+    def __init__(self, path: str):
+        lib = ctypes.CDLL(path)
+        P = ctypes.c_void_p
+        lib.oracle_bf16_to_double.argtypes = [ctypes.c_uint16]
+        lib.oracle_bf16_to_double.restype = ctypes.c_double
+        lib.oracle_logits.argtypes = [P, ctypes.c_int64, ctypes.c_int32, P, ctypes.c_int32, P,
+                                      ctypes.c_int32]
+        lib.oracle_logits.restype = ctypes.c_int
+        lib.oracle_topk.argtypes = [P, ctypes.c_int64, ctypes.c_int32, P, ctypes.c_int32,
+                                    ctypes.c_int32, P, P, ctypes.c_int32]
+        lib.oracle_topk.restype = ctypes.c_int
+        lib.oracle_scatter.argtypes = [P, P, ctypes.c_int32, ctypes.c_int32, ctypes.c_int64, P]
+        lib.oracle_scatter.restype = ctypes.c_int
+        lib.oracle_max_threads.argtypes = []
+        lib.oracle_max_threads.restype = ctypes.c_int
+        self.lib = lib
+        self.path = path
+
+    def max_threads(self) -> int:
+        return int(self.lib.oracle_max_threads())
+
+    def bf16_to_double(self, bits: int) -> float:
+        """Exact widening of one bf16 bit pattern."""
+        return float(self.lib.oracle_bf16_to_double(int(bits) & 0xFFFF))
+
+    def logits(self, W_bits: np.ndarray, h: np.ndarray, threads: int = 0) -> np.ndarray:
+        """fp64 logits [batch, V] of z = W_out h (Section 3)."""
+        W_bits, h = _check_inputs(W_bits, h)
+        V, d = W_bits.shape
+        out = np.empty((h.shape[0], V), dtype=np.float64)
+        rc = self.lib.oracle_logits(_ptr(W_bits), V, d, _ptr(h), h.shape[0], _ptr(out),
+                                    threads or self.max_threads())
+        if rc != 0:
+            raise ValueError(f"oracle_logits failed with code {rc}")
+        return out
+
+    def topk(self, W_bits: np.ndarray, h: np.ndarray, k: int, threads: int = 0):
+        """Exact top-k by full sort: (idx int32 [batch,k], logits fp64 [batch,k])."""
+        W_bits, h = _check_inputs(W_bits, h)
+        V, d = W_bits.shape
+        b = h.shape[0]
+        idx = np.empty((b, max(k, 0)), dtype=np.int32)
+        val = np.empty((b, max(k, 0)), dtype=np.float64)
+        rc = self.lib.oracle_topk(_ptr(W_bits), V, d, _ptr(h), b, k, _ptr(idx), _ptr(val),
+                                  threads or self.max_threads())
+        if rc != 0:
+            raise ValueError(f"oracle_topk failed with code {rc}")
+        return idx, val
+
+    def scatter(self, idx: np.ndarray, logits_f32: np.ndarray, V: int):
+        """Sparse [batch, V] fp32 tensor; returns (out, ok) where ok is False if
+        an index was out of range (that entry is skipped)."""
+        idx = np.ascontiguousarray(idx, dtype=np.int32)
+        logits_f32 = np.ascontiguousarray(logits_f32, dtype=np.float32)
+        if idx.ndim == 1:
+            idx = idx[None, :]
+            logits_f32 = logits_f32[None, :]
+        b, k = idx.shape
+        out = np.empty((b, V), dtype=np.float32)
+        rc = self.lib.oracle_scatter(_ptr(idx), _ptr(logits_f32), b, k, V, _ptr(out))
+        if rc not in (0, 1):
+            raise ValueError(f"oracle_scatter failed with code {rc}")
+        return out, rc == 0
+
+
+def _default() -> OracleLib:
+    global _lib
+    with _lock:
+        if _lib is None:
+            _lib = OracleLib(build())
+    return _lib
+
+
+def max_threads() -> int:
+    return _default().max_threads()
+
+
+def bf16_to_double(bits: int) -> float:
+    return _default().bf16_to_double(bits)
+
+
+def logits(W_bits, h, threads: int = 0):
+    return _default().logits(W_bits, h, threads)
+
+
+def topk(W_bits, h, k: int, threads: int = 0):
+    return _default().topk(W_bits, h, k, threads)
+
+
+def scatter(idx, logits_f32, V: int):
+    return _default().scatter(idx, logits_f32, V)
