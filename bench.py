@@ -1,0 +1,404 @@
+#!/usr/bin/env python3
+"""Benchmark of the exact output head: microseconds per decode step.
+
+One step = the whole hot path over one batch of queries: the fused
+projection + top-k launch (vie_head_topk) and the sparse -inf scatter
+(vie_scatter_sparse_logits).  Default workload: the Qwen3-0.6B-shaped head
+(W_out bf16 [151936, 1024] = 311 MB, larger than the 129 MB L2), batch 1,
+k = 50, seeded synthetic weights and queries (no real checkpoint here).
+
+Prints one JSON line (rank 0).  ``--impl reference`` times the CPU oracle on
+the same workload instead (the reference arm of this build).
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import re
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2608_27460_gb300 import synth  # noqa: E402
+
+METRIC = "output-head µs/decode-step at batch 1; achieved HBM GB/s vs 8 TB/s peak"
+UNIT = "us/step"
+NOMINAL_HBM_GBS = 8000.0
+PROFILE_DIR = os.path.join(ROOT, "profiles")
+KERNEL_SOURCES = ["vie_stream_topk.cuh", "vie_device.cuh", "vie_stream_topk_inst.cuh"]
+
+
+def parse_args(argv=None):
+    ap = argparse.ArgumentParser(description=__doc__)
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=200)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default="qwen3-0.6b", choices=sorted(synth.HEADS))
+    ap.add_argument("--batch", type=int, default=1)
+    ap.add_argument("--k", type=int, default=50)
+    ap.add_argument("--queries", type=int, default=64, help="distinct resident queries cycled")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=15.0, help="oracle sample budget")
+    ap.add_argument("--e2e-steps", type=int, default=200)
+    ap.add_argument("--seed", type=int, default=0)
+    return ap.parse_args(argv)
+
+
+# ---------------------------------------------------------------------------
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+def kernel_source_digest() -> str:
+    h = hashlib.sha256()
+    for f in KERNEL_SOURCES:
+        with open(os.path.join(ROOT, "paper_2608_27460_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def measured_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            return json.load(f), "measured"
+    return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}, "fallback"
+
+
+def profiled_traffic(workload: str, batch: int, k: int):
+    """dram bytes per launch of the projection kernel from a committed ncu
+    summary, if it was taken on the current kernel source; else None."""
+    path = os.path.join(PROFILE_DIR, f"stream_topk_{workload}_b{batch}_k{k}.md")
+    if not os.path.exists(path):
+        return None, None
+    text = open(path).read()
+    m_src = re.search(r"kernel_source_sha256:\s*([0-9a-f]+)", text)
+    m_b = re.search(r"dram_bytes_per_launch:\s*([0-9]+)", text)
+    if not m_src or not m_b:
+        return None, path
+    if m_src.group(1) != kernel_source_digest():
+        return None, path
+    return int(m_b.group(1)), path
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons sampled every 20 ms."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_id: str):
+        self.tmp = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+        self.proc = None
+        self.gpu_id = gpu_id
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu=timestamp,{self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-i", self.gpu_id, "-lms", "20"], stdout=self.tmp, stderr=subprocess.DEVNULL)
+        except (OSError, ValueError):
+            self.proc = None
+        time.sleep(0.3)
+
+    def stop(self):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+        self.tmp.flush()
+        self.tmp.seek(0)
+        rows = [r.split(", ") for r in self.tmp.read().strip().splitlines() if r.count(",") >= 9]
+        self.tmp.close()
+        os.unlink(self.tmp.name)
+        return rows
+
+    @staticmethod
+    def summarize(rows, t0, t1):
+        def ts(r):
+            try:
+                return time.mktime(time.strptime(r[0].split(".")[0], "%Y/%m/%d %H:%M:%S")) + \
+                    float("0." + r[0].split(".")[1]) if "." in r[0] else 0.0
+            except (ValueError, IndexError):
+                return 0.0
+        inside = [r for r in rows if t0 - 0.05 <= ts(r) <= t1 + 0.05]
+        used = inside if inside else rows[-10:]
+        if not used:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no nvidia-smi samples"],
+                    "samples": 0}
+        sm = [float(r[2]) for r in used if r[2].replace(".", "").isdigit()]
+        smax = [float(r[3]) for r in used if r[3].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({n for r in used for n, v in zip(names, r[6:10]) if v.strip() == "Active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(smax) if smax else None, "reasons": reasons,
+                "samples": len(used), "samples_in_timed_region": len(inside)}
+
+
+def gpu_id_for_smi(local_rank: int) -> str:
+    vis = os.environ.get("CUDA_VISIBLE_DEVICES")
+    if vis:
+        ids = [v.strip() for v in vis.split(",") if v.strip()]
+        if local_rank < len(ids):
+            return ids[local_rank]
+    return str(local_rank)
+
+
+# ---------------------------------------------------------------------------
+def cpu_oracle_sample(W, h_pool, k, budget_s, batch):
+    """The oracle, as it stands, on host cores: whole decode steps (top-k by
+    full sort + sparse tensor) until the time budget is spent."""
+    import oracle
+    threads = oracle.max_threads()
+    V = W.shape[0]
+    t0 = time.perf_counter()
+    n = 0
+    results = {}
+    while True:
+        q0 = (n * batch) % len(h_pool)
+        hb = h_pool[q0:q0 + batch]
+        idx, val = oracle.topk(W, hb, k, threads=threads)
+        oracle.scatter(idx, val.astype(np.float32), V)
+        results[q0] = (idx, val)
+        n += 1
+        if time.perf_counter() - t0 >= budget_s:
+            break
+    dt = time.perf_counter() - t0
+    return dt / n * 1e6, n, threads, results
+
+
+def run_reference(args, rank, world):
+    """Reference arm: the CPU oracle timed on this host on the same workload."""
+    if rank != 0:
+        return 0
+    shape = synth.HEADS[args.workload]
+    W, h, _, _ = synth.make_head(shape, seed=args.seed, n_queries=max(args.queries, args.batch))
+    import oracle
+    threads = oracle.max_threads()
+    V = W.shape[0]
+
+    def step(i):
+        q0 = (i * args.batch) % (len(h) - args.batch + 1)
+        idx, val = oracle.topk(W, h[q0:q0 + args.batch], args.k, threads=threads)
+        oracle.scatter(idx, val.astype(np.float32), V)
+
+    for i in range(args.warmup):
+        step(i)
+    t0 = time.perf_counter()
+    for i in range(args.steps):
+        step(i)
+    dt = time.perf_counter() - t0
+    us = dt / max(args.steps, 1) * 1e6
+    line = {
+        "impl": "reference", "metric": METRIC, "value": round(us, 3), "unit": UNIT,
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": round(us / 1e3, 6), "higher_is_better": False, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": workload_config(args, shape),
+        "cpu_baseline": {"value": round(us, 3), "unit": UNIT, "cores": threads, "kind": "oracle",
+                         "sample": f"{args.steps} whole decode steps (batch {args.batch}, full sort, "
+                                   f"sparse tensor) of the {args.workload} workload"},
+        "e2e": {"value": round(us, 3), "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def workload_config(args, shape):
+    return {"workload": f"{shape.name}-shaped head, batch {args.batch}, k {args.k}",
+            "V": shape.V, "d": shape.d, "batch": args.batch, "k": args.k,
+            "weights": "bf16 (fp32 accumulation)", "l2": "inputs larger than L2 (W_out "
+            f"{shape.V * shape.d * 2 / 1e6:.0f} MB vs 129 MB L2), no flush",
+            "queries_cycled": args.queries}
+
+
+# ---------------------------------------------------------------------------
+def main(argv=None):
+    args = parse_args(argv)
+    rank, world, local = dist_env()
+    if args.impl == "reference":
+        return run_reference(args, rank, world)
+
+    import torch
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
+    import paper_2608_27460_gb300 as vie
+    vie.load()
+    dev = torch.device("cuda", local if world > 1 else 0)
+    torch.cuda.set_device(dev)
+
+    shape = synth.HEADS[args.workload]
+    nq = max(args.queries, args.batch)
+    W, h, _, _ = synth.make_head(shape, seed=args.seed + rank * 7919, n_queries=nq)
+    Wd = torch.from_numpy(W.view(np.int16)).to(dev)
+    head = vie.Head(Wd)
+    del Wd
+    hd = torch.from_numpy(h).to(dev)
+    b, k, V = args.batch, args.k, shape.V
+    idx = torch.empty((b, k), dtype=torch.int32, device=dev)
+    val = torch.empty((b, k), dtype=torch.float32, device=dev)
+    sparse = torch.empty((b, V), dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    sptr = int(stream.cuda_stream)
+    starts = [(i * b) % (nq - b + 1) for i in range(nq)]
+
+    def step(i):
+        q0 = starts[i % nq]
+        vie.check(vie.vie_head_topk(head.handle, hd[q0].data_ptr(), b, k, idx.data_ptr(),
+                                    val.data_ptr(), sptr))
+        vie.check(vie.vie_scatter_sparse_logits(idx.data_ptr(), val.data_ptr(), b, k, V,
+                                                sparse.data_ptr(), sptr))
+
+    sampler = ClockSampler(gpu_id_for_smi(local)) if rank == 0 else None
+    if sampler:
+        sampler.start()
+    for i in range(args.warmup):
+        step(i)
+    torch.cuda.synchronize()
+    vie.check(head.device_status())
+
+    K = args.steps
+    ev_a = [torch.cuda.Event(enable_timing=True) for _ in range(K)]
+    ev_b = [torch.cuda.Event(enable_timing=True) for _ in range(K)]
+    start = torch.cuda.Event(enable_timing=True)
+    end = torch.cuda.Event(enable_timing=True)
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    t_wall0 = time.time()
+    start.record(stream)
+    for i in range(K):
+        q0 = starts[i % nq]
+        ev_a[i].record(stream)
+        vie.check(vie.vie_head_topk(head.handle, hd[q0].data_ptr(), b, k, idx.data_ptr(),
+                                    val.data_ptr(), sptr))
+        ev_b[i].record(stream)
+        vie.check(vie.vie_scatter_sparse_logits(idx.data_ptr(), val.data_ptr(), b, k, V,
+                                                sparse.data_ptr(), sptr))
+    end.record(stream)
+    torch.cuda.synchronize()
+    t_wall1 = time.time()
+    if world > 1:
+        torch.distributed.barrier()
+    total_ms = start.elapsed_time(end)
+    kern_ms = [a.elapsed_time(c) for a, c in zip(ev_a, ev_b)]
+    clocks = sampler.stop() if sampler else []
+    vie.check(head.device_status())
+
+    if world > 1:
+        t = torch.tensor([total_ms], device=dev)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        total_ms = float(t.item())
+
+    # end-to-end through the public API with host buffers: pinned h in, the
+    # step's top-k (indices + logits) back to pinned host memory every step
+    h_host = torch.from_numpy(h).pin_memory()
+    idx_host = torch.empty((b, k), dtype=torch.int32).pin_memory()
+    val_host = torch.empty((b, k), dtype=torch.float32).pin_memory()
+    h_stage = torch.empty((b, shape.d), dtype=torch.float32, device=dev)
+    E = args.e2e_steps
+    for i in range(min(20, E)):
+        q0 = starts[i % nq]
+        h_stage.copy_(h_host[q0:q0 + b], non_blocking=True)
+        head.topk(h_stage, k, out_idx=idx, out_logits=val)
+        head.sparse_logits(idx, val, out=sparse)
+        idx_host.copy_(idx, non_blocking=True)
+        val_host.copy_(val, non_blocking=True)
+        stream.synchronize()
+    e_start = torch.cuda.Event(enable_timing=True)
+    e_end = torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    e_start.record(stream)
+    for i in range(E):
+        q0 = starts[i % nq]
+        h_stage.copy_(h_host[q0:q0 + b], non_blocking=True)
+        head.topk(h_stage, k, out_idx=idx, out_logits=val)
+        head.sparse_logits(idx, val, out=sparse)
+        idx_host.copy_(idx, non_blocking=True)
+        val_host.copy_(val, non_blocking=True)
+        stream.synchronize()  # the host needs the step's tokens before the next step
+    e_end.record(stream)
+    torch.cuda.synchronize()
+    e2e_us = e_start.elapsed_time(e_end) * 1e3 / E
+
+    if rank != 0:
+        head.close()
+        if world > 1:
+            torch.distributed.destroy_process_group()
+        return 0
+
+    props = head.props
+    peaks, peak_src = measured_peaks()
+    kern_us = statistics.mean(kern_ms) * 1e3
+    w_bytes = shape.V * props.d_pad * 2
+    alg_bytes = w_bytes + b * shape.d * 4 + b * k * 8
+    achieved = alg_bytes / (kern_us * 1e-6) / 1e9
+    traffic, prof_path = profiled_traffic(args.workload, b, k)
+    step_us = total_ms * 1e3 / K
+    value = step_us / world
+    launches_per_step = -(-b // max(1, min(8, b))) + 1
+
+    line = {
+        "metric": METRIC, "value": round(value, 3), "unit": UNIT, "n_gpus": world,
+        "steps": K, "warmup": args.warmup, "ms_per_step": round(step_us / 1e3, 6),
+        "higher_is_better": False, "scaling": "weak", "vs_baseline": None,
+        "dtype": "f32", "data": "synthetic", "config": workload_config(args, shape),
+        "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": peaks["hbm_gbs"],
+                     "unit": "GB/s", "frac": round(achieved / peaks["hbm_gbs"], 4),
+                     "traffic": traffic, "peak_source": peak_src,
+                     "kernel": "stream_topk_kernel", "kernel_us": round(kern_us, 3),
+                     "algorithmic_bytes_per_launch": alg_bytes,
+                     "frac_of_nominal_8tbs": round(achieved / NOMINAL_HBM_GBS, 4),
+                     "w_only_gbs": round(w_bytes / (kern_us * 1e-6) / 1e9, 1),
+                     "kernel_us_p10_p50_p90": [round(float(np.percentile(kern_ms, q)) * 1e3, 2)
+                                               for q in (10, 50, 90)]},
+        "e2e": {"value": round(e2e_us, 3), "unit": UNIT, "h2d_bytes_per_step": b * shape.d * 4,
+                "d2h_bytes_per_step": b * k * 8},
+        "gpu_launches": K * launches_per_step,
+        "clocks": ClockSampler.summarize(clocks, t_wall0, t_wall1),
+    }
+    if not args.no_cpu_baseline and world == 1:
+        us, n, threads, results = cpu_oracle_sample(W, h, k, args.cpu_seconds, b)
+        line["cpu_baseline"] = {"value": round(us, 1), "unit": UNIT, "cores": threads, "kind": "oracle",
+                                "sample": f"{n} decode steps (batch {b}) of the same workload in "
+                                          f"{args.cpu_seconds:.0f} s: fp64 projection, full sort, "
+                                          "sparse tensor"}
+        # two of the sampled steps double as a parity check of the device path
+        sys.path.insert(0, os.path.join(ROOT, "tests"))
+        import oracle
+        from acceptance import check_topk
+        ok = True
+        for q0 in list(results)[:2]:
+            gi, gv = head.topk(hd[q0:q0 + b], k)
+            torch.cuda.synchronize()
+            z = oracle.logits(W, h[q0:q0 + b])
+            for q in range(b):
+                ok &= not check_topk(gi.cpu().numpy()[q], gv.cpu().numpy()[q], z[q], k)
+        line["parity_sample_ok"] = bool(ok)
+    print(json.dumps(line), flush=True)
+    head.close()
+    if world > 1:
+        torch.distributed.destroy_process_group()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

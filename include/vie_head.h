@@ -1,0 +1,155 @@
+/*
+ * vie_head.h - C ABI of the exact LLM output head for GB300 (sm_103a).
+ *
+ * The head computes, for each decode query h (paper, Section 3):
+ *     z = W_out h,            z_i = <w_i, h>        (W_out: V rows of width d)
+ * selects the k rows with the largest z_i (exhaustive maximum inner product
+ * search, Sections 2-3) and can write those k logits into a full-vocabulary
+ * tensor that is -infinity everywhere else (Section 3, the sparse logit
+ * tensor handed to standard logit processors).
+ *
+ * Conventions shared by every call:
+ *   - Pointers marked "device" are CUDA device pointers of the device that is
+ *     current on the calling thread; "host" pointers are ordinary memory.
+ *   - A vie_stream is a cudaStream_t (NULL = the legacy default stream).  Calls
+ *     that take a stream are asynchronous on it: they validate on the host,
+ *     enqueue kernels and return without synchronising.
+ *   - Every call returns a vie_status.  On anything but VIE_OK,
+ *     vie_last_error() returns a message for the calling thread.  Argument
+ *     errors are detected on the host before anything is enqueued; they leave
+ *     no CUDA error behind.
+ *   - Device-side problems (an out-of-range scatter index, a pipeline wait
+ *     that ran past its time limit) never trap: the kernel records a flag and
+ *     returns, and the next vie_device_status / vie_head_device_status call
+ *     reports VIE_ERR_DEVICE.
+ *   - Logits are fp32.  Ranking is by logit descending; equal logits are
+ *     ranked by ascending vocabulary index, and -0.0 ranks as +0.0 (and is
+ *     returned as +0.0).  Inputs must be finite; results for NaN or infinite
+ *     inputs are unspecified.
+ */
+#ifndef VIE_HEAD_H
+#define VIE_HEAD_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct vie_head vie_head; /* opaque handle */
+typedef void *vie_stream;         /* a cudaStream_t */
+
+typedef enum {
+    VIE_OK = 0,
+    VIE_ERR_INVALID_ARG = 1, /* a pointer, size or enum value is out of range */
+    VIE_ERR_UNSUPPORTED = 2, /* valid request beyond what this build serves  */
+    VIE_ERR_CUDA = 3,        /* a CUDA runtime call or a launch failed        */
+    VIE_ERR_OOM = 4,         /* device memory could not be allocated          */
+    VIE_ERR_DEVICE = 5       /* a kernel recorded a device-side problem       */
+} vie_status;
+
+typedef enum { VIE_DTYPE_BF16 = 0 } vie_dtype;
+
+/* Limits of this build. */
+#define VIE_K_MAX 1024     /* largest k of vie_head_topk                    */
+#define VIE_BATCH_MAX 1024 /* largest batch of vie_head_topk                */
+#define VIE_D_MAX 16384    /* largest hidden size d                         */
+
+/* Read-only facts about a handle (for callers that size buffers or report). */
+typedef struct {
+    int64_t V;            /* vocabulary rows                                 */
+    int32_t d;            /* hidden size                                     */
+    int32_t d_pad;        /* row pitch in elements: d rounded up to 8        */
+    int32_t ctas;         /* CTAs of one projection launch (one per SM max)  */
+    int32_t device;       /* CUDA device ordinal the handle lives on         */
+    int64_t weight_bytes; /* bytes of the owned padded copy of W_out         */
+    int64_t scratch_bytes;/* bytes of per-handle scratch                      */
+} vie_head_props;
+
+/*
+ * vie_head_create - take a copy of W_out in the layout the kernels stream.
+ * Section 3 treats the rows of W_out as a static database that is prepared
+ * once and reused for every query; this is that preparation step.
+ *
+ *   W_out  device, bf16 (raw bit patterns), row-major [V, d], any alignment
+ *          of 2 bytes.  Only read during the call; the caller may free it
+ *          afterwards.
+ *   V      1 <= V <= 2^31 - 2;   d   1 <= d <= VIE_D_MAX;
+ *   dtype  VIE_DTYPE_BF16 (the only dtype of this build).
+ *   out    host; receives the new handle.
+ *
+ * The handle owns a padded copy [V, d_pad] (d_pad = d rounded up to a
+ * multiple of 8, pad = +0) plus its scratch.  The copy runs on the legacy
+ * default stream of the current device and the call returns after the device
+ * has finished it.  Errors: VIE_ERR_INVALID_ARG (null pointer, bad size,
+ * W_out not device memory of the current device), VIE_ERR_UNSUPPORTED
+ * (dtype), VIE_ERR_OOM, VIE_ERR_CUDA.
+ */
+vie_status vie_head_create(const void *W_out, int64_t V, int32_t d, vie_dtype dtype,
+                           vie_head **out);
+
+/* Frees the padded copy and the scratch.  NULL is accepted.  The caller must
+ * make sure no work using the handle is still running (synchronise first). */
+vie_status vie_head_destroy(vie_head *head);
+
+/* Fills *props (host) with the handle's facts. */
+vie_status vie_head_get_props(const vie_head *head, vie_head_props *props);
+
+/*
+ * vie_head_topk - exact top-k of z = W_out h for a batch of queries
+ * (Section 3: output projection followed by top-k selection, computed by
+ * exhaustive MIPS over every row, Section 2).
+ *
+ *   h           device, fp32, row-major [batch, d] (4-byte aligned).
+ *   batch       1 <= batch <= VIE_BATCH_MAX.
+ *   k           1 <= k <= min(V, VIE_K_MAX).
+ *   out_idx     device, int32 [batch, k]: vocabulary indices, best first.
+ *   out_logits  device, fp32  [batch, k]: their logits (fp32 accumulation of
+ *               the bf16 x fp32 products).
+ *   stream      the stream the work is enqueued on.
+ *
+ * The full logit vector is never written to memory.  Calls using the same
+ * handle share its scratch, so at most one vie_head_topk per handle may be
+ * in flight at a time (calls on one stream are naturally serialised).
+ * No allocation and no host synchronisation happen inside the call.
+ * Errors: VIE_ERR_INVALID_ARG, VIE_ERR_CUDA (launch failure).
+ */
+vie_status vie_head_topk(vie_head *head, const float *h, int32_t batch, int32_t k,
+                         int32_t *out_idx, float *out_logits, vie_stream stream);
+
+/*
+ * vie_scatter_sparse_logits - the sparse full-vocabulary logit tensor of
+ * Section 3: out[b, v] = -inf (bit pattern 0xFF800000) for every v, then
+ * out[b, idx[b, j]] = logits[b, j] for j < k (values copied bit for bit).
+ *
+ *   idx     device, int32 [batch, k];   logits  device, fp32 [batch, k].
+ *   batch   >= 1;  k >= 1;  V >= 1.
+ *   out     device, fp32 [batch, V] (4-byte aligned).
+ *
+ * Indices within a row are expected to be distinct; if they repeat, which
+ * value lands is unspecified.  An index outside [0, V) is skipped and sets
+ * the device flag reported by vie_device_status.  No allocation, no sync.
+ */
+vie_status vie_scatter_sparse_logits(const int32_t *idx, const float *logits, int32_t batch,
+                                     int32_t k, int64_t V, float *out, vie_stream stream);
+
+/*
+ * vie_device_status - synchronises `stream`, then reads and clears the
+ * library's device-side flag word of the current device.  Returns VIE_OK when
+ * no kernel recorded a problem, VIE_ERR_DEVICE otherwise (vie_last_error()
+ * names the problem), VIE_ERR_CUDA if the synchronisation itself failed.
+ */
+vie_status vie_device_status(vie_stream stream);
+
+/* Same as vie_device_status for the handle's device, and also re-arms the
+ * handle's scratch counters after a device-side problem. */
+vie_status vie_head_device_status(vie_head *head, vie_stream stream);
+
+/* Message for the last failing call on this thread ("" if none). */
+const char *vie_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* VIE_HEAD_H */

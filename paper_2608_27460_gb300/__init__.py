@@ -1,0 +1,226 @@
+"""Exact LLM output head for GB300: Python binding of ``libviehead.so``.
+
+The computation (paper, Section 3): z = W_out h over the whole vocabulary,
+the k largest logits (exhaustive maximum inner product search), and the
+sparse full-vocabulary tensor holding those k logits with -inf elsewhere.
+Every step runs in the CUDA kernels of ``libviehead.so``; this module only
+marshals arguments through ctypes.  There is no CPU fallback: if the library
+cannot be built or loaded, :func:`load` raises.
+
+Functions named like the C ABI (``vie_head_create`` ...) take raw pointers
+(ints) and return the ``vie_status`` code; :class:`Head` wraps them for
+torch tensors and raises :class:`VieError` on failure.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "libviehead.so")
+
+VIE_OK = 0
+VIE_ERR_INVALID_ARG = 1
+VIE_ERR_UNSUPPORTED = 2
+VIE_ERR_CUDA = 3
+VIE_ERR_OOM = 4
+VIE_ERR_DEVICE = 5
+VIE_DTYPE_BF16 = 0
+VIE_K_MAX = 1024
+VIE_BATCH_MAX = 1024
+VIE_D_MAX = 16384
+
+STATUS_NAMES = {0: "VIE_OK", 1: "VIE_ERR_INVALID_ARG", 2: "VIE_ERR_UNSUPPORTED",
+                3: "VIE_ERR_CUDA", 4: "VIE_ERR_OOM", 5: "VIE_ERR_DEVICE"}
+
+# Every entry point of include/vie_head.h.
+EXPORTS = ("vie_head_create", "vie_head_destroy", "vie_head_get_props", "vie_head_topk",
+           "vie_scatter_sparse_logits", "vie_device_status", "vie_head_device_status",
+           "vie_last_error")
+
+
+class VieError(RuntimeError):
+    def __init__(self, status: int, message: str):
+        super().__init__(f"{STATUS_NAMES.get(status, status)}: {message}")
+        self.status = status
+        self.message = message
+
+
+class vie_head_props(ctypes.Structure):
+    _fields_ = [("V", ctypes.c_int64), ("d", ctypes.c_int32), ("d_pad", ctypes.c_int32),
+                ("ctas", ctypes.c_int32), ("device", ctypes.c_int32),
+                ("weight_bytes", ctypes.c_int64), ("scratch_bytes", ctypes.c_int64)]
+
+
+_lib = None
+_lock = threading.Lock()
+
+
+def load(path: str | None = None, build_if_missing: bool = True):
+    """Load libviehead.so (building it in-tree first if it is missing or
+    older than its sources).  Raises if that is impossible."""
+    global _lib
+    with _lock:
+        if _lib is not None and path is None:
+            return _lib
+        p = path or LIB_PATH
+        if path is None and build_if_missing:
+            from . import build as _build
+            if not _build.up_to_date():
+                _build.build()
+        if not os.path.exists(p):
+            raise RuntimeError(f"CUDA extension not built: {p} is missing "
+                               "(run python -m paper_2608_27460_gb300.build)")
+        lib = ctypes.CDLL(p)
+        P, I32, I64 = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64
+        sig = {
+            "vie_head_create": ([P, I64, I32, ctypes.c_int, ctypes.POINTER(P)], ctypes.c_int),
+            "vie_head_destroy": ([P], ctypes.c_int),
+            "vie_head_get_props": ([P, ctypes.POINTER(vie_head_props)], ctypes.c_int),
+            "vie_head_topk": ([P, P, I32, I32, P, P, P], ctypes.c_int),
+            "vie_scatter_sparse_logits": ([P, P, I32, I32, I64, P, P], ctypes.c_int),
+            "vie_device_status": ([P], ctypes.c_int),
+            "vie_head_device_status": ([P, P], ctypes.c_int),
+            "vie_last_error": ([], ctypes.c_char_p),
+        }
+        for name, (args, res) in sig.items():
+            fn = getattr(lib, name)
+            fn.argtypes = args
+            fn.restype = res
+        if path is None:
+            _lib = lib
+        return lib
+
+
+# ---- same names as the C ABI: raw pointers in, status out -----------------
+
+def vie_last_error() -> str:
+    return load().vie_last_error().decode(errors="replace")
+
+
+def vie_head_create(W_out: int, V: int, d: int, dtype: int = VIE_DTYPE_BF16):
+    """Returns (status, handle)."""
+    out = ctypes.c_void_p(0)
+    st = load().vie_head_create(W_out, V, d, dtype, ctypes.byref(out))
+    return st, out.value
+
+
+def vie_head_destroy(head: int) -> int:
+    return load().vie_head_destroy(head)
+
+
+def vie_head_get_props(head: int):
+    """Returns (status, vie_head_props)."""
+    props = vie_head_props()
+    st = load().vie_head_get_props(head, ctypes.byref(props))
+    return st, props
+
+
+def vie_head_topk(head: int, h: int, batch: int, k: int, out_idx: int, out_logits: int,
+                  stream: int = 0) -> int:
+    return load().vie_head_topk(head, h, batch, k, out_idx, out_logits, stream)
+
+
+def vie_scatter_sparse_logits(idx: int, logits: int, batch: int, k: int, V: int, out: int,
+                              stream: int = 0) -> int:
+    return load().vie_scatter_sparse_logits(idx, logits, batch, k, V, out, stream)
+
+
+def vie_device_status(stream: int = 0) -> int:
+    return load().vie_device_status(stream)
+
+
+def vie_head_device_status(head: int, stream: int = 0) -> int:
+    return load().vie_head_device_status(head, stream)
+
+
+def check(status: int) -> None:
+    if status != VIE_OK:
+        raise VieError(status, vie_last_error())
+
+
+# ---- torch convenience layer ----------------------------------------------
+
+def _stream_ptr(stream) -> int:
+    import torch
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return int(stream.cuda_stream)
+
+
+class Head:
+    """An output head on the current CUDA device.
+
+    ``W`` is a CUDA tensor [V, d] of dtype bfloat16 (or int16/uint16 holding
+    bf16 bit patterns).  The head keeps its own padded copy, so ``W`` may be
+    freed afterwards."""
+
+    def __init__(self, W):
+        import torch
+        if not W.is_cuda or W.dim() != 2:
+            raise ValueError("W must be a 2-D CUDA tensor")
+        if W.dtype not in (torch.bfloat16, torch.int16, torch.uint16):
+            raise ValueError("W must hold bf16 values (bfloat16, or int16/uint16 bit patterns)")
+        W = W.contiguous()
+        self.V, self.d = int(W.shape[0]), int(W.shape[1])
+        self.device = W.device
+        with torch.cuda.device(W.device):
+            st, hd = vie_head_create(W.data_ptr(), self.V, self.d, VIE_DTYPE_BF16)
+        check(st)
+        self._h = hd
+        st, self.props = vie_head_get_props(hd)
+        check(st)
+
+    @property
+    def handle(self) -> int:
+        if not self._h:
+            raise ValueError("head is closed")
+        return self._h
+
+    def topk(self, h, k: int, out_idx=None, out_logits=None, stream=None):
+        """Top-k (indices int32 [batch, k], logits fp32 [batch, k]) of W h."""
+        import torch
+        if h.dim() == 1:
+            h = h[None]
+        if h.dtype != torch.float32 or not h.is_cuda or h.shape[1] != self.d:
+            raise ValueError(f"h must be a CUDA float32 tensor [batch, {self.d}]")
+        h = h.contiguous()
+        b = int(h.shape[0])
+        if out_idx is None:
+            out_idx = torch.empty((b, k), dtype=torch.int32, device=h.device)
+        if out_logits is None:
+            out_logits = torch.empty((b, k), dtype=torch.float32, device=h.device)
+        check(vie_head_topk(self.handle, h.data_ptr(), b, k, out_idx.data_ptr(),
+                            out_logits.data_ptr(), _stream_ptr(stream)))
+        return out_idx, out_logits
+
+    def sparse_logits(self, idx, logits, out=None, stream=None):
+        """Sparse [batch, V] fp32 tensor: -inf except logits at idx."""
+        import torch
+        b, k = int(idx.shape[0]), int(idx.shape[1])
+        if out is None:
+            out = torch.empty((b, self.V), dtype=torch.float32, device=idx.device)
+        check(vie_scatter_sparse_logits(idx.data_ptr(), logits.data_ptr(), b, k, self.V,
+                                        out.data_ptr(), _stream_ptr(stream)))
+        return out
+
+    def device_status(self, stream=None) -> int:
+        return vie_head_device_status(self.handle, _stream_ptr(stream))
+
+    def close(self):
+        if getattr(self, "_h", None):
+            vie_head_destroy(self._h)
+            self._h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def __enter__(self):
+        return self
+
+    def __exit__(self, *exc):
+        self.close()

@@ -1,0 +1,395 @@
+// vie_head.cu - the C ABI declared in include/vie_head.h: argument checks,
+// handle life cycle, launch configuration, weight-layout preparation and
+// the sparse-logit scatter kernel.
+#include <cuda_runtime.h>
+
+#include <climits>
+#include <cstdarg>
+#include <cstdint>
+#include <cstdio>
+#include <cstring>
+#include <new>
+
+#include "vie_head.h"
+#include "vie_launch.h"
+
+namespace {
+
+thread_local char g_err[512] = "";
+
+vie_status fail(vie_status st, const char *fmt, ...) {
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(g_err, sizeof g_err, fmt, ap);
+    va_end(ap);
+    return st;
+}
+
+vie_status fail_cuda(cudaError_t e, const char *what) {
+    return fail(e == cudaErrorMemoryAllocation ? VIE_ERR_OOM : VIE_ERR_CUDA, "%s: %s (%s)", what,
+                cudaGetErrorString(e), cudaGetErrorName(e));
+}
+
+// Library-wide device flag word (used by kernels that have no handle).
+__device__ uint32_t g_dev_err = 0;
+
+constexpr int kMaxSmem = 232448;  // 227 KB opt-in dynamic shared memory per CTA
+constexpr int kMaxNB = 8;
+constexpr int kMaxHBytes = 64 * 1024;  // shared-memory budget for staged queries
+
+}  // namespace
+
+struct vie_head {
+    int device;
+    int64_t V;
+    int32_t d, d_pad;
+    int num_sms;
+    int G;
+    uint16_t *W;        // [V, d_pad] bf16 bits
+    uint64_t *cand;     // [kMaxNB][G][VIE_K_MAX] ranking keys
+    uint32_t *words;    // [0] completion ticket, [1] device flag word
+    int64_t scratch_bytes;
+};
+
+// ---------------------------------------------------------------------------
+// Weight-layout preparation: [V, d] (any 2-byte alignment) -> [V, d_pad]
+// with 16-byte rows, pad columns = +0.  One thread per 16-byte output chunk.
+__global__ void prep_weights_kernel(const uint16_t *__restrict__ src, int64_t V, int d, int d_pad,
+                                    uint16_t *__restrict__ dst) {
+    const int C = d_pad >> 3;
+    const int64_t n = V * C;
+    for (int64_t id = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; id < n;
+         id += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+        const int64_t row = id / C;
+        const int c = static_cast<int>(id - row * C);
+        uint16_t v[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+            const int col = c * 8 + e;
+            v[e] = col < d ? src[row * d + col] : static_cast<uint16_t>(0);
+        }
+        uint4 o;
+        o.x = v[0] | (static_cast<uint32_t>(v[1]) << 16);
+        o.y = v[2] | (static_cast<uint32_t>(v[3]) << 16);
+        o.z = v[4] | (static_cast<uint32_t>(v[5]) << 16);
+        o.w = v[6] | (static_cast<uint32_t>(v[7]) << 16);
+        reinterpret_cast<uint4 *>(dst)[id] = o;
+    }
+}
+
+// ---------------------------------------------------------------------------
+// Sparse full-vocabulary logits (paper, Section 3): row b of `out` becomes
+// -inf everywhere, then logits[b, j] lands at idx[b, j].  Each CTA owns a
+// contiguous slice of one row: it fills the slice, synchronises, then writes
+// the retrieved logits that fall inside the slice, so every fill of a slot
+// happens before its value is written.
+__global__ void scatter_sparse_kernel(const int32_t *__restrict__ idx,
+                                      const float *__restrict__ logits, int k, int64_t V,
+                                      int64_t per_cta, float *__restrict__ out, int batch_base,
+                                      uint32_t *err) {
+    const int b = batch_base + blockIdx.y;
+    float *row = out + static_cast<int64_t>(b) * V;
+    const int64_t lo = blockIdx.x * per_cta;
+    const int64_t hi = min(V, lo + per_cta);
+    const float ninf = __uint_as_float(0xFF800000u);
+    if (lo < hi) {
+        // scalar head up to 16-byte alignment, float4 body, scalar tail
+        const uintptr_t a = reinterpret_cast<uintptr_t>(row + lo);
+        int64_t head = static_cast<int64_t>(((16 - (a & 15)) & 15) >> 2);
+        if (head > hi - lo) head = hi - lo;
+        for (int64_t i = threadIdx.x; i < head; i += blockDim.x) row[lo + i] = ninf;
+        const int64_t body0 = lo + head;
+        const int64_t nvec = (hi - body0) >> 2;
+        float4 *vp = reinterpret_cast<float4 *>(row + body0);
+        const float4 f4 = make_float4(ninf, ninf, ninf, ninf);
+        for (int64_t i = threadIdx.x; i < nvec; i += blockDim.x) vp[i] = f4;
+        for (int64_t i = body0 + nvec * 4 + threadIdx.x; i < hi; i += blockDim.x) row[i] = ninf;
+    }
+    __syncthreads();
+    for (int j = threadIdx.x; j < k; j += blockDim.x) {
+        const int32_t t = idx[static_cast<int64_t>(b) * k + j];
+        if (t < 0 || static_cast<int64_t>(t) >= V) {
+            if (blockIdx.x == 0) atomicOr(err, vie::kErrScatterIndex);
+            continue;
+        }
+        if (t >= lo && t < hi) row[t] = logits[static_cast<int64_t>(b) * k + j];
+    }
+}
+
+// ---------------------------------------------------------------------------
+namespace {
+
+int pick_mm(int k) { return k <= 64 ? 2 : (k <= 256 ? 8 : 32); }
+
+// Widest query group for a row width and list width: the staged queries
+// must fit their shared-memory budget and the selector's lists its registers.
+int nb_cap_for(int d_pad, int mm) {
+    int nb = mm >= 32 ? 1 : (mm >= 8 ? 4 : kMaxNB);
+    while (nb > 1 && nb * d_pad * 4 > kMaxHBytes) nb >>= 1;
+    return nb;
+}
+
+// Stage rows and ring depth for one launch shape: aim for ~32 KB stages and
+// the deepest ring that fits in shared memory.
+bool pick_ring(int nb, int d_pad, int *rs_out, int *stages_out, uint32_t *smem_out) {
+    const int row_bytes = d_pad * 2;
+    int rs = 32768 / row_bytes;
+    if (rs < 1) rs = 1;
+    if (rs > 32) rs = 32;
+    for (; rs >= 1; rs = (rs > 1 ? rs / 2 : 0)) {
+        for (int s = vie::kMaxStages; s >= 2; --s) {
+            const vie::SmemLayout L(nb, d_pad, rs, s, row_bytes);
+            if (L.total <= static_cast<uint32_t>(kMaxSmem)) {
+                *rs_out = rs;
+                *stages_out = s;
+                *smem_out = L.total;
+                return true;
+            }
+        }
+        if (rs == 1) break;
+    }
+    return false;
+}
+
+vie_status check_device(const vie_head *hd) {
+    int dev = -1;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return fail_cuda(e, "cudaGetDevice");
+    if (dev != hd->device)
+        return fail(VIE_ERR_INVALID_ARG, "handle lives on device %d but device %d is current",
+                    hd->device, dev);
+    return VIE_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char *vie_last_error(void) { return g_err; }
+
+vie_status vie_head_create(const void *W_out, int64_t V, int32_t d, vie_dtype dtype,
+                           vie_head **out) {
+    if (out == nullptr) return fail(VIE_ERR_INVALID_ARG, "vie_head_create: out is NULL");
+    *out = nullptr;
+    if (W_out == nullptr) return fail(VIE_ERR_INVALID_ARG, "vie_head_create: W_out is NULL");
+    if (V < 1 || V > static_cast<int64_t>(INT32_MAX) - 1)
+        return fail(VIE_ERR_INVALID_ARG, "vie_head_create: V=%lld outside [1, 2^31-2]",
+                    static_cast<long long>(V));
+    if (d < 1 || d > VIE_D_MAX)
+        return fail(VIE_ERR_INVALID_ARG, "vie_head_create: d=%d outside [1, %d]", d, VIE_D_MAX);
+    if (dtype != VIE_DTYPE_BF16)
+        return fail(VIE_ERR_UNSUPPORTED, "vie_head_create: dtype %d is not supported (bf16 only)",
+                    static_cast<int>(dtype));
+    if (reinterpret_cast<uintptr_t>(W_out) & 1u)
+        return fail(VIE_ERR_INVALID_ARG, "vie_head_create: W_out is not 2-byte aligned");
+
+    int dev = -1;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return fail_cuda(e, "cudaGetDevice");
+    cudaPointerAttributes pa;
+    e = cudaPointerGetAttributes(&pa, W_out);
+    if (e != cudaSuccess) {
+        cudaGetLastError();
+        return fail(VIE_ERR_INVALID_ARG, "vie_head_create: W_out is not a CUDA pointer");
+    }
+    if ((pa.type != cudaMemoryTypeDevice && pa.type != cudaMemoryTypeManaged) || pa.device != dev)
+        return fail(VIE_ERR_INVALID_ARG,
+                    "vie_head_create: W_out must be device memory of the current device %d", dev);
+
+    int sms = 0;
+    e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (e != cudaSuccess) return fail_cuda(e, "cudaDeviceGetAttribute");
+
+    vie_head *hd = new (std::nothrow) vie_head();
+    if (hd == nullptr) return fail(VIE_ERR_OOM, "vie_head_create: host allocation failed");
+    hd->device = dev;
+    hd->V = V;
+    hd->d = d;
+    hd->d_pad = (d + 7) & ~7;
+    hd->num_sms = sms;
+    int64_t g = (V + 63) / 64;
+    if (g > sms) g = sms;
+    if (g > vie::kMaxLists) g = vie::kMaxLists;
+    hd->G = static_cast<int>(g < 1 ? 1 : g);
+
+    const size_t wbytes = static_cast<size_t>(V) * hd->d_pad * 2;
+    const size_t cbytes = static_cast<size_t>(kMaxNB) * hd->G * VIE_K_MAX * sizeof(uint64_t);
+    hd->scratch_bytes = static_cast<int64_t>(cbytes + 2 * sizeof(uint32_t));
+    e = cudaMalloc(&hd->W, wbytes);
+    if (e == cudaSuccess) e = cudaMalloc(&hd->cand, cbytes);
+    if (e == cudaSuccess) e = cudaMalloc(&hd->words, 2 * sizeof(uint32_t));
+    if (e == cudaSuccess) e = cudaMemset(hd->words, 0, 2 * sizeof(uint32_t));
+    if (e == cudaSuccess) {
+        const int64_t chunks = V * (hd->d_pad >> 3);
+        int64_t blocks = (chunks + 255) / 256;
+        if (blocks > 32LL * sms) blocks = 32LL * sms;
+        prep_weights_kernel<<<static_cast<unsigned>(blocks), 256>>>(
+            static_cast<const uint16_t *>(W_out), V, d, hd->d_pad, hd->W);
+        e = cudaGetLastError();
+    }
+    if (e == cudaSuccess) e = cudaDeviceSynchronize();
+    if (e != cudaSuccess) {
+        const vie_status st = fail_cuda(e, "vie_head_create");
+        cudaFree(hd->W);
+        cudaFree(hd->cand);
+        cudaFree(hd->words);
+        delete hd;
+        return st;
+    }
+    *out = hd;
+    return VIE_OK;
+}
+
+vie_status vie_head_destroy(vie_head *head) {
+    if (head == nullptr) return VIE_OK;
+    cudaFree(head->W);
+    cudaFree(head->cand);
+    cudaFree(head->words);
+    delete head;
+    return VIE_OK;
+}
+
+vie_status vie_head_get_props(const vie_head *head, vie_head_props *props) {
+    if (head == nullptr || props == nullptr)
+        return fail(VIE_ERR_INVALID_ARG, "vie_head_get_props: NULL argument");
+    props->V = head->V;
+    props->d = head->d;
+    props->d_pad = head->d_pad;
+    props->ctas = head->G;
+    props->device = head->device;
+    props->weight_bytes = head->V * head->d_pad * 2;
+    props->scratch_bytes = head->scratch_bytes;
+    return VIE_OK;
+}
+
+vie_status vie_head_topk(vie_head *head, const float *h, int32_t batch, int32_t k,
+                         int32_t *out_idx, float *out_logits, vie_stream stream) {
+    if (head == nullptr) return fail(VIE_ERR_INVALID_ARG, "vie_head_topk: head is NULL");
+    if (h == nullptr || out_idx == nullptr || out_logits == nullptr)
+        return fail(VIE_ERR_INVALID_ARG, "vie_head_topk: NULL buffer");
+    if (batch < 1 || batch > VIE_BATCH_MAX)
+        return fail(VIE_ERR_INVALID_ARG, "vie_head_topk: batch=%d outside [1, %d]", batch,
+                    VIE_BATCH_MAX);
+    if (k < 1 || k > VIE_K_MAX || static_cast<int64_t>(k) > head->V)
+        return fail(VIE_ERR_INVALID_ARG, "vie_head_topk: k=%d outside [1, min(V=%lld, %d)]", k,
+                    static_cast<long long>(head->V), VIE_K_MAX);
+    if ((reinterpret_cast<uintptr_t>(h) | reinterpret_cast<uintptr_t>(out_idx) |
+         reinterpret_cast<uintptr_t>(out_logits)) & 3u)
+        return fail(VIE_ERR_INVALID_ARG, "vie_head_topk: buffers must be 4-byte aligned");
+    vie_status st = check_device(head);
+    if (st != VIE_OK) return st;
+
+    const int mm = pick_mm(k);
+    const int cap = nb_cap_for(head->d_pad, mm);
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    for (int q0 = 0; q0 < batch; q0 += cap) {
+        const int nq = batch - q0 < cap ? batch - q0 : cap;
+        int nb = 1;
+        while (nb < nq) nb <<= 1;
+        int rs = 0, stages = 0;
+        uint32_t smem = 0;
+        if (!pick_ring(nb, head->d_pad, &rs, &stages, &smem))
+            return fail(VIE_ERR_UNSUPPORTED, "vie_head_topk: no shared-memory layout for d=%d",
+                        head->d);
+        vie::StreamTopkParams p;
+        p.W = head->W;
+        p.h = h + static_cast<int64_t>(q0) * head->d;
+        p.nq = nq;
+        p.V = head->V;
+        p.d = head->d;
+        p.d_pad = head->d_pad;
+        p.k = k;
+        p.rows_per_stage = rs;
+        p.stages = stages;
+        p.cand = head->cand;
+        p.ticket = head->words;
+        p.err = head->words + 1;
+        p.out_idx = out_idx + static_cast<int64_t>(q0) * k;
+        p.out_logits = out_logits + static_cast<int64_t>(q0) * k;
+        const cudaError_t e = vie::launch_stream_topk(nb, mm, p, head->G, smem, s);
+        if (e != cudaSuccess) return fail_cuda(e, "vie_head_topk launch");
+    }
+    return VIE_OK;
+}
+
+vie_status vie_scatter_sparse_logits(const int32_t *idx, const float *logits, int32_t batch,
+                                     int32_t k, int64_t V, float *out, vie_stream stream) {
+    if (idx == nullptr || logits == nullptr || out == nullptr)
+        return fail(VIE_ERR_INVALID_ARG, "vie_scatter_sparse_logits: NULL buffer");
+    if (batch < 1 || k < 1 || V < 1)
+        return fail(VIE_ERR_INVALID_ARG, "vie_scatter_sparse_logits: batch=%d k=%d V=%lld", batch,
+                    k, static_cast<long long>(V));
+    if (V > INT64_MAX / batch)
+        return fail(VIE_ERR_INVALID_ARG, "vie_scatter_sparse_logits: batch*V overflows");
+    if ((reinterpret_cast<uintptr_t>(idx) | reinterpret_cast<uintptr_t>(logits) |
+         reinterpret_cast<uintptr_t>(out)) & 3u)
+        return fail(VIE_ERR_INVALID_ARG, "vie_scatter_sparse_logits: buffers must be 4-byte aligned");
+    uint32_t *err = nullptr;
+    cudaError_t e = cudaGetSymbolAddress(reinterpret_cast<void **>(&err), g_dev_err);
+    if (e != cudaSuccess) return fail_cuda(e, "cudaGetSymbolAddress");
+    // ~16 KB of output per CTA, at most 1024 CTAs per row
+    int64_t per = 4096;
+    int64_t bx = (V + per - 1) / per;
+    if (bx > 1024) {
+        bx = 1024;
+        per = (V + bx - 1) / bx;
+        per = (per + 3) & ~static_cast<int64_t>(3);
+    }
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    for (int b0 = 0; b0 < batch; b0 += 65535) {
+        const int by = batch - b0 < 65535 ? batch - b0 : 65535;
+        scatter_sparse_kernel<<<dim3(static_cast<unsigned>(bx), by), 256, 0, s>>>(
+            idx, logits, k, V, per, out, b0, err);
+        e = cudaGetLastError();
+        if (e != cudaSuccess) return fail_cuda(e, "vie_scatter_sparse_logits launch");
+    }
+    return VIE_OK;
+}
+
+vie_status vie_device_status(vie_stream stream) {
+    cudaError_t e = cudaStreamSynchronize(static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return fail_cuda(e, "vie_device_status: stream synchronize");
+    uint32_t w = 0;
+    e = cudaMemcpyFromSymbol(&w, g_dev_err, sizeof w);
+    if (e != cudaSuccess) return fail_cuda(e, "vie_device_status: read flag");
+    if (w == 0) return VIE_OK;
+    const uint32_t zero = 0;
+    e = cudaMemcpyToSymbol(g_dev_err, &zero, sizeof zero);
+    if (e != cudaSuccess) return fail_cuda(e, "vie_device_status: clear flag");
+    return fail(VIE_ERR_DEVICE, "device flag 0x%x:%s%s", w,
+                (w & vie::kErrScatterIndex) ? " scatter index outside [0, V)" : "",
+                (w & vie::kErrWaitTimeout) ? " pipeline wait timed out" : "");
+}
+
+vie_status vie_head_device_status(vie_head *head, vie_stream stream) {
+    if (head == nullptr) return fail(VIE_ERR_INVALID_ARG, "vie_head_device_status: head is NULL");
+    vie_status st = check_device(head);
+    if (st != VIE_OK) return st;
+    st = vie_device_status(stream);
+    uint32_t words[2] = {0, 0};
+    cudaError_t e = cudaMemcpy(words, head->words, sizeof words, cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) return fail_cuda(e, "vie_head_device_status: read flag");
+    if (words[1] != 0) {
+        e = cudaMemset(head->words, 0, 2 * sizeof(uint32_t));
+        if (e != cudaSuccess) return fail_cuda(e, "vie_head_device_status: clear flag");
+        return fail(VIE_ERR_DEVICE, "handle device flag 0x%x:%s%s", words[1],
+                    (words[1] & vie::kErrWaitTimeout) ? " pipeline wait timed out" : "",
+                    (words[1] & vie::kErrScatterIndex) ? " scatter index outside [0, V)" : "");
+    }
+    return st;
+}
+
+}  // extern "C"
+
+namespace vie {
+cudaError_t launch_stream_topk(int nb, int mm, const StreamTopkParams &p, int grid,
+                               uint32_t smem, cudaStream_t stream) {
+    switch (nb) {
+        case 1: return launch_stream_topk_nb1(mm, p, grid, smem, stream);
+        case 2: return launch_stream_topk_nb2(mm, p, grid, smem, stream);
+        case 4: return launch_stream_topk_nb4(mm, p, grid, smem, stream);
+        case 8: return launch_stream_topk_nb8(mm, p, grid, smem, stream);
+        default: return cudaErrorInvalidValue;
+    }
+}
+}  // namespace vie

@@ -1,0 +1,43 @@
+// vie_stream_topk_inst.cuh - body shared by the per-width instantiation
+// units: sets the shared-memory opt-in once per device and launches.
+#pragma once
+
+#include "vie_launch.h"
+
+namespace vie {
+
+template <int NB, int MM>
+cudaError_t launch_one(const StreamTopkParams &p, int grid, uint32_t smem, cudaStream_t stream) {
+    constexpr int kR = 2;
+    static bool configured[64] = {};
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+    if (!configured[dev]) {
+        e = cudaFuncSetAttribute(stream_topk_kernel<NB, MM, kR>,
+                                 cudaFuncAttributeMaxDynamicSharedMemorySize, 232448);
+        if (e != cudaSuccess) return e;
+        configured[dev] = true;
+    }
+    stream_topk_kernel<NB, MM, kR><<<grid, kThreads, smem, stream>>>(p);
+    return cudaGetLastError();
+}
+
+template <int NB>
+cudaError_t launch_width(int mm, const StreamTopkParams &p, int grid, uint32_t smem,
+                         cudaStream_t stream) {
+    // Wide lists are only built for narrow query groups (register budget).
+    switch (mm) {
+        case 2: return launch_one<NB, 2>(p, grid, smem, stream);
+        case 8:
+            if constexpr (NB <= 4) return launch_one<NB, 8>(p, grid, smem, stream);
+            return cudaErrorInvalidValue;
+        case 32:
+            if constexpr (NB == 1) return launch_one<NB, 32>(p, grid, smem, stream);
+            return cudaErrorInvalidValue;
+        default: return cudaErrorInvalidValue;
+    }
+}
+
+}  // namespace vie

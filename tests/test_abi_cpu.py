@@ -1,0 +1,83 @@
+"""The C-ABI library builds, loads and exports every entry point that
+include/vie_head.h declares; host-side argument checks answer with status
+codes before any CUDA call (no GPU needed for these paths)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+import paper_2608_27460_gb300 as vie
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "vie_head.h")
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(vie_\w+)\s*\(", text)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    return vie.load()
+
+
+def test_header_declares_the_binding_exports():
+    assert declared_functions() == sorted(vie.EXPORTS)
+
+
+def test_library_exports_every_declared_symbol(lib):
+    for name in declared_functions():
+        assert hasattr(lib, name), name
+
+
+def test_header_is_plain_c():
+    import subprocess
+    src = '#include "vie_head.h"\nint main(void){vie_head_props p; (void)p; return VIE_OK;}\n'
+    r = subprocess.run(["gcc", "-std=c99", "-Wall", "-Werror", "-I", os.path.dirname(HEADER),
+                        "-x", "c", "-", "-fsyntax-only"], input=src, capture_output=True, text=True)
+    assert r.returncode == 0, r.stderr
+
+
+def test_create_rejects_bad_arguments_on_host(lib):
+    st, h = vie.vie_head_create(0, 10, 8)
+    assert st == vie.VIE_ERR_INVALID_ARG and h is None
+    assert "NULL" in vie.vie_last_error()
+    fake = 0x10000
+    assert vie.vie_head_create(fake, 0, 8)[0] == vie.VIE_ERR_INVALID_ARG
+    assert vie.vie_head_create(fake, 2 ** 31, 8)[0] == vie.VIE_ERR_INVALID_ARG
+    assert vie.vie_head_create(fake, 10, 0)[0] == vie.VIE_ERR_INVALID_ARG
+    assert vie.vie_head_create(fake, 10, vie.VIE_D_MAX + 1)[0] == vie.VIE_ERR_INVALID_ARG
+    assert vie.vie_head_create(fake, 10, 8, dtype=7)[0] == vie.VIE_ERR_UNSUPPORTED
+    assert vie.vie_head_create(fake + 1, 10, 8)[0] == vie.VIE_ERR_INVALID_ARG
+    out_null = lib.vie_head_create(fake, 10, 8, 0, None)
+    assert out_null == vie.VIE_ERR_INVALID_ARG
+
+
+def test_calls_on_null_handle_are_rejected(lib):
+    assert vie.vie_head_destroy(0) == vie.VIE_OK
+    assert vie.vie_head_topk(0, 16, 1, 1, 16, 16) == vie.VIE_ERR_INVALID_ARG
+    assert vie.vie_head_get_props(0)[0] == vie.VIE_ERR_INVALID_ARG
+    assert vie.vie_head_device_status(0) == vie.VIE_ERR_INVALID_ARG
+
+
+def test_scatter_rejects_bad_arguments_on_host(lib):
+    p = 0x10000
+    assert vie.vie_scatter_sparse_logits(0, p, 1, 1, 8, p) == vie.VIE_ERR_INVALID_ARG
+    assert vie.vie_scatter_sparse_logits(p, p, 0, 1, 8, p) == vie.VIE_ERR_INVALID_ARG
+    assert vie.vie_scatter_sparse_logits(p, p, 1, 0, 8, p) == vie.VIE_ERR_INVALID_ARG
+    assert vie.vie_scatter_sparse_logits(p, p, 1, 1, 0, p) == vie.VIE_ERR_INVALID_ARG
+    assert vie.vie_scatter_sparse_logits(p, p, 2, 1, 2 ** 62, p) == vie.VIE_ERR_INVALID_ARG
+    assert vie.vie_scatter_sparse_logits(p + 2, p, 1, 1, 8, p) == vie.VIE_ERR_INVALID_ARG
+
+
+def test_product_path_does_not_import_the_oracle():
+    pkg = os.path.join(ROOT, "paper_2608_27460_gb300")
+    for dirpath, _, files in os.walk(pkg):
+        for f in files:
+            if f.endswith((".py", ".cu", ".cuh", ".h")):
+                text = open(os.path.join(dirpath, f)).read()
+                assert not re.search(r"^\s*(import|from)\s+oracle\b", text, re.M), f
+                assert "oracle.c" not in text and "liboracle" not in text, f
