@@ -118,6 +118,19 @@ vie_status vie_head_topk(vie_head *head, const float *h, int32_t batch, int32_t 
                          int32_t *out_idx, float *out_logits, vie_stream stream);
 
 /*
+ * vie_head_topk_sparse - vie_head_topk and the sparse full-vocabulary logit
+ * tensor of Section 3 in one launch: besides out_idx / out_logits it writes
+ *   out_sparse  device, fp32 [batch, V] (4-byte aligned): -inf (0xFF800000)
+ *               everywhere except out_sparse[b, out_idx[b, j]] =
+ *               out_logits[b, j] (the same bits).
+ * The result equals vie_head_topk followed by vie_scatter_sparse_logits on
+ * its outputs.  Same limits, sharing rule and errors as vie_head_topk.
+ */
+vie_status vie_head_topk_sparse(vie_head *head, const float *h, int32_t batch, int32_t k,
+                                int32_t *out_idx, float *out_logits, float *out_sparse,
+                                vie_stream stream);
+
+/*
  * vie_scatter_sparse_logits - the sparse full-vocabulary logit tensor of
  * Section 3: out[b, v] = -inf (bit pattern 0xFF800000) for every v, then
  * out[b, idx[b, j]] = logits[b, j] for j < k (values copied bit for bit).

@@ -36,7 +36,7 @@ STATUS_NAMES = {0: "VIE_OK", 1: "VIE_ERR_INVALID_ARG", 2: "VIE_ERR_UNSUPPORTED",
 
 # Every entry point of include/vie_head.h.
 EXPORTS = ("vie_head_create", "vie_head_destroy", "vie_head_get_props", "vie_head_topk",
-           "vie_scatter_sparse_logits", "vie_device_status", "vie_head_device_status",
+           "vie_head_topk_sparse", "vie_scatter_sparse_logits", "vie_device_status", "vie_head_device_status",
            "vie_last_error")
 
 
@@ -79,6 +79,7 @@ def load(path: str | None = None, build_if_missing: bool = True):
             "vie_head_destroy": ([P], ctypes.c_int),
             "vie_head_get_props": ([P, ctypes.POINTER(vie_head_props)], ctypes.c_int),
             "vie_head_topk": ([P, P, I32, I32, P, P, P], ctypes.c_int),
+            "vie_head_topk_sparse": ([P, P, I32, I32, P, P, P, P], ctypes.c_int),
             "vie_scatter_sparse_logits": ([P, P, I32, I32, I64, P, P], ctypes.c_int),
             "vie_device_status": ([P], ctypes.c_int),
             "vie_head_device_status": ([P, P], ctypes.c_int),
@@ -120,6 +121,11 @@ def vie_head_get_props(head: int):
 def vie_head_topk(head: int, h: int, batch: int, k: int, out_idx: int, out_logits: int,
                   stream: int = 0) -> int:
     return load().vie_head_topk(head, h, batch, k, out_idx, out_logits, stream)
+
+
+def vie_head_topk_sparse(head: int, h: int, batch: int, k: int, out_idx: int, out_logits: int,
+                         out_sparse: int, stream: int = 0) -> int:
+    return load().vie_head_topk_sparse(head, h, batch, k, out_idx, out_logits, out_sparse, stream)
 
 
 def vie_scatter_sparse_logits(idx: int, logits: int, batch: int, k: int, V: int, out: int,
@@ -194,6 +200,25 @@ class Head:
         check(vie_head_topk(self.handle, h.data_ptr(), b, k, out_idx.data_ptr(),
                             out_logits.data_ptr(), _stream_ptr(stream)))
         return out_idx, out_logits
+
+    def topk_sparse(self, h, k: int, out_idx=None, out_logits=None, out_sparse=None, stream=None):
+        """Top-k and the sparse [batch, V] logit tensor in one launch."""
+        import torch
+        if h.dim() == 1:
+            h = h[None]
+        if h.dtype != torch.float32 or not h.is_cuda or h.shape[1] != self.d:
+            raise ValueError(f"h must be a CUDA float32 tensor [batch, {self.d}]")
+        h = h.contiguous()
+        b = int(h.shape[0])
+        if out_idx is None:
+            out_idx = torch.empty((b, k), dtype=torch.int32, device=h.device)
+        if out_logits is None:
+            out_logits = torch.empty((b, k), dtype=torch.float32, device=h.device)
+        if out_sparse is None:
+            out_sparse = torch.empty((b, self.V), dtype=torch.float32, device=h.device)
+        check(vie_head_topk_sparse(self.handle, h.data_ptr(), b, k, out_idx.data_ptr(),
+                                   out_logits.data_ptr(), out_sparse.data_ptr(), _stream_ptr(stream)))
+        return out_idx, out_logits, out_sparse
 
     def sparse_logits(self, idx, logits, out=None, stream=None):
         """Sparse [batch, V] fp32 tensor: -inf except logits at idx."""

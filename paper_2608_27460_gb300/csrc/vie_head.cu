@@ -7,6 +7,7 @@
 #include <cstdarg>
 #include <cstdint>
 #include <cstdio>
+#include <cstdlib>
 #include <cstring>
 #include <new>
 
@@ -47,7 +48,7 @@ struct vie_head {
     int G;
     uint16_t *W;        // [V, d_pad] bf16 bits
     uint64_t *cand;     // [kMaxNB][G][VIE_K_MAX] ranking keys
-    uint32_t *words;    // [0] completion ticket, [1] device flag word
+    uint32_t *words;    // [0] completion ticket, [1] device flag word, [2] chunk pool counter
     int64_t scratch_bytes;
 };
 
@@ -129,24 +130,44 @@ int nb_cap_for(int d_pad, int mm) {
     return nb;
 }
 
-// Stage rows and ring depth for one launch shape: aim for ~32 KB stages and
-// the deepest ring that fits in shared memory.
-bool pick_ring(int nb, int d_pad, int *rs_out, int *stages_out, uint32_t *smem_out) {
+int env_int(const char *name, int dflt) {
+    const char *v = getenv(name);
+    return (v != nullptr && *v != 0) ? atoi(v) : dflt;
+}
+
+// Launch-shape knobs (they change speed, never results):
+//   VIE_STAGE_MIN_KB     smallest weight stage worth one bulk copy (48)
+//   VIE_STATIC_PCT       share of the chunks assigned statically, in % (85)
+struct Knobs {
+    int stage_min_bytes, static_pct;
+};
+const Knobs &knobs() {
+    static const Knobs k = {env_int("VIE_STAGE_MIN_KB", 48) * 1024, env_int("VIE_STATIC_PCT", 85)};
+    return k;
+}
+
+struct LaunchShape {
+    int r, rs, stages;
+    uint32_t smem;
+};
+
+// Rows per warp per stage (R), stage rows (8*R, fewer for very wide rows),
+// and ring depth (deepest that fits) for one launch.
+bool pick_shape(int nb, int d_pad, LaunchShape *out) {
     const int row_bytes = d_pad * 2;
-    int rs = 32768 / row_bytes;
-    if (rs < 1) rs = 1;
-    if (rs > 32) rs = 32;
-    for (; rs >= 1; rs = (rs > 1 ? rs / 2 : 0)) {
+    int r = 1;
+    while (r < 4 && 8 * r * row_bytes < knobs().stage_min_bytes) r <<= 1;
+    for (int rs = 8 * r; rs >= 1; --rs) {
         for (int s = vie::kMaxStages; s >= 2; --s) {
             const vie::SmemLayout L(nb, d_pad, rs, s, row_bytes);
             if (L.total <= static_cast<uint32_t>(kMaxSmem)) {
-                *rs_out = rs;
-                *stages_out = s;
-                *smem_out = L.total;
+                out->r = r;
+                out->rs = rs;
+                out->stages = s;
+                out->smem = L.total;
                 return true;
             }
         }
-        if (rs == 1) break;
     }
     return false;
 }
@@ -214,11 +235,11 @@ vie_status vie_head_create(const void *W_out, int64_t V, int32_t d, vie_dtype dt
 
     const size_t wbytes = static_cast<size_t>(V) * hd->d_pad * 2;
     const size_t cbytes = static_cast<size_t>(kMaxNB) * hd->G * VIE_K_MAX * sizeof(uint64_t);
-    hd->scratch_bytes = static_cast<int64_t>(cbytes + 2 * sizeof(uint32_t));
+    hd->scratch_bytes = static_cast<int64_t>(cbytes + 4 * sizeof(uint32_t));
     e = cudaMalloc(&hd->W, wbytes);
     if (e == cudaSuccess) e = cudaMalloc(&hd->cand, cbytes);
-    if (e == cudaSuccess) e = cudaMalloc(&hd->words, 2 * sizeof(uint32_t));
-    if (e == cudaSuccess) e = cudaMemset(hd->words, 0, 2 * sizeof(uint32_t));
+    if (e == cudaSuccess) e = cudaMalloc(&hd->words, 4 * sizeof(uint32_t));
+    if (e == cudaSuccess) e = cudaMemset(hd->words, 0, 4 * sizeof(uint32_t));
     if (e == cudaSuccess) {
         const int64_t chunks = V * (hd->d_pad >> 3);
         int64_t blocks = (chunks + 255) / 256;
@@ -262,20 +283,20 @@ vie_status vie_head_get_props(const vie_head *head, vie_head_props *props) {
     return VIE_OK;
 }
 
-vie_status vie_head_topk(vie_head *head, const float *h, int32_t batch, int32_t k,
-                         int32_t *out_idx, float *out_logits, vie_stream stream) {
-    if (head == nullptr) return fail(VIE_ERR_INVALID_ARG, "vie_head_topk: head is NULL");
+static vie_status run_topk(const char *fn, vie_head *head, const float *h, int32_t batch,
+                           int32_t k, int32_t *out_idx, float *out_logits, float *sparse,
+                           vie_stream stream) {
+    if (head == nullptr) return fail(VIE_ERR_INVALID_ARG, "%s: head is NULL", fn);
     if (h == nullptr || out_idx == nullptr || out_logits == nullptr)
-        return fail(VIE_ERR_INVALID_ARG, "vie_head_topk: NULL buffer");
+        return fail(VIE_ERR_INVALID_ARG, "%s: NULL buffer", fn);
     if (batch < 1 || batch > VIE_BATCH_MAX)
-        return fail(VIE_ERR_INVALID_ARG, "vie_head_topk: batch=%d outside [1, %d]", batch,
-                    VIE_BATCH_MAX);
+        return fail(VIE_ERR_INVALID_ARG, "%s: batch=%d outside [1, %d]", fn, batch, VIE_BATCH_MAX);
     if (k < 1 || k > VIE_K_MAX || static_cast<int64_t>(k) > head->V)
-        return fail(VIE_ERR_INVALID_ARG, "vie_head_topk: k=%d outside [1, min(V=%lld, %d)]", k,
+        return fail(VIE_ERR_INVALID_ARG, "%s: k=%d outside [1, min(V=%lld, %d)]", fn, k,
                     static_cast<long long>(head->V), VIE_K_MAX);
     if ((reinterpret_cast<uintptr_t>(h) | reinterpret_cast<uintptr_t>(out_idx) |
-         reinterpret_cast<uintptr_t>(out_logits)) & 3u)
-        return fail(VIE_ERR_INVALID_ARG, "vie_head_topk: buffers must be 4-byte aligned");
+         reinterpret_cast<uintptr_t>(out_logits) | reinterpret_cast<uintptr_t>(sparse)) & 3u)
+        return fail(VIE_ERR_INVALID_ARG, "%s: buffers must be 4-byte aligned", fn);
     vie_status st = check_device(head);
     if (st != VIE_OK) return st;
 
@@ -286,11 +307,9 @@ vie_status vie_head_topk(vie_head *head, const float *h, int32_t batch, int32_t 
         const int nq = batch - q0 < cap ? batch - q0 : cap;
         int nb = 1;
         while (nb < nq) nb <<= 1;
-        int rs = 0, stages = 0;
-        uint32_t smem = 0;
-        if (!pick_ring(nb, head->d_pad, &rs, &stages, &smem))
-            return fail(VIE_ERR_UNSUPPORTED, "vie_head_topk: no shared-memory layout for d=%d",
-                        head->d);
+        LaunchShape shp;
+        if (!pick_shape(nb, head->d_pad, &shp))
+            return fail(VIE_ERR_UNSUPPORTED, "%s: no shared-memory layout for d=%d", fn, head->d);
         vie::StreamTopkParams p;
         p.W = head->W;
         p.h = h + static_cast<int64_t>(q0) * head->d;
@@ -299,17 +318,37 @@ vie_status vie_head_topk(vie_head *head, const float *h, int32_t batch, int32_t 
         p.d = head->d;
         p.d_pad = head->d_pad;
         p.k = k;
-        p.rows_per_stage = rs;
-        p.stages = stages;
+        p.rows_per_stage = shp.rs;
+        p.stages = shp.stages;
+        const int64_t n_chunks = (head->V + shp.rs - 1) / shp.rs;
+        int pct = knobs().static_pct;
+        pct = pct < 0 ? 0 : (pct > 100 ? 100 : pct);
+        p.static_chunks = static_cast<int32_t>(n_chunks * pct / 100 / head->G);
         p.cand = head->cand;
         p.ticket = head->words;
         p.err = head->words + 1;
+        p.next_chunk = head->words + 2;
         p.out_idx = out_idx + static_cast<int64_t>(q0) * k;
         p.out_logits = out_logits + static_cast<int64_t>(q0) * k;
-        const cudaError_t e = vie::launch_stream_topk(nb, mm, p, head->G, smem, s);
-        if (e != cudaSuccess) return fail_cuda(e, "vie_head_topk launch");
+        p.sparse = sparse != nullptr ? sparse + static_cast<int64_t>(q0) * head->V : nullptr;
+        const cudaError_t e = vie::launch_stream_topk(nb, mm, shp.r, p, head->G, shp.smem, s);
+        if (e != cudaSuccess) return fail_cuda(e, fn);
     }
     return VIE_OK;
+}
+
+vie_status vie_head_topk(vie_head *head, const float *h, int32_t batch, int32_t k,
+                         int32_t *out_idx, float *out_logits, vie_stream stream) {
+    return run_topk("vie_head_topk", head, h, batch, k, out_idx, out_logits, nullptr, stream);
+}
+
+vie_status vie_head_topk_sparse(vie_head *head, const float *h, int32_t batch, int32_t k,
+                                int32_t *out_idx, float *out_logits, float *out_sparse,
+                                vie_stream stream) {
+    if (out_sparse == nullptr)
+        return fail(VIE_ERR_INVALID_ARG, "vie_head_topk_sparse: out_sparse is NULL");
+    return run_topk("vie_head_topk_sparse", head, h, batch, k, out_idx, out_logits, out_sparse,
+                    stream);
 }
 
 vie_status vie_scatter_sparse_logits(const int32_t *idx, const float *logits, int32_t batch,
@@ -370,7 +409,7 @@ vie_status vie_head_device_status(vie_head *head, vie_stream stream) {
     cudaError_t e = cudaMemcpy(words, head->words, sizeof words, cudaMemcpyDeviceToHost);
     if (e != cudaSuccess) return fail_cuda(e, "vie_head_device_status: read flag");
     if (words[1] != 0) {
-        e = cudaMemset(head->words, 0, 2 * sizeof(uint32_t));
+        e = cudaMemset(head->words, 0, 4 * sizeof(uint32_t));
         if (e != cudaSuccess) return fail_cuda(e, "vie_head_device_status: clear flag");
         return fail(VIE_ERR_DEVICE, "handle device flag 0x%x:%s%s", words[1],
                     (words[1] & vie::kErrWaitTimeout) ? " pipeline wait timed out" : "",
@@ -382,13 +421,13 @@ vie_status vie_head_device_status(vie_head *head, vie_stream stream) {
 }  // extern "C"
 
 namespace vie {
-cudaError_t launch_stream_topk(int nb, int mm, const StreamTopkParams &p, int grid,
+cudaError_t launch_stream_topk(int nb, int mm, int r, const StreamTopkParams &p, int grid,
                                uint32_t smem, cudaStream_t stream) {
     switch (nb) {
-        case 1: return launch_stream_topk_nb1(mm, p, grid, smem, stream);
-        case 2: return launch_stream_topk_nb2(mm, p, grid, smem, stream);
-        case 4: return launch_stream_topk_nb4(mm, p, grid, smem, stream);
-        case 8: return launch_stream_topk_nb8(mm, p, grid, smem, stream);
+        case 1: return launch_stream_topk_nb1(mm, r, p, grid, smem, stream);
+        case 2: return launch_stream_topk_nb2(mm, r, p, grid, smem, stream);
+        case 4: return launch_stream_topk_nb4(mm, r, p, grid, smem, stream);
+        case 8: return launch_stream_topk_nb8(mm, r, p, grid, smem, stream);
         default: return cudaErrorInvalidValue;
     }
 }

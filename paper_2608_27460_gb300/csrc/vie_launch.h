@@ -8,19 +8,19 @@
 
 namespace vie {
 
-// Launches stream_topk_kernel<nb, mm, R> on `grid` CTAs; nb in {1,2,4,8},
-// mm in {2,8,32}.  Returns the launch error (cudaErrorInvalidValue for an
-// unsupported nb/mm pair).
-cudaError_t launch_stream_topk(int nb, int mm, const StreamTopkParams &p, int grid,
+// Launches stream_topk_kernel<nb, mm, r> on `grid` CTAs; nb in {1,2,4,8},
+// mm in {2,8,32}, r in {1,2,4}.  Returns the launch error
+// (cudaErrorInvalidValue for an unsupported combination).
+cudaError_t launch_stream_topk(int nb, int mm, int r, const StreamTopkParams &p, int grid,
                                uint32_t smem, cudaStream_t stream);
 
-cudaError_t launch_stream_topk_nb1(int mm, const StreamTopkParams &p, int grid, uint32_t smem,
-                                   cudaStream_t stream);
-cudaError_t launch_stream_topk_nb2(int mm, const StreamTopkParams &p, int grid, uint32_t smem,
-                                   cudaStream_t stream);
-cudaError_t launch_stream_topk_nb4(int mm, const StreamTopkParams &p, int grid, uint32_t smem,
-                                   cudaStream_t stream);
-cudaError_t launch_stream_topk_nb8(int mm, const StreamTopkParams &p, int grid, uint32_t smem,
-                                   cudaStream_t stream);
+cudaError_t launch_stream_topk_nb1(int mm, int r, const StreamTopkParams &p, int grid,
+                                   uint32_t smem, cudaStream_t stream);
+cudaError_t launch_stream_topk_nb2(int mm, int r, const StreamTopkParams &p, int grid,
+                                   uint32_t smem, cudaStream_t stream);
+cudaError_t launch_stream_topk_nb4(int mm, int r, const StreamTopkParams &p, int grid,
+                                   uint32_t smem, cudaStream_t stream);
+cudaError_t launch_stream_topk_nb8(int mm, int r, const StreamTopkParams &p, int grid,
+                                   uint32_t smem, cudaStream_t stream);
 
 }  // namespace vie

@@ -1,26 +1,39 @@
 // vie_stream_topk.cuh - the small-batch output head in one launch:
 // streaming projection z = W_out h (paper, Section 3) fused with the exact
-// top-k selection (exhaustive MIPS, Sections 2-3).
+// top-k selection (exhaustive MIPS, Sections 2-3) and, optionally, the
+// sparse -inf logit tensor (Section 3).
 //
-// One persistent CTA per SM owns a contiguous slice of the vocabulary rows.
-//   warp 0     producer: 1-D bulk copies (TMA) of whole row groups into a
-//              ring of shared-memory stages, L2 evict-first, mbarrier
-//              transaction counts;
-//   warps 2-9  projection: each warp takes rows of a stage, every lane a
-//              strided set of 16-byte column chunks; bf16 -> fp32 widening,
-//              fp32 FMA against h (staged in shared memory, one load per
-//              chunk reused for R rows), then a warp-shuffle butterfly sum;
+// One persistent CTA per SM.  The vocabulary is cut into chunks of RS rows
+// (one weight stage each).  The first G * Ns chunks are dealt round robin
+// (chunk c to CTA c mod G, so the CTAs sweep W together and keep every HBM
+// channel busy); the rest form a pool that CTAs draw from in order with an
+// atomic counter once their own chunks are done, so all CTAs finish together.
+//   warp 0     producer: 1-D bulk copies (TMA) of chunks into a ring of
+//              shared-memory stages (mbarrier transaction counts, L2
+//              evict-first); the chunk id travels with the stage; an id of
+//              -1 closes the stream;
+//   warps 2-9  projection: warp w owns rows w, w+8, .. (at most R) of each
+//              stage and every lane a strided set of 16-byte column chunks;
+//              bf16 -> fp32 widening, fp32 FMA against h (staged in shared
+//              memory, one load per chunk reused for the warp's rows).  The
+//              stage is released as soon as its last shared-memory read
+//              retires; the warp-shuffle sums then go to a separate, deeper
+//              score ring;
 //   warp 1     selector: keeps the best keys seen so far as a sorted list
 //              spread over the warp's registers; a row enters only if it
-//              beats the current k-th key.
-// The full logit vector never leaves the chip.  After the stream, each CTA
-// writes its sorted top-k list to scratch and takes a ticket; the CTA that
-// draws the last ticket merges the G lists into the final top-k:
+//              beats the current k-th key.  It never holds a weight stage.
+// The full logit vector never leaves the chip.  Afterwards each CTA writes
+// its sorted top-k list to scratch and takes a ticket (an acq_rel atomic, no
+// full fences); the CTA that draws the last ticket copies every list into
+// shared memory in one pass (when they fit) and merges them:
 //   1. tau* = k-th largest key among the first J = ceil(k/G) entries of all
 //      lists (a lower bound of the true k-th key: k keys are >= it);
 //   2. every list contributes its prefix of keys >= tau*;
 //   3. exact top-k of those candidates (rank counting, or radix select when
 //      there are many), written best first.
+// With a sparse output, every CTA first fills a fixed slice of each output
+// row with -inf; the merging CTA writes the k logits after the last ticket,
+// so each fill happens before the value at the same position.
 #pragma once
 
 #include <cstdint>
@@ -31,11 +44,14 @@ namespace vie {
 
 constexpr int kDotWarps = 8;
 constexpr int kThreads = 32 * (2 + kDotWarps);
-constexpr int kMaxStages = 16;
+constexpr int kMaxStages = 16;         // weight ring depth limit
+constexpr int kScoreStages = 16;       // score ring depth
 constexpr int kMergePrefixCap = 2048;  // keys: first-J prefixes of all lists
 constexpr int kMergeCandCap = 2048;    // keys: gathered candidates
 constexpr int kRankCountMax = 640;     // rank counting below this many keys
 constexpr int kMaxLists = 1024;        // G <= 1024 CTAs
+constexpr int kFastE = 4;              // fast merge: entries read per list
+constexpr int kFastMaxK = 64;          // fast merge: largest k
 
 struct StreamTopkParams {
     const uint16_t *W;   // padded [V, d_pad] bf16 bits
@@ -44,13 +60,16 @@ struct StreamTopkParams {
     int64_t V;
     int32_t d, d_pad;
     int32_t k;
-    int32_t rows_per_stage;  // RS
-    int32_t stages;          // S
+    int32_t rows_per_stage;  // RS <= 8 * R: rows of one chunk / weight stage
+    int32_t stages;          // S, weight ring depth
+    int32_t static_chunks;   // chunks each CTA owns before drawing from the pool
     uint64_t *cand;          // [NB][G][k] keys
     uint32_t *ticket;        // CTA completion counter (self-resetting)
+    uint32_t *next_chunk;    // pool counter (self-resetting)
     uint32_t *err;           // device flag word
     int32_t *out_idx;        // [nq, k]
     float *out_logits;       // [nq, k]
+    float *sparse;           // [nq, V] fp32 or nullptr
 };
 
 // Shared-memory carve-up; all offsets are multiples of 128 bytes.
@@ -59,15 +78,17 @@ struct SmemLayout {
     __host__ __device__ static uint32_t align128(uint32_t x) { return (x + 127u) & ~127u; }
     __host__ __device__ SmemLayout(int nb, int d_pad, int rs, int stages, int row_bytes) {
         bars = 0;
-        misc = align128(bars + 3u * kMaxStages * 8u);
-        h = align128(misc + 128u);
+        misc = align128(bars + 8u * (2 * kMaxStages + 2 * kScoreStages));
+        h = align128(misc + 256u);
         scores = align128(h + 4u * nb * d_pad);
-        ring = align128(scores + 4u * stages * rs * nb);
+        ring = align128(scores + 4u * kScoreStages * rs * nb);
         merge = ring;  // the merge reuses the ring once the stream is drained
         uint32_t ring_end = ring + static_cast<uint32_t>(stages) * rs * row_bytes;
-        uint32_t merge_end = merge + 8u * (kMergePrefixCap + kMergeCandCap + 1024) +
-                             4u * (2 * kMaxLists + 256 + 32);
+        uint32_t merge_end = merge + merge_fixed_bytes();
         total = ring_end > merge_end ? ring_end : merge_end;
+    }
+    __host__ __device__ static uint32_t merge_fixed_bytes() {
+        return 8u * (kMergePrefixCap + kMergeCandCap + 1024) + 4u * (2 * kMaxLists + 256 + 32);
     }
 };
 
@@ -80,7 +101,23 @@ struct MiscSmem {
     int n_win;
     unsigned long long tau;
     unsigned long long prefix;
+    unsigned int tau_v;
+    int overflow;
+    int chunk_w[kMaxStages];     // chunk id of each weight stage (-1: end)
+    int chunk_s[kScoreStages];   // chunk id of each score stage (-1: end)
 };
+
+__device__ __forceinline__ uint32_t atomic_add_acq_rel_gpu(uint32_t *p, uint32_t v) {
+    uint32_t old;
+    asm volatile("atom.add.acq_rel.gpu.u32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
+    return old;
+}
+
+__device__ __forceinline__ uint32_t atomic_add_relaxed_gpu(uint32_t *p, uint32_t v) {
+    uint32_t old;
+    asm volatile("atom.add.relaxed.gpu.u32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
+    return old;
+}
 
 // --------------------------------------------------------------------------
 // Warp-distributed sorted list of the best keys (descending).  Lane L holds
@@ -194,12 +231,30 @@ __device__ uint64_t block_radix_threshold(Keys keys, int n, int k, uint64_t lo, 
     return prefix;
 }
 
+// Number of keys in keys[0..n) (shared memory, 16-byte aligned) above x.
+// Every thread of a warp reads the same address, so each load is a broadcast;
+// two keys per load and an unrolled loop keep many loads in flight.
+__device__ __forceinline__ int rank_among(const uint64_t *keys, int n, uint64_t x) {
+    const ulonglong2 *k2 = reinterpret_cast<const ulonglong2 *>(keys);
+    const int n2 = n >> 1;
+    int r0 = 0, r1 = 0;
+#pragma unroll 8
+    for (int j = 0; j < n2; ++j) {
+        const ulonglong2 v = k2[j];
+        r0 += (v.x > x) ? 1 : 0;
+        r1 += (v.y > x) ? 1 : 0;
+    }
+    if (n & 1) r0 += (keys[n - 1] > x) ? 1 : 0;
+    return r0 + r1;
+}
+
 // Exact top-k of n unique nonzero keys in shared memory, written best first
-// to out_idx / out_logits.  Uses rank counting for small n, otherwise a
-// radix-select threshold followed by rank counting of the k winners.
+// to out_idx / out_logits (and into the sparse row, if any).  Rank counting
+// for small n, otherwise a radix-select threshold and rank counting of the
+// k winners.
 __device__ inline void block_topk_to_output(const uint64_t *keys, int n, int k, uint64_t *win,
-                                     uint32_t *hist, MiscSmem *ms, int32_t *out_idx,
-                                     float *out_logits) {
+                                            uint32_t *hist, MiscSmem *ms, int32_t *out_idx,
+                                            float *out_logits, float *sparse_row) {
     const int tid = threadIdx.x;
     const uint64_t *src = keys;
     int m = n;
@@ -217,27 +272,221 @@ __device__ inline void block_topk_to_output(const uint64_t *keys, int n, int k, 
     }
     for (int i = tid; i < m; i += kThreads) {
         const uint64_t x = src[i];
-        int rank = 0;
-        for (int j = 0; j < m; ++j) rank += (src[j] > x) ? 1 : 0;
+        const int rank = rank_among(src, m, x);
         if (rank < k) {
             out_idx[rank] = key_index(x);
             out_logits[rank] = key_value(x);
+            if (sparse_row != nullptr) sparse_row[key_index(x)] = key_value(x);
         }
     }
     __syncthreads();
+}
+
+// Shared-memory buffers of the merge.
+struct MergeBufs {
+    uint64_t *pref, *cands, *win;
+    int *counts, *offsets;
+    uint32_t *hist;
+};
+
+// Merges the G sorted lists of one query (G x k keys, `lists`) into the
+// exact top-k.  Keys = SmemKeys when the lists were staged in shared memory.
+template <class Keys>
+__device__ void merge_lists(Keys lists, int G, int k, const MergeBufs &mb, MiscSmem *ms,
+                            int32_t *oi, float *ol, float *sp) {
+    const int tid = threadIdx.x;
+    const int J = (k + G - 1) / G;
+    const int P = G * J;
+
+    // 1. tau*: k-th largest among the first J entries of every list
+    uint64_t tau = 0;
+    const bool have_pref = P <= kMergePrefixCap;
+    if (have_pref) {
+        for (int i = tid; i < P; i += kThreads) {
+            const int c = i / J, j = i - c * J;
+            mb.pref[i] = lists[c * k + j];
+        }
+        if (tid == 0) ms->tau = 0;
+        __syncthreads();
+        if (P <= kRankCountMax) {
+            for (int i = tid; i < P; i += kThreads) {
+                const uint64_t x = mb.pref[i];
+                if (x != 0 && rank_among(mb.pref, P, x) == k - 1) ms->tau = x;
+            }
+            __syncthreads();
+            tau = ms->tau;
+        } else {
+            int nz = 0;  // nonzero keys among the prefixes
+            for (int i = 0; i < P; ++i) nz += mb.pref[i] != 0;
+            tau = (nz >= k) ? block_radix_threshold(SmemKeys{mb.pref}, P, k, 1, mb.hist, ms) : 0;
+        }
+    }
+    // 2. per-list count of keys >= tau* (lists are sorted descending); the
+    //    first J entries are in the prefix buffer, deeper entries are read
+    //    eight at a time with independent loads.
+    const uint64_t lo = tau > 0 ? tau : 1;
+    for (int c = tid; c < G; c += kThreads) {
+        int n = 0;
+        if (have_pref)
+            while (n < J && mb.pref[c * J + n] >= lo) ++n;
+        if (!have_pref || n == J) {
+            for (int b = n; b < k && n == b; b += 8) {
+                uint64_t e[8];
+#pragma unroll
+                for (int q = 0; q < 8; ++q) e[q] = (b + q < k) ? lists[c * k + b + q] : 0;
+#pragma unroll
+                for (int q = 0; q < 8; ++q)
+                    if (n == b + q && b + q < k && e[q] >= lo) ++n;
+            }
+        }
+        mb.counts[c] = n;
+    }
+    __syncthreads();
+    if (tid < 32) {
+        // exclusive scan of counts[0..G) by one warp, a run of lists per lane
+        const int per = (G + 31) / 32;
+        const int b0 = tid * per;
+        int local = 0;
+        for (int c = b0; c < min(G, b0 + per); ++c) local += mb.counts[c];
+        int incl = local;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int t2 = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+            if (tid >= o) incl += t2;
+        }
+        int run = incl - local;
+        for (int c = b0; c < min(G, b0 + per); ++c) {
+            mb.offsets[c] = run;
+            run += mb.counts[c];
+        }
+        if (tid == 31) ms->n_cand = incl;
+    }
+    __syncthreads();
+    const int M = ms->n_cand;
+    if (M <= kMergeCandCap) {
+        // 3a. gather the candidates, exact top-k among them
+        for (int c = tid; c < G; c += kThreads)
+            for (int j = 0; j < mb.counts[c]; ++j)
+                mb.cands[mb.offsets[c] + j] =
+                    (have_pref && j < J) ? mb.pref[c * J + j] : lists[c * k + j];
+        __syncthreads();
+        block_topk_to_output(mb.cands, M, k, mb.win, mb.hist, ms, oi, ol, sp);
+    } else {
+        // 3b. too many candidates: radix-select the threshold over all lists
+        const uint64_t T = block_radix_threshold(lists, G * k, k, lo, mb.hist, ms);
+        if (tid == 0) ms->n_win = 0;
+        __syncthreads();
+        for (int i = tid; i < G * k; i += kThreads) {
+            const uint64_t x = lists[i];
+            if (x >= T && x >= lo) mb.win[atomicAdd(&ms->n_win, 1)] = x;
+        }
+        __syncthreads();
+        block_topk_to_output(mb.win, k, k, mb.win, mb.hist, ms, oi, ol, sp);
+    }
+}
+
+// Latency-lean merge of one query for small k, spread over every warp of
+// the CTA.  fe = the first kFastE keys of each of the G sorted lists, hv =
+// their heads' value bits (padded with 0 to a multiple of 8).  tau = the
+// k-th largest head value counted with multiplicity: at least k keys are
+// >= (tau << 32), so every top-k key is too, and each list contributes its
+// prefix of keys above that bound.  Returns false (writing nothing) if some
+// list might hold more than kFastE such keys or fewer than k heads are
+// real; the caller then merges in full.  Requires 2 * G <= kThreads.
+__device__ inline bool merge_fast_query(const uint64_t *fe, const uint32_t *hv, int G, int k,
+                                        uint64_t *cands, int *rank_part, MiscSmem *ms, int32_t *oi,
+                                        float *ol, float *sp) {
+    const int tid = threadIdx.x, lane = tid & 31;
+    const int G8 = (G + 7) & ~7;
+    if (tid == 0) {
+        ms->tau_v = 0;
+        ms->n_cand = 0;
+        ms->overflow = 0;
+    }
+    for (int i = tid; i < kFastE * kThreads / 2; i += kThreads) rank_part[i] = 0;  // M <= G * kFastE
+    __syncthreads();
+    // tau: thread pair (2c, 2c+1) counts the heads >= head c, half each
+    {
+        const int c = tid >> 1, half = tid & 1;
+        const bool real = c < G && fe[c * kFastE] != 0;
+        const uint32_t v = c < G ? hv[c] : 0xFFFFFFFFu;
+        const uint4 *h4 = reinterpret_cast<const uint4 *>(hv) + half * (G8 / 8);
+        int ge = 0;
+#pragma unroll 4
+        for (int j = 0; j < G8 / 8; ++j) {
+            const uint4 q = h4[j];
+            ge += (q.x >= v) + (q.y >= v) + (q.z >= v) + (q.w >= v);
+        }
+        ge += __shfl_xor_sync(0xFFFFFFFFu, ge, 1);
+        uint32_t best = (real && ge >= k) ? v : 0u;
+        best = __reduce_max_sync(0xFFFFFFFFu, best);
+        if (lane == 0 && best != 0) atomicMax(&ms->tau_v, best);
+    }
+    __syncthreads();
+    const uint32_t tv = ms->tau_v;
+    if (tv == 0) return false;  // uniform: fewer than k real heads
+    const uint64_t lo = static_cast<uint64_t>(tv) << 32;
+    const int En = k < kFastE ? k : kFastE;
+    // gather: list c's keys >= lo, slots taken per warp
+    {
+        const int c = tid;
+        int n = 0;
+        if (c < G)
+            while (n < En && fe[c * kFastE + n] >= lo) ++n;
+        if (n == En && k > En) ms->overflow = 1;
+        int incl = n;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int t = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+            if (lane >= o) incl += t;
+        }
+        int base = 0;
+        if (lane == 31 && incl > 0) base = atomicAdd(&ms->n_cand, incl);
+        base = __shfl_sync(0xFFFFFFFFu, base, 31);
+        for (int j = 0; j < n; ++j) cands[base + incl - n + j] = fe[c * kFastE + j];
+    }
+    __syncthreads();
+    if (ms->overflow) return false;
+    const int M = ms->n_cand;
+    // rank: candidate i is counted by up to kRankSplit threads, each over a
+    // slice of the candidates; partial counts meet in shared memory
+    constexpr int kRankSplit = 5;
+    const int per = (M + kRankSplit - 1) / kRankSplit;
+    for (int t = tid; t < M * kRankSplit; t += kThreads) {
+        const int i = t % M, part = t / M;
+        const uint64_t x = cands[i];
+        const int j0 = part * per, j1 = min(M, j0 + per);
+        int r = 0;
+#pragma unroll 4
+        for (int j = j0; j < j1; ++j) r += (cands[j] > x) ? 1 : 0;
+        if (r) atomicAdd(&rank_part[i], r);
+    }
+    __syncthreads();
+    for (int i = tid; i < M; i += kThreads) {
+        const int rank = rank_part[i];
+        if (rank < k) {
+            const uint64_t x = cands[i];
+            oi[rank] = key_index(x);
+            ol[rank] = key_value(x);
+            if (sp != nullptr) sp[key_index(x)] = key_value(x);
+        }
+    }
+    __syncthreads();
+    return true;
 }
 
 // --------------------------------------------------------------------------
 template <int NB, int MM, int R>
 __global__ void __launch_bounds__(kThreads, 1) stream_topk_kernel(const StreamTopkParams p) {
     extern __shared__ __align__(128) unsigned char smem[];
-    const int RS = p.rows_per_stage;
+    const int RS = p.rows_per_stage;  // <= 8 * R
     const int S = p.stages;
     const int row_bytes = p.d_pad * 2;
     const SmemLayout L(NB, p.d_pad, RS, S, row_bytes);
     uint64_t *full = reinterpret_cast<uint64_t *>(smem + L.bars);
     uint64_t *empty = full + kMaxStages;
     uint64_t *sfull = empty + kMaxStages;
+    uint64_t *sempty = sfull + kScoreStages;
     MiscSmem *ms = reinterpret_cast<MiscSmem *>(smem + L.misc);
     float *h_s = reinterpret_cast<float *>(smem + L.h);
     float *scores = reinterpret_cast<float *>(smem + L.scores);
@@ -249,18 +498,18 @@ __global__ void __launch_bounds__(kThreads, 1) stream_topk_kernel(const StreamTo
     const int lane = tid & 31;
     const int G = gridDim.x;
     const int cta = blockIdx.x;
-    const int64_t base = p.V / G, rem = p.V % G;
-    const int64_t r0 = cta * base + (cta < rem ? cta : rem);
-    const int n_rows = static_cast<int>(base + (cta < rem ? 1 : 0));
-    const int n_st = (n_rows + RS - 1) / RS;
+    const int n_chunks = static_cast<int>((p.V + RS - 1) / RS);
     const int C = p.d_pad >> 3;  // 16-byte chunks per row
     const int stage_bytes = RS * row_bytes;
 
     if (tid == 0) {
         for (int s = 0; s < S; ++s) {
             mbar_init(&full[s], 1);
-            mbar_init(&empty[s], kDotWarps + 1);
+            mbar_init(&empty[s], kDotWarps);
+        }
+        for (int s = 0; s < kScoreStages; ++s) {
             mbar_init(&sfull[s], kDotWarps);
+            mbar_init(&sempty[s], 1);
         }
         ms->abort = 0;
         ms->is_last = 0;
@@ -280,137 +529,173 @@ __global__ void __launch_bounds__(kThreads, 1) stream_topk_kernel(const StreamTo
         // ---------------- producer ----------------
         if (lane == 0) {
             const uint64_t pol = l2_evict_first_policy();
-            const unsigned char *src = reinterpret_cast<const unsigned char *>(p.W) +
-                                       static_cast<size_t>(r0) * row_bytes;
+            const unsigned char *W = reinterpret_cast<const unsigned char *>(p.W);
+            const int Ns = p.static_chunks;
+            const int pool0 = G * Ns;
+            // first draw from the pool, issued early so its latency is hidden
+            uint32_t draw = (Ns == 0) ? atomic_add_relaxed_gpu(p.next_chunk, 1u) : 0u;
             int issued = 0;
             bool ok = true;
-            for (int t = 0; t < n_st; ++t) {
+            for (int t = 0;; ++t) {
+                int chunk;
+                if (t < Ns) {
+                    chunk = t * G + cta;
+                } else {
+                    chunk = pool0 + static_cast<int>(draw);
+                    if (chunk >= n_chunks) chunk = -1;
+                }
                 const int s = t % S, u = t / S;
                 if (t >= S && !mbar_wait(&empty[s], (u - 1) & 1, abort_flag)) {
                     ok = false;
                     break;
                 }
-                const int rows = min(RS, n_rows - t * RS);
+                ms->chunk_w[s] = chunk;
+                if (chunk < 0) {
+                    mbar_arrive(&full[s]);  // closes the stream: no bytes
+                    break;
+                }
+                const int64_t row0 = static_cast<int64_t>(chunk) * RS;
+                const int64_t rows = min(static_cast<int64_t>(RS), p.V - row0);
                 const uint32_t bytes = static_cast<uint32_t>(rows * row_bytes);
                 mbar_arrive_expect_tx(&full[s], bytes);
-                bulk_g2s(ring + s * stage_bytes, src + static_cast<size_t>(t) * stage_bytes, bytes,
-                         &full[s], pol);
+                bulk_g2s(ring + s * stage_bytes, W + row0 * row_bytes, bytes, &full[s], pol);
                 issued = t + 1;
+                if (t + 1 >= Ns) draw = atomic_add_relaxed_gpu(p.next_chunk, 1u);
             }
             if (!ok) {
                 atomicOr(p.err, kErrWaitTimeout);
                 ms->abort = 1;
                 // drain: copies still in flight must land before the CTA exits
                 const int never = 0;
-                for (int t = max(0, issued - S); t < issued; ++t)
-                    mbar_wait(&full[t % S], (t / S) & 1, const_cast<volatile int *>(&never));
+                for (int t2 = max(0, issued - S); t2 < issued; ++t2)
+                    mbar_wait(&full[t2 % S], (t2 / S) & 1, const_cast<volatile int *>(&never));
             }
         }
-    } else if (warp == 1) {
-        // ---------------- selector ----------------
-        WarpList<MM> list[NB];
-        uint64_t tau[NB];
-#pragma unroll
-        for (int nb = 0; nb < NB; ++nb) {
-            list[nb].clear();
-            tau[nb] = 0;
-        }
-        for (int t = 0; t < n_st; ++t) {
-            const int s = t % S, u = t / S;
-            if (!mbar_wait(&sfull[s], u & 1, abort_flag)) {
-                if (lane == 0) {
-                    atomicOr(p.err, kErrWaitTimeout);
-                    ms->abort = 1;
-                }
-                break;
+    } else {
+        // fused sparse output: a fixed slice of every query row = -inf
+        if (p.sparse != nullptr) {
+            const float ninf = __uint_as_float(0xFF800000u);
+            const int64_t base = p.V / G, rem = p.V % G;
+            const int64_t f0 = cta * base + (cta < rem ? cta : rem);
+            const int64_t fn = base + (cta < rem ? 1 : 0);
+            for (int q = 0; q < p.nq; ++q) {
+                float *row = p.sparse + static_cast<int64_t>(q) * p.V + f0;
+                for (int64_t i = tid - 32; i < fn; i += kThreads - 32) row[i] = ninf;
             }
-            const int rows = min(RS, n_rows - t * RS);
-            const uint32_t row_base = static_cast<uint32_t>(r0 + static_cast<int64_t>(t) * RS);
-            const float *sc = scores + s * RS * NB;
+        }
+        if (warp == 1) {
+            // ---------------- selector ----------------
+            WarpList<MM> list[NB];
+            uint64_t tau[NB];
 #pragma unroll
             for (int nb = 0; nb < NB; ++nb) {
-                if (nb >= p.nq) break;
-                for (int rb = 0; rb < rows; rb += 32) {
-                    const int r = rb + lane;
-                    const uint64_t key = (r < rows) ? make_key(sc[r * NB + nb], row_base + r) : 0;
-                    unsigned m = __ballot_sync(0xFFFFFFFFu, key > tau[nb]);
-                    while (m) {
-                        const int src = __ffs(m) - 1;
-                        m &= m - 1;
-                        const uint64_t x = shfl_u64(key, src);
-                        if (x > tau[nb]) {
-                            list[nb].insert(x, lane);
-                            tau[nb] = list[nb].at(p.k - 1);
+                list[nb].clear();
+                tau[nb] = 0;
+            }
+            for (int t = 0;; ++t) {
+                const int s = t % kScoreStages, u = t / kScoreStages;
+                if (!mbar_wait(&sfull[s], u & 1, abort_flag)) {
+                    if (lane == 0) {
+                        atomicOr(p.err, kErrWaitTimeout);
+                        ms->abort = 1;
+                    }
+                    break;
+                }
+                const int chunk = ms->chunk_s[s];
+                if (chunk < 0) break;
+                const int64_t row0 = static_cast<int64_t>(chunk) * RS;
+                const int rows = static_cast<int>(min(static_cast<int64_t>(RS), p.V - row0));
+                const float *sc = scores + s * RS * NB;
+#pragma unroll
+                for (int nb = 0; nb < NB; ++nb) {
+                    if (nb >= p.nq) break;
+                    for (int rb = 0; rb < rows; rb += 32) {
+                        const int r = rb + lane;
+                        const uint64_t key =
+                            (r < rows) ? make_key(sc[r * NB + nb], static_cast<uint32_t>(row0 + r)) : 0;
+                        unsigned m = __ballot_sync(0xFFFFFFFFu, key > tau[nb]);
+                        while (m) {
+                            const int srcl = __ffs(m) - 1;
+                            m &= m - 1;
+                            const uint64_t x = shfl_u64(key, srcl);
+                            if (x > tau[nb]) {
+                                list[nb].insert(x, lane);
+                                tau[nb] = list[nb].at(p.k - 1);
+                            }
                         }
                     }
                 }
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&sempty[s]);
             }
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&empty[s]);
-        }
-        // this CTA's sorted top-k per query -> scratch
+            // this CTA's sorted top-k per query -> scratch
 #pragma unroll
-        for (int nb = 0; nb < NB; ++nb) {
-            uint64_t *dst = p.cand + (static_cast<size_t>(nb) * G + cta) * p.k;
+            for (int nb = 0; nb < NB; ++nb) {
+                uint64_t *dst = p.cand + (static_cast<size_t>(nb) * G + cta) * p.k;
 #pragma unroll
-            for (int s = 0; s < MM; ++s) {
-                const int pos = lane * MM + s;
-                if (pos < p.k) dst[pos] = list[nb].v[s];
-            }
-        }
-        __threadfence();
-    } else {
-        // ---------------- projection ----------------
-        const int w = warp - 2;
-        for (int t = 0; t < n_st; ++t) {
-            const int s = t % S, u = t / S;
-            if (!mbar_wait(&full[s], u & 1, abort_flag)) {
-                if (lane == 0) {
-                    atomicOr(p.err, kErrWaitTimeout);
-                    ms->abort = 1;
+                for (int s = 0; s < MM; ++s) {
+                    const int pos = lane * MM + s;
+                    if (pos < p.k) dst[pos] = list[nb].v[s];
                 }
-                break;
             }
-            const int rows = min(RS, n_rows - t * RS);
-            const unsigned char *stage = ring + s * stage_bytes;
-            float *sc = scores + s * RS * NB;
-            // rows of this stage owned by warp w: global row index = w mod 8
-            const int first = (w - ((t * RS) & (kDotWarps - 1)) + kDotWarps) & (kDotWarps - 1);
-            for (int rg = first; rg < rows; rg += kDotWarps * R) {
+        } else {
+            // ---------------- projection ----------------
+            const int w = warp - 2;
+            int t = 0;
+            for (;; ++t) {
+                const int s = t % S, u = t / S;
+                if (!mbar_wait(&full[s], u & 1, abort_flag)) {
+                    if (lane == 0) {
+                        atomicOr(p.err, kErrWaitTimeout);
+                        ms->abort = 1;
+                    }
+                    break;
+                }
+                const int chunk = ms->chunk_w[s];
+                if (chunk < 0) break;
+                const int64_t row0 = static_cast<int64_t>(chunk) * RS;
+                const int rows = static_cast<int>(min(static_cast<int64_t>(RS), p.V - row0));
+                const unsigned char *stage = ring + s * stage_bytes;
+                // warp w owns rows w, w + 8, ... (at most R of them) of the stage
                 int rr[R];
 #pragma unroll
-                for (int i = 0; i < R; ++i) rr[i] = min(rg + i * kDotWarps, rows - 1);
+                for (int i = 0; i < R; ++i) rr[i] = min(w + i * kDotWarps, rows - 1);
                 float acc[R][NB];
 #pragma unroll
                 for (int i = 0; i < R; ++i)
 #pragma unroll
                     for (int nb = 0; nb < NB; ++nb) acc[i][nb] = 0.0f;
-                for (int c = lane; c < C; c += 32) {
-                    uint4 wv[R];
+                if (w < rows) {
+                    for (int c = lane; c < C; c += 32) {
+                        uint4 wv[R];
 #pragma unroll
-                    for (int i = 0; i < R; ++i)
-                        wv[i] = *reinterpret_cast<const uint4 *>(stage + rr[i] * row_bytes + c * 16);
+                        for (int i = 0; i < R; ++i)
+                            wv[i] = *reinterpret_cast<const uint4 *>(stage + rr[i] * row_bytes + c * 16);
 #pragma unroll
-                    for (int nb = 0; nb < NB; ++nb) {
-                        const float4 ha =
-                            *reinterpret_cast<const float4 *>(h_s + (nb * 2 + 0) * (C * 4) + c * 4);
-                        const float4 hb =
-                            *reinterpret_cast<const float4 *>(h_s + (nb * 2 + 1) * (C * 4) + c * 4);
+                        for (int nb = 0; nb < NB; ++nb) {
+                            const float4 ha = *reinterpret_cast<const float4 *>(
+                                h_s + (nb * 2 + 0) * (C * 4) + c * 4);
+                            const float4 hb = *reinterpret_cast<const float4 *>(
+                                h_s + (nb * 2 + 1) * (C * 4) + c * 4);
 #pragma unroll
-                        for (int i = 0; i < R; ++i) {
-                            float a = acc[i][nb];
-                            a = fmaf(bf16_lo(wv[i].x), ha.x, a);
-                            a = fmaf(bf16_hi(wv[i].x), ha.y, a);
-                            a = fmaf(bf16_lo(wv[i].y), ha.z, a);
-                            a = fmaf(bf16_hi(wv[i].y), ha.w, a);
-                            a = fmaf(bf16_lo(wv[i].z), hb.x, a);
-                            a = fmaf(bf16_hi(wv[i].z), hb.y, a);
-                            a = fmaf(bf16_lo(wv[i].w), hb.z, a);
-                            a = fmaf(bf16_hi(wv[i].w), hb.w, a);
-                            acc[i][nb] = a;
+                            for (int i = 0; i < R; ++i) {
+                                float a = acc[i][nb];
+                                a = fmaf(bf16_lo(wv[i].x), ha.x, a);
+                                a = fmaf(bf16_hi(wv[i].x), ha.y, a);
+                                a = fmaf(bf16_lo(wv[i].y), ha.z, a);
+                                a = fmaf(bf16_hi(wv[i].y), ha.w, a);
+                                a = fmaf(bf16_lo(wv[i].z), hb.x, a);
+                                a = fmaf(bf16_hi(wv[i].z), hb.y, a);
+                                a = fmaf(bf16_lo(wv[i].w), hb.z, a);
+                                a = fmaf(bf16_hi(wv[i].w), hb.w, a);
+                                acc[i][nb] = a;
+                            }
                         }
                     }
                 }
+                // every read of the weight stage has retired: hand it back
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&empty[s]);
 #pragma unroll
                 for (int i = 0; i < R; ++i)
 #pragma unroll
@@ -420,148 +705,135 @@ __global__ void __launch_bounds__(kThreads, 1) stream_topk_kernel(const StreamTo
                         for (int o = 16; o >= 1; o >>= 1) a += __shfl_xor_sync(0xFFFFFFFFu, a, o);
                         acc[i][nb] = a;
                     }
+                const int ss = t % kScoreStages, su = t / kScoreStages;
+                if (t >= kScoreStages && !mbar_wait(&sempty[ss], (su - 1) & 1, abort_flag)) {
+                    if (lane == 0) {
+                        atomicOr(p.err, kErrWaitTimeout);
+                        ms->abort = 1;
+                    }
+                    break;
+                }
+                float *sc = scores + ss * RS * NB;
                 if (lane == 0) {
+                    if (w == 0) ms->chunk_s[ss] = chunk;
 #pragma unroll
                     for (int i = 0; i < R; ++i) {
-                        const int r = rg + i * kDotWarps;
+                        const int r = w + i * kDotWarps;
                         if (r < rows) {
 #pragma unroll
                             for (int nb = 0; nb < NB; ++nb) sc[r * NB + nb] = acc[i][nb];
                         }
                     }
                 }
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&sfull[ss]);
             }
-            __syncwarp();
-            if (lane == 0) {
-                mbar_arrive(&empty[s]);
-                mbar_arrive(&sfull[s]);
+            // pass the end of the stream on to the selector
+            if (!*abort_flag) {
+                const int ss = t % kScoreStages, su = t / kScoreStages;
+                if (t < kScoreStages || mbar_wait(&sempty[ss], (su - 1) & 1, abort_flag)) {
+                    if (lane == 0) {
+                        if (w == 0) ms->chunk_s[ss] = -1;
+                        mbar_arrive(&sfull[ss]);
+                    }
+                } else if (lane == 0) {
+                    atomicOr(p.err, kErrWaitTimeout);
+                    ms->abort = 1;
+                }
             }
         }
     }
 
     // ---------------- completion ticket ----------------
+    // bar.sync orders every thread's writes (lists, sparse fill) before
+    // thread 0's release; its acquire, then bar.sync, orders the merging
+    // CTA's reads after every other CTA's writes.
     __syncthreads();
     if (tid == 0) {
-        __threadfence();
-        const uint32_t ticket = atomicAdd(p.ticket, 1u);
+        const uint32_t ticket = atomic_add_acq_rel_gpu(p.ticket, 1u);
         ms->is_last = (ticket == static_cast<uint32_t>(G - 1)) ? 1 : 0;
     }
     __syncthreads();
     if (!ms->is_last) return;
-    __threadfence();
 
     // ---------------- global merge (last CTA) ----------------
-    uint64_t *pref = reinterpret_cast<uint64_t *>(smem + L.merge);
-    uint64_t *cands = pref + kMergePrefixCap;
-    uint64_t *win = cands + kMergeCandCap;
-    int *counts = reinterpret_cast<int *>(win + 1024);
-    int *offsets = counts + kMaxLists;
-    uint32_t *hist = reinterpret_cast<uint32_t *>(offsets + kMaxLists);
+    MergeBufs mb;
+    mb.pref = reinterpret_cast<uint64_t *>(smem + L.merge);
+    mb.cands = mb.pref + kMergePrefixCap;
+    mb.win = mb.cands + kMergeCandCap;
+    mb.counts = reinterpret_cast<int *>(mb.win + 1024);
+    mb.offsets = mb.counts + kMaxLists;
+    mb.hist = reinterpret_cast<uint32_t *>(mb.offsets + kMaxLists);
+    uint64_t *staged = reinterpret_cast<uint64_t *>(smem + L.merge + SmemLayout::merge_fixed_bytes());
+    const int stage_cap =
+        static_cast<int>((L.total - L.merge - SmemLayout::merge_fixed_bytes()) / 8);
     const int k = p.k;
-    const int J = (k + G - 1) / G;
-    const int P = G * J;
     const bool aborted = (*reinterpret_cast<volatile uint32_t *>(p.err) & kErrWaitTimeout) != 0;
 
+    // Small k: one pass of independent L2 loads fetches the first kFastE
+    // entries of every list of every query (thread c: list c), then each
+    // query is merged in shared memory; a query the fast merge cannot settle
+    // is merged in full.
+    const int G8 = (G + 7) & ~7;
+    const bool fast = !aborted && k <= kFastMaxK && G >= k && 2 * G <= kThreads &&
+                      p.nq * (G * kFastE * 8 + G8 * 4) <= stage_cap * 8;
+    uint32_t fast_done = 0;  // bit nb: query nb settled by the fast merge
+    if (fast) {
+        uint64_t *fe = staged;                                               // [nq][G][E]
+        uint32_t *hv = reinterpret_cast<uint32_t *>(fe + p.nq * G * kFastE);  // [nq][G8]
+        const int En = k < kFastE ? k : kFastE;
+        for (int q = 0; q < p.nq; ++q) {
+            if (tid < G8) {
+                uint64_t key[kFastE];
+                const unsigned long long *lc = reinterpret_cast<const unsigned long long *>(p.cand) +
+                                               (static_cast<size_t>(q) * G + tid) * k;
+#pragma unroll
+                for (int e = 0; e < kFastE; ++e) key[e] = (tid < G && e < En) ? __ldcg(lc + e) : 0ull;
+                if (tid < G) {
+#pragma unroll
+                    for (int e = 0; e < kFastE; ++e) fe[(q * G + tid) * kFastE + e] = key[e];
+                }
+                hv[q * G8 + tid] = tid < G ? static_cast<uint32_t>(key[0] >> 32) : 0u;
+            }
+        }
+        __syncthreads();
+        for (int nb = 0; nb < p.nq; ++nb) {
+            int32_t *oi = p.out_idx + static_cast<size_t>(nb) * k;
+            float *ol = p.out_logits + static_cast<size_t>(nb) * k;
+            float *sp = p.sparse != nullptr ? p.sparse + static_cast<int64_t>(nb) * p.V : nullptr;
+            if (merge_fast_query(fe + nb * G * kFastE, hv + nb * G8, G, k, mb.cands,
+                                 mb.counts, ms, oi, ol, sp))
+                fast_done |= 1u << nb;
+        }
+    }
     for (int nb = 0; nb < p.nq && !aborted; ++nb) {
+        if (fast_done & (1u << nb)) continue;
         const uint64_t *lists = p.cand + static_cast<size_t>(nb) * G * k;
         int32_t *oi = p.out_idx + static_cast<size_t>(nb) * k;
         float *ol = p.out_logits + static_cast<size_t>(nb) * k;
-
-        // 1. tau*: k-th largest among the first J entries of every list
-        uint64_t tau = 0;
-        if (P <= kMergePrefixCap) {
-            for (int i = tid; i < P; i += kThreads) {
-                const int c = i / J, j = i - c * J;
-                pref[i] = __ldcg(reinterpret_cast<const unsigned long long *>(lists) +
-                                 static_cast<size_t>(c) * k + j);
-            }
-            if (tid == 0) ms->tau = 0;
-            __syncthreads();
-            if (P <= kRankCountMax) {
-                for (int i = tid; i < P; i += kThreads) {
-                    const uint64_t x = pref[i];
-                    if (x == 0) continue;
-                    int rank = 0;
-                    for (int j = 0; j < P; ++j) rank += (pref[j] > x) ? 1 : 0;
-                    if (rank == k - 1) ms->tau = x;
-                }
-                __syncthreads();
-                tau = ms->tau;
+        float *sp = p.sparse != nullptr ? p.sparse + static_cast<int64_t>(nb) * p.V : nullptr;
+        const int n_all = G * k;
+        if (n_all <= stage_cap) {
+            // one pass of independent L2 loads brings every list in
+            const unsigned long long *src = reinterpret_cast<const unsigned long long *>(lists);
+            if ((reinterpret_cast<uintptr_t>(src) & 15u) == 0) {
+                const ulonglong2 *src2 = reinterpret_cast<const ulonglong2 *>(src);
+                ulonglong2 *dst2 = reinterpret_cast<ulonglong2 *>(staged);
+                for (int i = tid; i < (n_all >> 1); i += kThreads) dst2[i] = __ldcg(src2 + i);
+                if ((n_all & 1) && tid == 0) staged[n_all - 1] = __ldcg(src + n_all - 1);
             } else {
-                int nz = 0;  // nonzero keys among the prefixes
-                for (int i = 0; i < P; ++i) nz += pref[i] != 0;
-                tau = (nz >= k) ? block_radix_threshold(SmemKeys{pref}, P, k, 1, hist, ms) : 0;
-            }
-        }
-        // 2. per-list count of keys >= tau* (lists are sorted descending); the
-        //    first J entries are already in shared memory, deeper entries are
-        //    fetched eight at a time with independent loads.
-        const uint64_t lo = tau > 0 ? tau : 1;
-        const bool have_pref = P <= kMergePrefixCap;
-        for (int c = tid; c < G; c += kThreads) {
-            const unsigned long long *lc =
-                reinterpret_cast<const unsigned long long *>(lists) + static_cast<size_t>(c) * k;
-            int n = 0;
-            if (have_pref)
-                while (n < J && pref[c * J + n] >= lo) ++n;
-            if (!have_pref || n == J) {
-                for (int b = n; b < k && n == b; b += 8) {
-                    uint64_t e[8];
-#pragma unroll
-                    for (int q = 0; q < 8; ++q) e[q] = (b + q < k) ? __ldcg(lc + b + q) : 0;
-#pragma unroll
-                    for (int q = 0; q < 8; ++q)
-                        if (n == b + q && b + q < k && e[q] >= lo) ++n;
-                }
-            }
-            counts[c] = n;
-        }
-        __syncthreads();
-        if (tid < 32) {
-            // exclusive scan of counts[0..G) by one warp, chunk per lane
-            const int per = (G + 31) / 32;
-            const int b0 = tid * per;
-            int local = 0;
-            for (int c = b0; c < min(G, b0 + per); ++c) local += counts[c];
-            int incl = local;
-#pragma unroll
-            for (int o = 1; o < 32; o <<= 1) {
-                const int t2 = __shfl_up_sync(0xFFFFFFFFu, incl, o);
-                if (tid >= o) incl += t2;
-            }
-            int run = incl - local;
-            for (int c = b0; c < min(G, b0 + per); ++c) {
-                offsets[c] = run;
-                run += counts[c];
-            }
-            if (tid == 31) ms->n_cand = incl;
-        }
-        __syncthreads();
-        const int M = ms->n_cand;
-        if (M <= kMergeCandCap) {
-            // 3a. gather the candidates, exact top-k among them
-            for (int c = tid; c < G; c += kThreads) {
-                const unsigned long long *lc =
-                    reinterpret_cast<const unsigned long long *>(lists) + static_cast<size_t>(c) * k;
-                for (int j = 0; j < counts[c]; ++j)
-                    cands[offsets[c] + j] = (have_pref && j < J) ? pref[c * J + j] : __ldcg(lc + j);
+                for (int i = tid; i < n_all; i += kThreads) staged[i] = __ldcg(src + i);
             }
             __syncthreads();
-            block_topk_to_output(cands, M, k, win, hist, ms, oi, ol);
+            merge_lists(SmemKeys{staged}, G, k, mb, ms, oi, ol, sp);
         } else {
-            // 3b. too many candidates: radix-select the threshold over all lists
-            const uint64_t T = block_radix_threshold(GlobalKeys{lists}, G * k, k, lo, hist, ms);
-            if (tid == 0) ms->n_win = 0;
-            __syncthreads();
-            for (int i = tid; i < G * k; i += kThreads) {
-                const uint64_t x = __ldcg(reinterpret_cast<const unsigned long long *>(lists) + i);
-                if (x >= T && x >= lo) win[atomicAdd(&ms->n_win, 1)] = x;
-            }
-            __syncthreads();
-            block_topk_to_output(win, k, k, win, hist, ms, oi, ol);
+            merge_lists(GlobalKeys{lists}, G, k, mb, ms, oi, ol, sp);
         }
     }
-    if (tid == 0) *p.ticket = 0;  // re-arm for the next launch
+    if (tid == 0) {
+        *p.ticket = 0;  // re-arm both counters for the next launch
+        *p.next_chunk = 0;
+    }
 }
 
 }  // namespace vie

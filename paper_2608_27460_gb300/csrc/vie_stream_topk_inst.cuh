@@ -6,9 +6,8 @@
 
 namespace vie {
 
-template <int NB, int MM>
+template <int NB, int MM, int kR>
 cudaError_t launch_one(const StreamTopkParams &p, int grid, uint32_t smem, cudaStream_t stream) {
-    constexpr int kR = 2;
     static bool configured[64] = {};
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
@@ -24,18 +23,29 @@ cudaError_t launch_one(const StreamTopkParams &p, int grid, uint32_t smem, cudaS
     return cudaGetLastError();
 }
 
-template <int NB>
-cudaError_t launch_width(int mm, const StreamTopkParams &p, int grid, uint32_t smem,
-                         cudaStream_t stream) {
+template <int NB, int R>
+cudaError_t launch_rows(int mm, const StreamTopkParams &p, int grid, uint32_t smem,
+                        cudaStream_t stream) {
     // Wide lists are only built for narrow query groups (register budget).
     switch (mm) {
-        case 2: return launch_one<NB, 2>(p, grid, smem, stream);
+        case 2: return launch_one<NB, 2, R>(p, grid, smem, stream);
         case 8:
-            if constexpr (NB <= 4) return launch_one<NB, 8>(p, grid, smem, stream);
+            if constexpr (NB <= 4) return launch_one<NB, 8, R>(p, grid, smem, stream);
             return cudaErrorInvalidValue;
         case 32:
-            if constexpr (NB == 1) return launch_one<NB, 32>(p, grid, smem, stream);
+            if constexpr (NB == 1) return launch_one<NB, 32, R>(p, grid, smem, stream);
             return cudaErrorInvalidValue;
+        default: return cudaErrorInvalidValue;
+    }
+}
+
+template <int NB>
+cudaError_t launch_width(int mm, int r, const StreamTopkParams &p, int grid, uint32_t smem,
+                         cudaStream_t stream) {
+    switch (r) {
+        case 1: return launch_rows<NB, 1>(mm, p, grid, smem, stream);
+        case 2: return launch_rows<NB, 2>(mm, p, grid, smem, stream);
+        case 4: return launch_rows<NB, 4>(mm, p, grid, smem, stream);
         default: return cudaErrorInvalidValue;
     }
 }

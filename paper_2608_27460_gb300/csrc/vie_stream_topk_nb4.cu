@@ -2,8 +2,8 @@
 #include "vie_stream_topk_inst.cuh"
 
 namespace vie {
-cudaError_t launch_stream_topk_nb4(int mm, const StreamTopkParams &p, int grid, uint32_t smem,
-                                   cudaStream_t stream) {
-    return launch_width<4>(mm, p, grid, smem, stream);
+cudaError_t launch_stream_topk_nb4(int mm, int r, const StreamTopkParams &p, int grid,
+                                   uint32_t smem, cudaStream_t stream) {
+    return launch_width<4>(mm, r, p, grid, smem, stream);
 }
 }  // namespace vie

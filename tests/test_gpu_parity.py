@@ -112,6 +112,32 @@ def test_scatter_is_bit_exact(vie):
         np.testing.assert_array_equal(out.cpu().numpy().view(np.uint32), want.view(np.uint32))
 
 
+@pytest.mark.parametrize("V,d,batch,k", [(50021, 256, 4, 50), (20011, 640, 1, 1), (4099, 100, 3, 300),
+                                         (151936, 1024, 1, 50), (70001, 512, 13, 64)])
+def test_fused_sparse_equals_topk_then_scatter(vie, V, d, batch, k):
+    """One-launch top-k + sparse tensor: same top-k as vie_head_topk and the
+    sparse rows bit-equal to the oracle's scatter of those results."""
+    import torch
+    W, h = workload(V, d, batch, seed=V + k)
+    with vie.Head(to_device_bits(W)) as head:
+        hd = torch.from_numpy(h).cuda()
+        i1, v1 = head.topk(hd, k)
+        base = torch.empty(batch * V + 1, dtype=torch.float32, device="cuda")
+        sp_out = base[1:].view(batch, V)  # rows that start off 16-byte alignment
+        sp_out.fill_(7.0)
+        i2, v2, sp = head.topk_sparse(hd, k, out_sparse=sp_out)
+        torch.cuda.synchronize()
+        assert head.device_status() == vie.VIE_OK
+        np.testing.assert_array_equal(i1.cpu().numpy(), i2.cpu().numpy())
+        np.testing.assert_array_equal(v1.cpu().numpy().view(np.uint32), v2.cpu().numpy().view(np.uint32))
+        want, ok = oracle.scatter(i2.cpu().numpy(), v2.cpu().numpy(), V)
+        assert ok
+        np.testing.assert_array_equal(sp.cpu().numpy().view(np.uint32), want.view(np.uint32))
+    z = oracle.logits(W, h)
+    for q in range(batch):
+        assert not check_topk(i2.cpu().numpy()[q], v2.cpu().numpy()[q], z[q], k)
+
+
 @pytest.mark.parametrize("V,batch,k,offset", [(1, 1, 1, 0), (7, 3, 7, 1), (262144, 2, 50, 3),
                                                (151936, 1, 1024, 1), (100000, 70, 5, 2)])
 def test_scatter_shapes_and_alignment(vie, V, batch, k, offset):
@@ -122,11 +148,12 @@ def test_scatter_shapes_and_alignment(vie, V, batch, k, offset):
     val = rng.standard_normal((batch, k)).astype(np.float32)
     base = torch.empty(batch * V + offset, dtype=torch.float32, device="cuda")
     out = base[offset:]
-    st = vie.vie_scatter_sparse_logits(torch.from_numpy(idx).cuda().data_ptr(),
-                                       torch.from_numpy(val).cuda().data_ptr(), batch, k, V,
+    idx_d = torch.from_numpy(idx).cuda()  # keep both alive while the kernel runs
+    val_d = torch.from_numpy(val).cuda()
+    st = vie.vie_scatter_sparse_logits(idx_d.data_ptr(), val_d.data_ptr(), batch, k, V,
                                        out.data_ptr(), torch.cuda.current_stream().cuda_stream)
     assert st == vie.VIE_OK
-    torch.cuda.synchronize()
+    assert vie.vie_device_status() == vie.VIE_OK
     want, ok = oracle.scatter(idx, val, V)
     np.testing.assert_array_equal(out.view(batch, V).cpu().numpy().view(np.uint32),
                                   want.view(np.uint32))
