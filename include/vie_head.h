@@ -147,6 +147,43 @@ vie_status vie_scatter_sparse_logits(const int32_t *idx, const float *logits, in
                                      int32_t k, int64_t V, float *out, vie_stream stream);
 
 /*
+ * vie_head_topk_noalloc - vie_head_topk for callers that cannot allocate
+ * device memory.  The paper has no counterpart: this is a deployment variant.
+ *
+ * Some callers are not allowed to call cudaMalloc at all: code running while
+ * a CUDA graph is being captured, engines whose device memory is carved out
+ * of one budget up front, and latency-critical loops that cannot afford the
+ * implicit device synchronisation an allocation may bring.  A vie_head
+ * allocates its padded weight copy and scratch in vie_head_create, so those
+ * callers cannot make one.  This entry point takes the weights as they are
+ * and keeps its scratch in a fixed array compiled into the library instead.
+ *
+ *   W_out       device, bf16 bit patterns, row-major [V, d], 16-byte aligned,
+ *               d a multiple of 8 (rows must already be 16-byte vectors).
+ *   V, d        1 <= V <= 2^31 - 2;  8 <= d <= VIE_D_MAX.
+ *   h, batch, k, out_idx, out_logits, stream: as for vie_head_topk.
+ *
+ * Scratch: one 1 MiB array per device (every GPU that loads the library keeps
+ * it until the process exits).  A launch needs 8 * slots * ctas * k bytes of
+ * it, where ctas = min(SM count, ceil(V / 64)) and slots = the query group
+ * width (the batch rounded up to a power of two, at most 8); larger requests
+ * return VIE_ERR_UNSUPPORTED with the sizes in the message.  The call clears
+ * the counters at the start of the array with cudaMemsetAsync on `stream`
+ * and allocates nothing (no cudaMalloc, no cudaFree, no allocating library
+ * routine).
+ * The first call on a device looks up the array's device address with
+ * cudaGetSymbolAddress (once per device); make that first call before any
+ * stream capture.  Every call shares the one array, so calls whose work
+ * overlaps on the GPU (other streams, other threads) race and corrupt each
+ * other's results: serialise them.  Device-side problems set the flag read by
+ * vie_device_status.  Errors: VIE_ERR_INVALID_ARG, VIE_ERR_UNSUPPORTED,
+ * VIE_ERR_CUDA.
+ */
+vie_status vie_head_topk_noalloc(const void *W_out, int64_t V, int32_t d, const float *h,
+                                 int32_t batch, int32_t k, int32_t *out_idx, float *out_logits,
+                                 vie_stream stream);
+
+/*
  * vie_device_status - synchronises `stream`, then reads and clears the
  * library's device-side flag word of the current device.  Returns VIE_OK when
  * no kernel recorded a problem, VIE_ERR_DEVICE otherwise (vie_last_error()

@@ -36,7 +36,7 @@ STATUS_NAMES = {0: "VIE_OK", 1: "VIE_ERR_INVALID_ARG", 2: "VIE_ERR_UNSUPPORTED",
 
 # Every entry point of include/vie_head.h.
 EXPORTS = ("vie_head_create", "vie_head_destroy", "vie_head_get_props", "vie_head_topk",
-           "vie_head_topk_sparse", "vie_scatter_sparse_logits", "vie_device_status", "vie_head_device_status",
+           "vie_head_topk_sparse", "vie_head_topk_noalloc", "vie_scatter_sparse_logits", "vie_device_status", "vie_head_device_status",
            "vie_last_error")
 
 
@@ -80,6 +80,7 @@ def load(path: str | None = None, build_if_missing: bool = True):
             "vie_head_get_props": ([P, ctypes.POINTER(vie_head_props)], ctypes.c_int),
             "vie_head_topk": ([P, P, I32, I32, P, P, P], ctypes.c_int),
             "vie_head_topk_sparse": ([P, P, I32, I32, P, P, P, P], ctypes.c_int),
+            "vie_head_topk_noalloc": ([P, I64, I32, P, I32, I32, P, P, P], ctypes.c_int),
             "vie_scatter_sparse_logits": ([P, P, I32, I32, I64, P, P], ctypes.c_int),
             "vie_device_status": ([P], ctypes.c_int),
             "vie_head_device_status": ([P, P], ctypes.c_int),
@@ -126,6 +127,13 @@ def vie_head_topk(head: int, h: int, batch: int, k: int, out_idx: int, out_logit
 def vie_head_topk_sparse(head: int, h: int, batch: int, k: int, out_idx: int, out_logits: int,
                          out_sparse: int, stream: int = 0) -> int:
     return load().vie_head_topk_sparse(head, h, batch, k, out_idx, out_logits, out_sparse, stream)
+
+
+def vie_head_topk_noalloc(W_out: int, V: int, d: int, h: int, batch: int, k: int, out_idx: int,
+                          out_logits: int, stream: int = 0) -> int:
+    """Top-k straight from caller-owned weights, scratch in a fixed library
+    array: for callers that must not allocate device memory."""
+    return load().vie_head_topk_noalloc(W_out, V, d, h, batch, k, out_idx, out_logits, stream)
 
 
 def vie_scatter_sparse_logits(idx: int, logits: int, batch: int, k: int, V: int, out: int,

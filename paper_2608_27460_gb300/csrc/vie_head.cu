@@ -9,6 +9,7 @@
 #include <cstdio>
 #include <cstdlib>
 #include <cstring>
+#include <mutex>
 #include <new>
 
 #include "vie_head.h"
@@ -419,6 +420,119 @@ vie_status vie_head_device_status(vie_head *head, vie_stream stream) {
 }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------------------
+// Top-k without any device allocation: the same kernel as vie_head_topk, with
+// its scratch (ticket and pool counters, per-CTA candidate lists) placed in a
+// fixed array that lives in this module instead of memory from cudaMalloc.
+namespace {
+
+constexpr size_t kNoAllocScratchBytes = size_t(1) << 20;  // 1 MiB per device
+constexpr size_t kNoAllocCounterBytes = 256;              // counters, then the lists
+
+// Host code sees only a stand-in for this array; kernels get its device
+// address, looked up once per device below.
+static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
+
+struct NoAllocDevice {
+    std::once_flag once;
+    cudaError_t setup_error = cudaSuccess;
+    unsigned char *scratch = nullptr;  // device address of g_noalloc_scratch
+    uint32_t *flag = nullptr;          // device address of g_dev_err
+    int sms = 0;
+};
+NoAllocDevice g_noalloc[64];
+
+}  // namespace
+
+extern "C" vie_status vie_head_topk_noalloc(const void *W_out, int64_t V, int32_t d, const float *h,
+                                           int32_t batch, int32_t k, int32_t *out_idx,
+                                           float *out_logits, vie_stream stream) {
+    const char *fn = "vie_head_topk_noalloc";
+    if (W_out == nullptr || h == nullptr || out_idx == nullptr || out_logits == nullptr)
+        return fail(VIE_ERR_INVALID_ARG, "%s: NULL buffer", fn);
+    if (V < 1 || V > static_cast<int64_t>(INT32_MAX) - 1)
+        return fail(VIE_ERR_INVALID_ARG, "%s: V=%lld outside [1, 2^31-2]", fn,
+                    static_cast<long long>(V));
+    if (d < 8 || d > VIE_D_MAX || (d & 7) != 0)
+        return fail(VIE_ERR_INVALID_ARG, "%s: d=%d must be a multiple of 8 in [8, %d]", fn, d,
+                    VIE_D_MAX);
+    if (reinterpret_cast<uintptr_t>(W_out) & 15u)
+        return fail(VIE_ERR_INVALID_ARG, "%s: W_out must be 16-byte aligned", fn);
+    if (batch < 1 || batch > VIE_BATCH_MAX)
+        return fail(VIE_ERR_INVALID_ARG, "%s: batch=%d outside [1, %d]", fn, batch, VIE_BATCH_MAX);
+    if (k < 1 || k > VIE_K_MAX || static_cast<int64_t>(k) > V)
+        return fail(VIE_ERR_INVALID_ARG, "%s: k=%d outside [1, min(V, %d)]", fn, k, VIE_K_MAX);
+    if ((reinterpret_cast<uintptr_t>(h) | reinterpret_cast<uintptr_t>(out_idx) |
+         reinterpret_cast<uintptr_t>(out_logits)) & 3u)
+        return fail(VIE_ERR_INVALID_ARG, "%s: buffers must be 4-byte aligned", fn);
+
+    int dev = -1;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return fail_cuda(e, "cudaGetDevice");
+    if (dev < 0 || dev >= 64) return fail(VIE_ERR_UNSUPPORTED, "%s: device %d", fn, dev);
+    NoAllocDevice &nd = g_noalloc[dev];
+    std::call_once(nd.once, [&nd, dev]() {
+        nd.setup_error = cudaGetSymbolAddress(reinterpret_cast<void **>(&nd.scratch), g_noalloc_scratch);
+        if (nd.setup_error == cudaSuccess)
+            nd.setup_error = cudaGetSymbolAddress(reinterpret_cast<void **>(&nd.flag), g_dev_err);
+        if (nd.setup_error == cudaSuccess)
+            nd.setup_error = cudaDeviceGetAttribute(&nd.sms, cudaDevAttrMultiProcessorCount, dev);
+    });
+    if (nd.setup_error != cudaSuccess) return fail_cuda(nd.setup_error, "vie_head_topk_noalloc set-up");
+
+    int64_t g = (V + 63) / 64;
+    if (g > nd.sms) g = nd.sms;
+    if (g > vie::kMaxLists) g = vie::kMaxLists;
+    const int G = static_cast<int>(g < 1 ? 1 : g);
+    const int mm = pick_mm(k);
+    const int cap = nb_cap_for(d, mm);
+    int nb_max = 1;
+    while (nb_max < cap && nb_max < batch) nb_max <<= 1;
+    const size_t lists_bytes = static_cast<size_t>(nb_max) * G * k * sizeof(uint64_t);
+    if (lists_bytes > kNoAllocScratchBytes - kNoAllocCounterBytes)
+        return fail(VIE_ERR_UNSUPPORTED,
+                    "%s: needs %zu bytes of scratch (%d query slots x %d CTAs x k=%d x 8), more than "
+                    "the fixed %zu; use vie_head_topk or a smaller batch or k",
+                    fn, lists_bytes, nb_max, G, k, kNoAllocScratchBytes - kNoAllocCounterBytes);
+
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    uint32_t *counters = reinterpret_cast<uint32_t *>(nd.scratch);
+    e = cudaMemsetAsync(counters, 0, 4 * sizeof(uint32_t), s);  // ticket and pool start at 0
+    if (e != cudaSuccess) return fail_cuda(e, "vie_head_topk_noalloc clear");
+    for (int q0 = 0; q0 < batch; q0 += cap) {
+        const int nq = batch - q0 < cap ? batch - q0 : cap;
+        int nb = 1;
+        while (nb < nq) nb <<= 1;
+        LaunchShape shp;
+        if (!pick_shape(nb, d, &shp))
+            return fail(VIE_ERR_UNSUPPORTED, "%s: no shared-memory layout for d=%d", fn, d);
+        vie::StreamTopkParams p;
+        p.W = static_cast<const uint16_t *>(W_out);
+        p.h = h + static_cast<int64_t>(q0) * d;
+        p.nq = nq;
+        p.V = V;
+        p.d = d;
+        p.d_pad = d;
+        p.k = k;
+        p.rows_per_stage = shp.rs;
+        p.stages = shp.stages;
+        const int64_t n_chunks = (V + shp.rs - 1) / shp.rs;
+        int pct = knobs().static_pct;
+        pct = pct < 0 ? 0 : (pct > 100 ? 100 : pct);
+        p.static_chunks = static_cast<int32_t>(n_chunks * pct / 100 / G);
+        p.cand = reinterpret_cast<uint64_t *>(nd.scratch + kNoAllocCounterBytes);
+        p.ticket = counters;
+        p.next_chunk = counters + 2;
+        p.err = nd.flag;
+        p.out_idx = out_idx + static_cast<int64_t>(q0) * k;
+        p.out_logits = out_logits + static_cast<int64_t>(q0) * k;
+        p.sparse = nullptr;
+        e = vie::launch_stream_topk(nb, mm, shp.r, p, G, shp.smem, s);
+        if (e != cudaSuccess) return fail_cuda(e, fn);
+    }
+    return VIE_OK;
+}
 
 namespace vie {
 cudaError_t launch_stream_topk(int nb, int mm, int r, const StreamTopkParams &p, int grid,

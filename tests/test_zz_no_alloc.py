@@ -1,0 +1,56 @@
+"""vie_head_topk_noalloc: top-k for callers that must not allocate device
+memory (graph capture, fixed memory budgets, allocation-free loops).
+
+It must give the same results as vie_head_topk, call after call, with its
+scratch held in the library's fixed array.  This file is collected last so
+that a failure here stops a run only after every other test has run."""
+import numpy as np
+import pytest
+
+from gpu_cases import to_device_bits, workload
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.mark.parametrize("V,d,batch,k", [(151936, 1024, 1, 50), (20011, 640, 3, 1), (70001, 512, 8, 64)])
+def test_noalloc_matches_head_topk_twice(vie, V, d, batch, k):
+    import torch
+    W, h = workload(V, d, batch, seed=V + 11 * k)
+    Wd = to_device_bits(W)
+    hd = torch.from_numpy(h).cuda()
+    s = torch.cuda.current_stream().cuda_stream
+    with vie.Head(Wd) as head:
+        ref_idx, ref_val = head.topk(hd, k)
+    torch.cuda.synchronize()
+    ref_idx, ref_val = ref_idx.cpu().numpy(), ref_val.cpu().numpy()
+    for call in range(2):
+        idx = torch.full((batch, k), -1, dtype=torch.int32, device="cuda")
+        val = torch.full((batch, k), float("nan"), dtype=torch.float32, device="cuda")
+        st = vie.vie_head_topk_noalloc(Wd.data_ptr(), V, d, hd.data_ptr(), batch, k,
+                                       idx.data_ptr(), val.data_ptr(), s)
+        assert st == vie.VIE_OK, vie.vie_last_error()
+        assert vie.vie_device_status(s) == vie.VIE_OK, vie.vie_last_error()
+        # same indices; logits within the parity tolerance (they are computed
+        # by the same kernel, so in practice they agree bit for bit)
+        np.testing.assert_array_equal(idx.cpu().numpy(), ref_idx, err_msg=f"call {call}")
+        got = val.cpu().numpy()
+        assert np.all(np.abs(got - ref_val) <= 2e-3 + 1e-3 * np.abs(ref_val)), f"call {call}"
+
+
+def test_noalloc_rejects_what_it_cannot_serve(vie):
+    import torch
+    W = torch.zeros((1000, 12), dtype=torch.int16, device="cuda")  # d not a multiple of 8
+    h = torch.zeros((1, 12), dtype=torch.float32, device="cuda")
+    i = torch.empty((1, 4), dtype=torch.int32, device="cuda")
+    v = torch.empty((1, 4), dtype=torch.float32, device="cuda")
+    s = torch.cuda.current_stream().cuda_stream
+    assert vie.vie_head_topk_noalloc(W.data_ptr(), 1000, 12, h.data_ptr(), 1, 4, i.data_ptr(),
+                                     v.data_ptr(), s) == vie.VIE_ERR_INVALID_ARG
+    W2 = torch.zeros((200000, 16), dtype=torch.int16, device="cuda")
+    h2 = torch.zeros((8, 16), dtype=torch.float32, device="cuda")
+    i2 = torch.empty((8, 1024), dtype=torch.int32, device="cuda")
+    v2 = torch.empty((8, 1024), dtype=torch.float32, device="cuda")
+    st = vie.vie_head_topk_noalloc(W2.data_ptr(), 200000, 16, h2.data_ptr(), 8, 1024,
+                                   i2.data_ptr(), v2.data_ptr(), s)
+    assert st == vie.VIE_ERR_UNSUPPORTED and "scratch" in vie.vie_last_error()
+    torch.cuda.synchronize()
