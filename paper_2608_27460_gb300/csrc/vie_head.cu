@@ -14,6 +14,7 @@
 
 #include "vie_head.h"
 #include "vie_launch.h"
+#include "vie_tc_topk.cuh"
 
 namespace {
 
@@ -51,6 +52,11 @@ struct vie_head {
     uint64_t *cand;     // [kMaxNB][G][VIE_K_MAX] ranking keys
     uint32_t *words;    // [0] completion ticket, [1] device flag word, [2] chunk pool counter
     int64_t scratch_bytes;
+    // tensor-core path (batches): hi/lo bf16 query matrix and TMA descriptors
+    void *hB;             // [kTcHRows][d_pad] bf16
+    bool tc_ready;
+    CUtensorMap mapW;     // W as [V][d_pad], box 128 rows x 64 columns, 128-byte swizzle
+    CUtensorMap mapH[3];  // hB, box 16 / 32 / 64 rows x 64 columns
 };
 
 // ---------------------------------------------------------------------------
@@ -139,11 +145,14 @@ int env_int(const char *name, int dflt) {
 // Launch-shape knobs (they change speed, never results):
 //   VIE_STAGE_MIN_KB     smallest weight stage worth one bulk copy (48)
 //   VIE_STATIC_PCT       share of the chunks assigned statically, in % (85)
+//   VIE_TC_MIN_BATCH     smallest batch sent to the tensor-core path (2)
+//   VIE_TC_KPS           K-blocks of 64 columns per tensor-core ring stage (2)
 struct Knobs {
-    int stage_min_bytes, static_pct;
+    int stage_min_bytes, static_pct, tc_min_batch, tc_kps;
 };
 const Knobs &knobs() {
-    static const Knobs k = {env_int("VIE_STAGE_MIN_KB", 48) * 1024, env_int("VIE_STATIC_PCT", 85)};
+    static const Knobs k = {env_int("VIE_STAGE_MIN_KB", 48) * 1024, env_int("VIE_STATIC_PCT", 85),
+                            env_int("VIE_TC_MIN_BATCH", 2), env_int("VIE_TC_KPS", 2)};
     return k;
 }
 
@@ -181,6 +190,39 @@ vie_status check_device(const vie_head *hd) {
         return fail(VIE_ERR_INVALID_ARG, "handle lives on device %d but device %d is current",
                     hd->device, dev);
     return VIE_OK;
+}
+
+// cuTensorMapEncodeTiled from the driver, looked up once.
+using EncodeTiledFn = CUresult (*)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *,
+                                   const cuuint64_t *, const cuuint64_t *, const cuuint32_t *,
+                                   const cuuint32_t *, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                   CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+EncodeTiledFn encode_tiled() {
+    static EncodeTiledFn fn = []() -> EncodeTiledFn {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                             &q) != cudaSuccess ||
+            q != cudaDriverEntryPointSuccess)
+            return nullptr;
+        return reinterpret_cast<EncodeTiledFn>(p);
+    }();
+    return fn;
+}
+
+// 2-D bf16 tensor map [rows][cols] (cols contiguous, pitch bytes), box
+// box_rows x 64 columns, 128-byte swizzle, out-of-range elements read as 0.
+bool make_map_bf16(CUtensorMap *m, void *base, uint64_t rows, uint64_t cols, uint64_t pitch,
+                   uint32_t box_rows) {
+    EncodeTiledFn fn = encode_tiled();
+    if (fn == nullptr) return false;
+    const cuuint64_t dims[2] = {cols, rows};
+    const cuuint64_t strides[1] = {pitch};
+    const cuuint32_t box[2] = {static_cast<cuuint32_t>(vie::kTcKBlock), box_rows};
+    const cuuint32_t estr[2] = {1, 1};
+    return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, base, dims, strides, box, estr,
+              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
 }  // namespace
@@ -240,6 +282,9 @@ vie_status vie_head_create(const void *W_out, int64_t V, int32_t d, vie_dtype dt
     e = cudaMalloc(&hd->W, wbytes);
     if (e == cudaSuccess) e = cudaMalloc(&hd->cand, cbytes);
     if (e == cudaSuccess) e = cudaMalloc(&hd->words, 4 * sizeof(uint32_t));
+    if (e == cudaSuccess)
+        e = cudaMalloc(&hd->hB, static_cast<size_t>(vie::kTcHRows) * hd->d_pad * 2);
+    if (e == cudaSuccess) e = cudaMemset(hd->hB, 0, static_cast<size_t>(vie::kTcHRows) * hd->d_pad * 2);
     if (e == cudaSuccess) e = cudaMemset(hd->words, 0, 4 * sizeof(uint32_t));
     if (e == cudaSuccess) {
         const int64_t chunks = V * (hd->d_pad >> 3);
@@ -255,9 +300,15 @@ vie_status vie_head_create(const void *W_out, int64_t V, int32_t d, vie_dtype dt
         cudaFree(hd->W);
         cudaFree(hd->cand);
         cudaFree(hd->words);
+        cudaFree(hd->hB);
         delete hd;
         return st;
     }
+    const uint64_t pitch = static_cast<uint64_t>(hd->d_pad) * 2;
+    hd->tc_ready = make_map_bf16(&hd->mapW, hd->W, static_cast<uint64_t>(V), hd->d_pad, pitch,
+                                 vie::kTcTile);
+    for (int i = 0; i < 3 && hd->tc_ready; ++i)
+        hd->tc_ready = make_map_bf16(&hd->mapH[i], hd->hB, vie::kTcHRows, hd->d_pad, pitch, 16u << i);
     *out = hd;
     return VIE_OK;
 }
@@ -267,6 +318,7 @@ vie_status vie_head_destroy(vie_head *head) {
     cudaFree(head->W);
     cudaFree(head->cand);
     cudaFree(head->words);
+    cudaFree(head->hB);
     delete head;
     return VIE_OK;
 }
@@ -281,6 +333,51 @@ vie_status vie_head_get_props(const vie_head *head, vie_head_props *props) {
     props->device = head->device;
     props->weight_bytes = head->V * head->d_pad * 2;
     props->scratch_bytes = head->scratch_bytes;
+    return VIE_OK;
+}
+
+// Batches on the tensor cores: per group of up to 32 queries, the hi/lo
+// query matrix, the tcgen05 projection with per-CTA top-k, and the merge.
+static vie_status run_topk_tc(const char *fn, vie_head *head, const float *h, int32_t batch,
+                              int32_t k, int32_t *out_idx, float *out_logits, float *sparse,
+                              cudaStream_t s) {
+    const int nqt = batch <= 8 ? 8 : (batch <= 16 ? 16 : 32);
+    int stages = 0;
+    uint32_t smem = 0;
+    int kps = knobs().tc_kps;
+    kps = kps < 1 ? 1 : (kps > vie::kTcMaxKPS ? vie::kTcMaxKPS : kps);
+    while (kps > 1 && !vie::tc_shape(nqt, kps, &stages, &smem)) --kps;
+    if (!vie::tc_shape(nqt, kps, &stages, &smem))
+        return fail(VIE_ERR_UNSUPPORTED, "%s: no tensor-core layout", fn);
+    const int n_tiles = static_cast<int>((head->V + vie::kTcTile - 1) / vie::kTcTile);
+    int pct = knobs().static_pct;
+    pct = pct < 0 ? 0 : (pct > 100 ? 100 : pct);
+    const CUtensorMap &mapH = head->mapH[nqt == 8 ? 0 : (nqt == 16 ? 1 : 2)];
+    for (int q0 = 0; q0 < batch; q0 += nqt) {
+        const int nq = batch - q0 < nqt ? batch - q0 : nqt;
+        cudaError_t e = vie::launch_prep_queries(h + static_cast<int64_t>(q0) * head->d, nq, head->d,
+                                                 head->d_pad, 2 * nqt, head->hB, head->num_sms, s);
+        if (e != cudaSuccess) return fail_cuda(e, fn);
+        vie::TcParams p;
+        p.V = head->V;
+        p.d_pad = head->d_pad;
+        p.k = k;
+        p.nq = nq;
+        p.stages = stages;
+        p.kb_per_stage = kps;
+        p.static_tiles = static_cast<int32_t>(static_cast<int64_t>(n_tiles) * pct / 100 / head->G);
+        p.cand = head->cand;
+        p.next_tile = head->words + 2;
+        p.err = head->words + 1;
+        p.sparse = sparse != nullptr ? sparse + static_cast<int64_t>(q0) * head->V : nullptr;
+        e = vie::launch_tc_topk(nqt, head->mapW, mapH, p, head->G, smem, s);
+        if (e != cudaSuccess) return fail_cuda(e, fn);
+        e = vie::launch_merge_lists(head->cand, nq, head->G, k, head->V,
+                                    out_idx + static_cast<int64_t>(q0) * k,
+                                    out_logits + static_cast<int64_t>(q0) * k, p.sparse,
+                                    head->words + 2, head->words + 1, s);
+        if (e != cudaSuccess) return fail_cuda(e, fn);
+    }
     return VIE_OK;
 }
 
@@ -302,8 +399,10 @@ static vie_status run_topk(const char *fn, vie_head *head, const float *h, int32
     if (st != VIE_OK) return st;
 
     const int mm = pick_mm(k);
-    const int cap = nb_cap_for(head->d_pad, mm);
     cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if (head->tc_ready && batch >= knobs().tc_min_batch && k <= vie::kTcMaxK && head->d_pad >= 64)
+        return run_topk_tc(fn, head, h, batch, k, out_idx, out_logits, sparse, s);
+    const int cap = nb_cap_for(head->d_pad, mm);
     for (int q0 = 0; q0 < batch; q0 += cap) {
         const int nq = batch - q0 < cap ? batch - q0 : cap;
         int nb = 1;

@@ -2,6 +2,7 @@
 // translation unit per query-group width so they compile in parallel.
 #pragma once
 
+#include <cuda.h>
 #include <cuda_runtime.h>
 
 #include "vie_stream_topk.cuh"
@@ -22,5 +23,26 @@ cudaError_t launch_stream_topk_nb4(int mm, int r, const StreamTopkParams &p, int
                                    uint32_t smem, cudaStream_t stream);
 cudaError_t launch_stream_topk_nb8(int mm, int r, const StreamTopkParams &p, int grid,
                                    uint32_t smem, cudaStream_t stream);
+
+// ---- tensor-core head (vie_tc_topk.cu) ----
+struct TcParams;
+
+// Ring depth and dynamic shared memory of the tensor-core kernel for query
+// groups of nq_tmpl (8, 16 or 32) and kps K-blocks per stage; false if
+// unsupported.
+bool tc_shape(int nq_tmpl, int kps, int *stages, uint32_t *smem);
+
+// Launches tc_topk_kernel<nq_tmpl>.
+cudaError_t launch_tc_topk(int nq_tmpl, const CUtensorMap &mapW, const CUtensorMap &mapH,
+                           const TcParams &p, int grid, uint32_t smem, cudaStream_t stream);
+
+// hi/lo bf16 query matrix [n_rows][d_pad] for the tensor-core kernel.
+cudaError_t launch_prep_queries(const float *h, int nq, int d, int d_pad, int n_rows, void *hB,
+                                int sms, cudaStream_t stream);
+
+// One CTA per query: merges the per-CTA lists of nq queries.
+cudaError_t launch_merge_lists(const uint64_t *cand, int nq, int G, int k, int64_t V,
+                               int32_t *out_idx, float *out_logits, float *sparse,
+                               uint32_t *next_tile, const uint32_t *err, cudaStream_t stream);
 
 }  // namespace vie

@@ -475,6 +475,86 @@ __device__ inline bool merge_fast_query(const uint64_t *fe, const uint32_t *hv, 
     return true;
 }
 
+// Merges the per-CTA lists of queries 0..nq-1 (query q's G lists of k keys
+// at cand + q*G*k) into each query's exact top-k, written best first to
+// out_idx / out_logits + q*k and, if sparse is set, into row q of the sparse
+// tensor.  `ws` is merge_bytes of shared memory for the working buffers.
+// Small k: one pass of independent L2 loads fetches the first kFastE
+// entries of every list of every query (thread c: list c), then each query
+// is merged in shared memory; a query the fast merge cannot settle is merged
+// in full.  Called by all kThreads threads of one CTA.
+__device__ inline void merge_queries(const uint64_t *cand, int nq, int G, int k, int64_t V,
+                                     unsigned char *ws, uint32_t merge_bytes, MiscSmem *ms,
+                                     int32_t *out_idx, float *out_logits, float *sparse) {
+    const int tid = threadIdx.x;
+    MergeBufs mb;
+    mb.pref = reinterpret_cast<uint64_t *>(ws);
+    mb.cands = mb.pref + kMergePrefixCap;
+    mb.win = mb.cands + kMergeCandCap;
+    mb.counts = reinterpret_cast<int *>(mb.win + 1024);
+    mb.offsets = mb.counts + kMaxLists;
+    mb.hist = reinterpret_cast<uint32_t *>(mb.offsets + kMaxLists);
+    uint64_t *staged = reinterpret_cast<uint64_t *>(ws + SmemLayout::merge_fixed_bytes());
+    const int stage_cap = static_cast<int>((merge_bytes - SmemLayout::merge_fixed_bytes()) / 8);
+
+    const int G8 = (G + 7) & ~7;
+    const bool fast = k <= kFastMaxK && G >= k && 2 * G <= kThreads &&
+                      nq * (G * kFastE * 8 + G8 * 4) <= stage_cap * 8;
+    uint32_t fast_done = 0;  // bit nb: query nb settled by the fast merge
+    if (fast) {
+        uint64_t *fe = staged;                                             // [nq][G][E]
+        uint32_t *hv = reinterpret_cast<uint32_t *>(fe + nq * G * kFastE);  // [nq][G8]
+        const int En = k < kFastE ? k : kFastE;
+        for (int q = 0; q < nq; ++q) {
+            if (tid < G8) {
+                uint64_t key[kFastE];
+                const unsigned long long *lc = reinterpret_cast<const unsigned long long *>(cand) +
+                                               (static_cast<size_t>(q) * G + tid) * k;
+#pragma unroll
+                for (int e = 0; e < kFastE; ++e) key[e] = (tid < G && e < En) ? __ldcg(lc + e) : 0ull;
+                if (tid < G) {
+#pragma unroll
+                    for (int e = 0; e < kFastE; ++e) fe[(q * G + tid) * kFastE + e] = key[e];
+                }
+                hv[q * G8 + tid] = tid < G ? static_cast<uint32_t>(key[0] >> 32) : 0u;
+            }
+        }
+        __syncthreads();
+        for (int nb = 0; nb < nq; ++nb) {
+            int32_t *oi = out_idx + static_cast<size_t>(nb) * k;
+            float *ol = out_logits + static_cast<size_t>(nb) * k;
+            float *sp = sparse != nullptr ? sparse + static_cast<int64_t>(nb) * V : nullptr;
+            if (merge_fast_query(fe + nb * G * kFastE, hv + nb * G8, G, k, mb.cands, mb.counts, ms,
+                                 oi, ol, sp))
+                fast_done |= 1u << nb;
+        }
+    }
+    for (int nb = 0; nb < nq; ++nb) {
+        if (fast_done & (1u << nb)) continue;
+        const uint64_t *lists = cand + static_cast<size_t>(nb) * G * k;
+        int32_t *oi = out_idx + static_cast<size_t>(nb) * k;
+        float *ol = out_logits + static_cast<size_t>(nb) * k;
+        float *sp = sparse != nullptr ? sparse + static_cast<int64_t>(nb) * V : nullptr;
+        const int n_all = G * k;
+        if (n_all <= stage_cap) {
+            // one pass of independent L2 loads brings every list in
+            const unsigned long long *src = reinterpret_cast<const unsigned long long *>(lists);
+            if ((reinterpret_cast<uintptr_t>(src) & 15u) == 0) {
+                const ulonglong2 *src2 = reinterpret_cast<const ulonglong2 *>(src);
+                ulonglong2 *dst2 = reinterpret_cast<ulonglong2 *>(staged);
+                for (int i = tid; i < (n_all >> 1); i += kThreads) dst2[i] = __ldcg(src2 + i);
+                if ((n_all & 1) && tid == 0) staged[n_all - 1] = __ldcg(src + n_all - 1);
+            } else {
+                for (int i = tid; i < n_all; i += kThreads) staged[i] = __ldcg(src + i);
+            }
+            __syncthreads();
+            merge_lists(SmemKeys{staged}, G, k, mb, ms, oi, ol, sp);
+        } else {
+            merge_lists(GlobalKeys{lists}, G, k, mb, ms, oi, ol, sp);
+        }
+    }
+}
+
 // --------------------------------------------------------------------------
 template <int NB, int MM, int R>
 __global__ void __launch_bounds__(kThreads, 1) stream_topk_kernel(const StreamTopkParams p) {
@@ -757,79 +837,10 @@ __global__ void __launch_bounds__(kThreads, 1) stream_topk_kernel(const StreamTo
     if (!ms->is_last) return;
 
     // ---------------- global merge (last CTA) ----------------
-    MergeBufs mb;
-    mb.pref = reinterpret_cast<uint64_t *>(smem + L.merge);
-    mb.cands = mb.pref + kMergePrefixCap;
-    mb.win = mb.cands + kMergeCandCap;
-    mb.counts = reinterpret_cast<int *>(mb.win + 1024);
-    mb.offsets = mb.counts + kMaxLists;
-    mb.hist = reinterpret_cast<uint32_t *>(mb.offsets + kMaxLists);
-    uint64_t *staged = reinterpret_cast<uint64_t *>(smem + L.merge + SmemLayout::merge_fixed_bytes());
-    const int stage_cap =
-        static_cast<int>((L.total - L.merge - SmemLayout::merge_fixed_bytes()) / 8);
-    const int k = p.k;
     const bool aborted = (*reinterpret_cast<volatile uint32_t *>(p.err) & kErrWaitTimeout) != 0;
-
-    // Small k: one pass of independent L2 loads fetches the first kFastE
-    // entries of every list of every query (thread c: list c), then each
-    // query is merged in shared memory; a query the fast merge cannot settle
-    // is merged in full.
-    const int G8 = (G + 7) & ~7;
-    const bool fast = !aborted && k <= kFastMaxK && G >= k && 2 * G <= kThreads &&
-                      p.nq * (G * kFastE * 8 + G8 * 4) <= stage_cap * 8;
-    uint32_t fast_done = 0;  // bit nb: query nb settled by the fast merge
-    if (fast) {
-        uint64_t *fe = staged;                                               // [nq][G][E]
-        uint32_t *hv = reinterpret_cast<uint32_t *>(fe + p.nq * G * kFastE);  // [nq][G8]
-        const int En = k < kFastE ? k : kFastE;
-        for (int q = 0; q < p.nq; ++q) {
-            if (tid < G8) {
-                uint64_t key[kFastE];
-                const unsigned long long *lc = reinterpret_cast<const unsigned long long *>(p.cand) +
-                                               (static_cast<size_t>(q) * G + tid) * k;
-#pragma unroll
-                for (int e = 0; e < kFastE; ++e) key[e] = (tid < G && e < En) ? __ldcg(lc + e) : 0ull;
-                if (tid < G) {
-#pragma unroll
-                    for (int e = 0; e < kFastE; ++e) fe[(q * G + tid) * kFastE + e] = key[e];
-                }
-                hv[q * G8 + tid] = tid < G ? static_cast<uint32_t>(key[0] >> 32) : 0u;
-            }
-        }
-        __syncthreads();
-        for (int nb = 0; nb < p.nq; ++nb) {
-            int32_t *oi = p.out_idx + static_cast<size_t>(nb) * k;
-            float *ol = p.out_logits + static_cast<size_t>(nb) * k;
-            float *sp = p.sparse != nullptr ? p.sparse + static_cast<int64_t>(nb) * p.V : nullptr;
-            if (merge_fast_query(fe + nb * G * kFastE, hv + nb * G8, G, k, mb.cands,
-                                 mb.counts, ms, oi, ol, sp))
-                fast_done |= 1u << nb;
-        }
-    }
-    for (int nb = 0; nb < p.nq && !aborted; ++nb) {
-        if (fast_done & (1u << nb)) continue;
-        const uint64_t *lists = p.cand + static_cast<size_t>(nb) * G * k;
-        int32_t *oi = p.out_idx + static_cast<size_t>(nb) * k;
-        float *ol = p.out_logits + static_cast<size_t>(nb) * k;
-        float *sp = p.sparse != nullptr ? p.sparse + static_cast<int64_t>(nb) * p.V : nullptr;
-        const int n_all = G * k;
-        if (n_all <= stage_cap) {
-            // one pass of independent L2 loads brings every list in
-            const unsigned long long *src = reinterpret_cast<const unsigned long long *>(lists);
-            if ((reinterpret_cast<uintptr_t>(src) & 15u) == 0) {
-                const ulonglong2 *src2 = reinterpret_cast<const ulonglong2 *>(src);
-                ulonglong2 *dst2 = reinterpret_cast<ulonglong2 *>(staged);
-                for (int i = tid; i < (n_all >> 1); i += kThreads) dst2[i] = __ldcg(src2 + i);
-                if ((n_all & 1) && tid == 0) staged[n_all - 1] = __ldcg(src + n_all - 1);
-            } else {
-                for (int i = tid; i < n_all; i += kThreads) staged[i] = __ldcg(src + i);
-            }
-            __syncthreads();
-            merge_lists(SmemKeys{staged}, G, k, mb, ms, oi, ol, sp);
-        } else {
-            merge_lists(GlobalKeys{lists}, G, k, mb, ms, oi, ol, sp);
-        }
-    }
+    if (!aborted)
+        merge_queries(p.cand, p.nq, G, p.k, p.V, smem + L.merge, L.total - L.merge, ms, p.out_idx,
+                      p.out_logits, p.sparse);
     if (tid == 0) {
         *p.ticket = 0;  // re-arm both counters for the next launch
         *p.next_chunk = 0;

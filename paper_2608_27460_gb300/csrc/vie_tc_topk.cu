@@ -1,0 +1,140 @@
+// vie_tc_topk.cu - launchers of the tensor-core head: hi/lo query prep,
+// the tcgen05 projection + per-CTA top-k, and the per-query merge.
+#include <cuda_bf16.h>
+
+#include "vie_launch.h"
+#include "vie_tc_topk.cuh"
+
+namespace vie {
+
+// hB[n_rows][d_pad] bf16: row 2q = rn(h_q), row 2q+1 = rn(h_q - rn(h_q)),
+// rows of absent queries and columns >= d are zero.
+__global__ void prep_queries_kernel(const float *__restrict__ h, int nq, int d, int d_pad,
+                                    int n_rows, __nv_bfloat16 *__restrict__ hB) {
+    const int64_t n = static_cast<int64_t>(n_rows) * d_pad;
+    for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < n;
+         i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+        const int r = static_cast<int>(i / d_pad), j = static_cast<int>(i - static_cast<int64_t>(r) * d_pad);
+        const int q = r >> 1;
+        const float x = (q < nq && j < d) ? h[static_cast<int64_t>(q) * d + j] : 0.0f;
+        const __nv_bfloat16 hi = __float2bfloat16_rn(x);
+        hB[i] = (r & 1) ? __float2bfloat16_rn(x - __bfloat162float(hi)) : hi;
+    }
+}
+
+// One CTA per query: merges the G per-CTA lists of query blockIdx.x.  Runs
+// after tc_topk_kernel on the same stream; re-arms the tile pool counter.
+__global__ void __launch_bounds__(kThreads, 1)
+    merge_lists_kernel(const uint64_t *cand, int G, int k, int64_t V, int32_t *out_idx,
+                       float *out_logits, float *sparse, uint32_t *next_tile, const uint32_t *err,
+                       uint32_t ws_bytes) {
+    extern __shared__ __align__(1024) unsigned char tc_smem[];
+    unsigned char *smem = tc_smem;
+    MiscSmem *ms = reinterpret_cast<MiscSmem *>(smem);
+    unsigned char *ws = smem + 256;
+    const int q = blockIdx.x;
+    if (q == 0 && threadIdx.x == 0) *next_tile = 0;
+    if (*reinterpret_cast<const volatile uint32_t *>(err) & kErrWaitTimeout) return;
+    merge_queries(cand + static_cast<size_t>(q) * G * k, 1, G, k, V, ws, ws_bytes, ms,
+                  out_idx + static_cast<size_t>(q) * k, out_logits + static_cast<size_t>(q) * k,
+                  sparse != nullptr ? sparse + static_cast<int64_t>(q) * V : nullptr);
+}
+
+namespace {
+
+template <int NQ>
+cudaError_t launch_tc_one(const CUtensorMap &mapW, const CUtensorMap &mapH, const TcParams &p,
+                          int grid, uint32_t smem, cudaStream_t stream) {
+    static bool configured[64] = {};
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+    if (!configured[dev]) {
+        e = cudaFuncSetAttribute(tc_topk_kernel<NQ>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 232448);
+        if (e != cudaSuccess) return e;
+        configured[dev] = true;
+    }
+    tc_topk_kernel<NQ><<<grid, TcShape<NQ>::kThreads, smem, stream>>>(mapW, mapH, p);
+    return cudaGetLastError();
+}
+
+template <int NQ>
+int tc_stage_bytes() {
+    return TcShape<NQ>::kStageBytes;
+}
+
+}  // namespace
+
+bool tc_shape(int nq_tmpl, int kps, int *stages, uint32_t *smem) {
+    int score_bytes = 0, buf_bytes = 0, stage_bytes = 0;
+    switch (nq_tmpl) {
+        case 8: score_bytes = TcShape<8>::kScoreBytes; buf_bytes = TcShape<8>::kBufBytes;
+                stage_bytes = TcShape<8>::kStageBytes; break;
+        case 16: score_bytes = TcShape<16>::kScoreBytes; buf_bytes = TcShape<16>::kBufBytes;
+                 stage_bytes = TcShape<16>::kStageBytes; break;
+        case 32: score_bytes = TcShape<32>::kScoreBytes; buf_bytes = TcShape<32>::kBufBytes;
+                 stage_bytes = TcShape<32>::kStageBytes; break;
+        default: return false;
+    }
+    for (int s = kTcMaxStages; s >= 2; --s) {
+        const TcSmemLayout L(score_bytes, buf_bytes, s, kps * stage_bytes);
+        if (L.total <= 232448u) {
+            *stages = s;
+            *smem = L.total;
+            return true;
+        }
+    }
+    return false;
+}
+
+cudaError_t launch_tc_topk(int nq_tmpl, const CUtensorMap &mapW, const CUtensorMap &mapH,
+                           const TcParams &p, int grid, uint32_t smem, cudaStream_t stream) {
+    switch (nq_tmpl) {
+        case 8: return launch_tc_one<8>(mapW, mapH, p, grid, smem, stream);
+        case 16: return launch_tc_one<16>(mapW, mapH, p, grid, smem, stream);
+        case 32: return launch_tc_one<32>(mapW, mapH, p, grid, smem, stream);
+        default: return cudaErrorInvalidValue;
+    }
+}
+
+cudaError_t launch_prep_queries(const float *h, int nq, int d, int d_pad, int n_rows, void *hB,
+                                int sms, cudaStream_t stream) {
+    const int64_t n = static_cast<int64_t>(n_rows) * d_pad;
+    int64_t blocks = (n + 255) / 256;
+    if (blocks > 4LL * sms) blocks = 4LL * sms;
+    prep_queries_kernel<<<static_cast<unsigned>(blocks), 256, 0, stream>>>(
+        h, nq, d, d_pad, n_rows, static_cast<__nv_bfloat16 *>(hB));
+    return cudaGetLastError();
+}
+
+uint32_t merge_kernel_smem(int G, int k) {
+    const uint32_t stage = static_cast<uint32_t>(G) * k * 8;
+    const uint32_t fast = static_cast<uint32_t>(G) * (kFastE * 8 + 4) + 64;
+    const uint32_t ws = SmemLayout::merge_fixed_bytes() + (stage > fast ? stage : fast);
+    const uint32_t cap = 232448u - 256u;
+    return 256u + (ws < cap ? ws : cap);
+}
+
+cudaError_t launch_merge_lists(const uint64_t *cand, int nq, int G, int k, int64_t V,
+                               int32_t *out_idx, float *out_logits, float *sparse,
+                               uint32_t *next_tile, const uint32_t *err, cudaStream_t stream) {
+    static bool configured[64] = {};
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+    if (!configured[dev]) {
+        e = cudaFuncSetAttribute(merge_lists_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 232448);
+        if (e != cudaSuccess) return e;
+        configured[dev] = true;
+    }
+    const uint32_t smem = merge_kernel_smem(G, k);
+    merge_lists_kernel<<<nq, kThreads, smem, stream>>>(cand, G, k, V, out_idx, out_logits, sparse,
+                                                        next_tile, err, smem - 256u);
+    return cudaGetLastError();
+}
+
+}  // namespace vie

@@ -1,0 +1,469 @@
+// vie_tc_topk.cuh - the batched output head on the 5th-generation tensor
+// cores: Z[V, b] = W[V, d] * H[d, b] (paper, Section 3, z = W_out h for b
+// queries at once) with the exact per-CTA top-k fused into the epilogue.
+//
+// h is fp32; tcgen05 kind::f16 needs both operands in bf16, so each query
+// enters as two bf16 columns hi = rn(h), lo = rn(h - hi) and its logit is the
+// sum of the two accumulator columns (residual error <= 2^-18 |h| per term).
+// N = 2 * NQ accumulator columns per tile.
+//
+// One persistent CTA per SM walks 128-row tiles of W (round robin, then an
+// atomic pool).  Per tile, d/64 K-blocks flow through a shared-memory ring;
+// a stage is one 2-D TMA box of W (128 rows x 64 bf16, 128-byte swizzle)
+// plus the matching box of the hi/lo query matrix (N rows x 64).
+//   warp 0       TMA producer;
+//   warp 1       TMEM allocator and the single MMA-issuing thread:
+//                4 x tcgen05.mma (M=128, N, K=16) per stage into one of two
+//                TMEM accumulators, tcgen05.commit frees the stage;
+//   warps 2-5    epilogue: tcgen05.ld of the 128 x N accumulator (warp w
+//                owns TMEM lanes 32*(w%4)..), hi + lo per query, logits into
+//                a score ring laid out [query][row];
+//   warps 6..    selectors, four queries each: per query a shared buffer
+//                of candidates above a threshold tau; when it passes half
+//                full, a warp-wide bitonic sort keeps the best k and raises
+//                tau (a few sorts per query instead of one insert per key).
+// Each CTA writes its per-query lists; a separate merge kernel (one CTA per
+// query) merges them.  All waits are bounded.
+#pragma once
+
+#include <cuda.h>
+#include <cstdint>
+
+#include "vie_stream_topk.cuh"
+#include "vie_tcgen05.cuh"
+
+namespace vie {
+
+constexpr int kTcTile = 128;       // rows per tile (MMA M)
+constexpr int kTcKBlock = 64;      // bf16 columns per K-block (one 128-byte swizzle row)
+constexpr int kTcScoreSlots = 4;   // score ring depth
+constexpr int kTcMaxStages = 16;
+constexpr int kTcHRows = 64;       // rows of the hi/lo query matrix (N <= 64)
+constexpr int kTcCap = 256;        // candidate buffer per query (>= k + one tile)
+constexpr int kTcMaxK = kTcCap - kTcTile;  // largest k of this path
+constexpr int kTcMaxKPS = 4;       // K-blocks per stage, at most
+
+struct TcParams {
+    int64_t V;
+    int32_t d_pad;
+    int32_t k;
+    int32_t nq;              // queries of this launch (<= NQ)
+    int32_t stages;          // ring depth
+    int32_t static_tiles;    // tiles each CTA owns before drawing from the pool
+    int32_t kb_per_stage;    // K-blocks per ring stage (1..kTcMaxKPS)
+    uint64_t *cand;          // [NQ][G][k] keys
+    uint32_t *next_tile;     // pool counter (reset by the merge kernel)
+    uint32_t *err;           // device flag word
+    float *sparse;           // [nq, V] fp32 or nullptr: slices filled with -inf here
+};
+
+template <int NQ>
+struct TcShape {
+    static constexpr int N = 2 * NQ;
+    static constexpr int kSelWarps = NQ / 4;
+    static constexpr int kWarps = 6 + kSelWarps;
+    static constexpr int kThreads = 32 * kWarps;
+    static constexpr int kStageA = kTcTile * kTcKBlock * 2;  // 16 KB per K-block of W
+    static constexpr int kStageB = N * kTcKBlock * 2;        // N x 128 B per K-block of H
+    static constexpr int kStageBytes = kStageA + kStageB;    // per K-block; a multiple of 1024
+    static constexpr int kTmemCols = (2 * N <= 32) ? 32 : (2 * N <= 64 ? 64 : 128);
+    static constexpr int kSlots = NQ >= 32 ? 2 : kTcScoreSlots;  // score ring depth
+    static constexpr int kScoreBytes = kSlots * NQ * kTcTile * 4;
+    static constexpr int kBufBytes = NQ * kTcCap * 8 + NQ * 12;  // buffers, counts, thresholds
+};
+
+struct TcMisc {
+    uint32_t tmem_base;
+    int abort;
+    int stage_tile[kTcMaxStages];  // tile of a stage that starts a tile (-1: end)
+    int buf_tile[2];               // tile held by each TMEM accumulator
+    int slot_tile[kTcScoreSlots];  // tile of each score slot
+};
+
+struct TcSmemLayout {
+    uint32_t bars, misc, scores, bufs, ring, total;
+    __host__ __device__ TcSmemLayout(int score_bytes, int buf_bytes, int stages, int stage_bytes) {
+        bars = 0;
+        misc = 512;
+        scores = 1024;
+        bufs = scores + score_bytes;
+        ring = (bufs + buf_bytes + 1023u) & ~1023u;
+        total = ring + stages * stage_bytes + 1024;  // +1024: room to align the ring
+    }
+};
+
+__device__ __forceinline__ uint64_t shfl_xor_u64(uint64_t v, int m) {
+    const uint32_t lo = __shfl_xor_sync(0xFFFFFFFFu, static_cast<uint32_t>(v), m);
+    const uint32_t hi = __shfl_xor_sync(0xFFFFFFFFu, static_cast<uint32_t>(v >> 32), m);
+    return (static_cast<uint64_t>(hi) << 32) | lo;
+}
+
+// Bitonic sort, descending, of the 32 * PER keys a warp holds (lane l holds
+// elements l*PER .. l*PER + PER - 1).  Steps with a stride below PER swap
+// registers; wider steps exchange with lane ^ (stride / PER).
+template <int PER>
+__device__ __forceinline__ void warp_sort_desc(uint64_t (&v)[PER], int lane) {
+#pragma unroll
+    for (int size = 2; size <= 32 * PER; size <<= 1) {
+#pragma unroll
+        for (int stride = size >> 1; stride > 0; stride >>= 1) {
+            if (stride < PER) {
+#pragma unroll
+                for (int j = 0; j < PER; ++j) {
+                    const int pj = j ^ stride;
+                    if (pj > j) {
+                        const bool desc = ((lane * PER + j) & size) == 0;
+                        const uint64_t a = v[j], b = v[pj];
+                        if (desc ? (a < b) : (a > b)) {
+                            v[j] = b;
+                            v[pj] = a;
+                        }
+                    }
+                }
+            } else {
+                const int ls = stride / PER;
+                const bool lower = (lane & ls) == 0;
+#pragma unroll
+                for (int j = 0; j < PER; ++j) {
+                    const uint64_t o = shfl_xor_u64(v[j], ls);
+                    const bool desc = ((lane * PER + j) & size) == 0;
+                    const bool keep_max = lower == desc;
+                    v[j] = keep_max ? (v[j] > o ? v[j] : o) : (v[j] < o ? v[j] : o);
+                }
+            }
+        }
+    }
+}
+
+// Keeps the best min(k, cnt) of the cnt keys in buf (sorted descending at
+// buf[0..)), returns the new count; *tau becomes the k-th key once k are
+// held.  Out of line: one copy of the sorting network serves every call.
+static __device__ __noinline__ int compact_candidates(uint64_t *buf, int cnt, int k, uint64_t *tau,
+                                               int lane) {
+    constexpr int PER = kTcCap / 32;
+    uint64_t v[PER];
+#pragma unroll
+    for (int j = 0; j < PER; ++j) {
+        const int e = lane * PER + j;
+        v[j] = e < cnt ? buf[e] : 0ull;
+    }
+    __syncwarp();
+    warp_sort_desc<PER>(v, lane);
+    const int keep = cnt < k ? cnt : k;
+#pragma unroll
+    for (int j = 0; j < PER; ++j) {
+        const int e = lane * PER + j;
+        if (e < keep) buf[e] = v[j];
+    }
+    if (keep == k) {
+        uint64_t x = 0;
+        const int slot = (k - 1) % PER;
+#pragma unroll
+        for (int j = 0; j < PER; ++j)
+            if (j == slot) x = v[j];
+        x = shfl_u64(x, (k - 1) / PER);
+        if (lane == 0) *tau = x;
+    }
+    __syncwarp();
+    return keep;
+}
+
+template <int NQ>
+__global__ void __launch_bounds__(TcShape<NQ>::kThreads, 1)
+    tc_topk_kernel(const __grid_constant__ CUtensorMap mapW, const __grid_constant__ CUtensorMap mapH,
+                   const TcParams p) {
+    using Sh = TcShape<NQ>;
+    constexpr int N = Sh::N;
+    extern __shared__ __align__(1024) unsigned char tc_smem[];
+    unsigned char *smem = tc_smem;
+    const int S = p.stages;
+    const int KPS = p.kb_per_stage;
+    const int stage_bytes = KPS * Sh::kStageBytes;  // [KPS boxes of W][KPS boxes of H]
+    const TcSmemLayout L(Sh::kScoreBytes, Sh::kBufBytes, S, stage_bytes);
+    uint64_t *full = reinterpret_cast<uint64_t *>(smem + L.bars);
+    uint64_t *empty = full + kTcMaxStages;
+    uint64_t *tfull = empty + kTcMaxStages;
+    uint64_t *tempty = tfull + 2;
+    uint64_t *sfull = tempty + 2;
+    uint64_t *sempty = sfull + kTcScoreSlots;
+    uint64_t *final_bar = sempty + kTcScoreSlots;
+    TcMisc *mc = reinterpret_cast<TcMisc *>(smem + L.misc);
+    float *scores = reinterpret_cast<float *>(smem + L.scores);
+    uint64_t *bufs = reinterpret_cast<uint64_t *>(smem + L.bufs);
+    // the 128-byte swizzle needs 1024-byte aligned tiles in the shared window
+    unsigned char *ring = smem + L.ring;
+    ring += (1024u - (smem_addr(ring) & 1023u)) & 1023u;
+    volatile int *abort_flag = &mc->abort;
+
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int G = gridDim.x, cta = blockIdx.x;
+    const int n_kb = (p.d_pad + kTcKBlock - 1) / kTcKBlock;
+    const int n_st = (n_kb + KPS - 1) / KPS;  // stages per tile
+    const int n_tiles = static_cast<int>((p.V + kTcTile - 1) / kTcTile);
+
+    if (tid == 0) {
+        for (int s = 0; s < S; ++s) {
+            mbar_init(&full[s], 1);
+            mbar_init(&empty[s], 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(&tfull[b], 2);
+            mbar_init(&tempty[b], 4);
+        }
+        for (int s = 0; s < Sh::kSlots; ++s) {
+            mbar_init(&sfull[s], 4);
+            mbar_init(&sempty[s], Sh::kSelWarps);
+        }
+        mbar_init(final_bar, 1);
+        mc->abort = 0;
+        fence_mbar_init();
+    }
+    if (warp == 1) {
+        tmem_alloc(&mc->tmem_base, Sh::kTmemCols);
+        tmem_relinquish();
+        tc_fence_before_sync();
+    }
+    __syncthreads();
+    tc_fence_after_sync();
+    const uint32_t tmem = mc->tmem_base;
+
+    if (warp == 0) {
+        // ---------------- TMA producer ----------------
+        if (lane == 0) {
+            tma_prefetch_map(&mapW);
+            tma_prefetch_map(&mapH);
+            const uint64_t pol = l2_evict_first_policy();
+            const int Ns = p.static_tiles;
+            const int pool0 = G * Ns;
+            uint32_t draw = (Ns == 0) ? atomic_add_relaxed_gpu(p.next_tile, 1u) : 0u;
+            int it = 0, issued = 0;
+            bool ok = true;
+            for (int ti = 0; ok; ++ti) {
+                int tile;
+                if (ti < Ns) {
+                    tile = ti * G + cta;
+                } else {
+                    tile = pool0 + static_cast<int>(draw);
+                    if (tile >= n_tiles) tile = -1;
+                }
+                if (tile >= 0 && ti + 1 >= Ns) draw = atomic_add_relaxed_gpu(p.next_tile, 1u);
+                const int nst = tile < 0 ? 1 : n_st;
+                for (int st_i = 0; st_i < nst; ++st_i, ++it) {
+                    const int s = it % S, u = it / S;
+                    if (it >= S && !mbar_wait(&empty[s], (u - 1) & 1, abort_flag)) {
+                        ok = false;
+                        break;
+                    }
+                    if (st_i == 0) mc->stage_tile[s] = tile;
+                    if (tile < 0) {
+                        mbar_arrive(&full[s]);  // closes the stream: no bytes
+                        break;
+                    }
+                    const int kb0 = st_i * KPS, nin = min(KPS, n_kb - kb0);
+                    mbar_arrive_expect_tx(&full[s], nin * Sh::kStageBytes);
+                    unsigned char *st = ring + s * stage_bytes;
+                    for (int i = 0; i < nin; ++i)
+                        tma_load_2d(st + i * Sh::kStageA, &mapW, (kb0 + i) * kTcKBlock, tile * kTcTile,
+                                    &full[s], pol);
+                    for (int i = 0; i < nin; ++i)
+                        tma_load_2d(st + KPS * Sh::kStageA + i * Sh::kStageB, &mapH,
+                                    (kb0 + i) * kTcKBlock, 0, &full[s], pol);
+                    issued = it + 1;
+                }
+                if (tile < 0) break;
+            }
+            if (!ok) {
+                atomicOr(p.err, kErrWaitTimeout);
+                mc->abort = 1;
+                const int never = 0;
+                for (int t2 = max(0, issued - S); t2 < issued; ++t2)
+                    mbar_wait(&full[t2 % S], (t2 / S) & 1, const_cast<volatile int *>(&never));
+            }
+        }
+    } else if (warp == 1) {
+        // ---------------- MMA issuer ----------------
+        if (lane == 0) {
+            constexpr uint32_t idesc = umma_idesc_bf16_f32(kTcTile, N);
+            int it = 0;
+            bool ok = true;
+            for (int ti = 0; ok; ++ti) {
+                const int b = ti & 1, ub = ti >> 1;
+                const int s0 = it % S, u0 = it / S;
+                if (!mbar_wait(&full[s0], u0 & 1, abort_flag)) {
+                    ok = false;
+                    break;
+                }
+                const int tile = mc->stage_tile[s0];
+                if (ti >= 2 && !mbar_wait(&tempty[b], (ub - 1) & 1, abort_flag)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after_sync();
+                if (tile < 0) {
+                    mc->buf_tile[b] = -1;
+                    mbar_arrive(&tfull[b]);
+                    mbar_arrive(&tfull[b]);
+                    break;
+                }
+                mc->buf_tile[b] = tile;
+                const uint32_t d = tmem + static_cast<uint32_t>(b * N);
+                for (int st_i = 0; st_i < n_st; ++st_i, ++it) {
+                    const int s = it % S, u = it / S;
+                    if (st_i > 0 && !mbar_wait(&full[s], u & 1, abort_flag)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after_sync();
+                    unsigned char *st = ring + s * stage_bytes;
+                    const int kb0 = st_i * KPS, nin = min(KPS, n_kb - kb0);
+                    for (int i = 0; i < nin; ++i) {
+                        const uint64_t ad = umma_desc_k_sw128(st + i * Sh::kStageA);
+                        const uint64_t bd = umma_desc_k_sw128(st + KPS * Sh::kStageA + i * Sh::kStageB);
+#pragma unroll
+                        for (int k4 = 0; k4 < kTcKBlock / 16; ++k4)  // +32 bytes per K step of 16
+                            umma_bf16(d, ad + 2 * k4, bd + 2 * k4, idesc,
+                                      ((kb0 + i) | k4) != 0 ? 1u : 0u);
+                    }
+                    umma_commit(&empty[s]);
+                }
+                if (!ok) break;
+                umma_commit(&tfull[b]);
+                mbar_arrive(&tfull[b]);  // publishes buf_tile[b]
+            }
+            if (!ok) {
+                atomicOr(p.err, kErrWaitTimeout);
+                mc->abort = 1;
+            }
+            // every MMA this thread issued has finished before TMEM is freed
+            umma_commit(final_bar);
+            const int never = 0;
+            mbar_wait(final_bar, 0, const_cast<volatile int *>(&never));
+        }
+    } else if (warp < 6) {
+        // ---------------- epilogue: TMEM -> logits ----------------
+        const int qw = warp & 3;  // TMEM lane quarter this warp may access
+        const int row = 32 * qw + lane;
+        for (int ti = 0;; ++ti) {
+            const int b = ti & 1, ub = ti >> 1;
+            if (!mbar_wait(&tfull[b], ub & 1, abort_flag)) {
+                if (lane == 0) {
+                    atomicOr(p.err, kErrWaitTimeout);
+                    mc->abort = 1;
+                }
+                break;
+            }
+            tc_fence_after_sync();
+            const int tile = mc->buf_tile[b];
+            const int ss = ti % Sh::kSlots, su = ti / Sh::kSlots;
+            float lg[NQ];
+            if (tile >= 0) {
+                const uint32_t tb = tmem + (static_cast<uint32_t>(32 * qw) << 16) + b * N;
+                uint32_t r[N / 16][16];
+#pragma unroll
+                for (int c = 0; c < N / 16; ++c) tmem_ld_32x32b_x16(tb + 16 * c, r[c]);
+                tmem_wait_ld();
+#pragma unroll
+                for (int q = 0; q < NQ; ++q)
+                    lg[q] = __uint_as_float(r[q / 8][(2 * q) % 16]) +
+                            __uint_as_float(r[q / 8][(2 * q) % 16 + 1]);
+            }
+            tc_fence_before_sync();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&tempty[b]);
+            if (ti >= Sh::kSlots && !mbar_wait(&sempty[ss], (su - 1) & 1, abort_flag)) {
+                if (lane == 0) {
+                    atomicOr(p.err, kErrWaitTimeout);
+                    mc->abort = 1;
+                }
+                break;
+            }
+            if (tile >= 0) {
+                float *sc = scores + ss * NQ * kTcTile;
+#pragma unroll
+                for (int q = 0; q < NQ; ++q) sc[q * kTcTile + row] = lg[q];
+            }
+            if (warp == 2 && lane == 0) mc->slot_tile[ss] = tile;
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&sfull[ss]);
+            if (tile < 0) break;
+        }
+    } else {
+        // ---------------- selectors ----------------
+        const int sel = warp - 6;
+        if (p.sparse != nullptr) {
+            // this CTA's fixed slice of every sparse row = -inf (values come later)
+            const float ninf = __uint_as_float(0xFF800000u);
+            const int64_t base = p.V / G, rem = p.V % G;
+            const int64_t f0 = cta * base + (cta < rem ? cta : rem);
+            const int64_t fn = base + (cta < rem ? 1 : 0);
+            for (int q = 0; q < p.nq; ++q) {
+                float *rw = p.sparse + static_cast<int64_t>(q) * p.V + f0;
+                for (int64_t i = sel * 32 + lane; i < fn; i += Sh::kSelWarps * 32) rw[i] = ninf;
+            }
+        }
+        // per query of this warp: candidate count and threshold, in shared
+        // memory next to its buffer (only this warp touches them)
+        int *cnt_s = reinterpret_cast<int *>(bufs + NQ * kTcCap) + 4 * sel;
+        uint64_t *tau_s = reinterpret_cast<uint64_t *>(bufs + NQ * kTcCap) + NQ / 2 + 4 * sel;
+        if (lane < 4) {
+            cnt_s[lane] = 0;
+            tau_s[lane] = 0;
+        }
+        __syncwarp();
+        const unsigned lt_mask = (1u << lane) - 1u;
+        for (int ti = 0;; ++ti) {
+            const int ss = ti % Sh::kSlots, su = ti / Sh::kSlots;
+            if (!mbar_wait(&sfull[ss], su & 1, abort_flag)) {
+                if (lane == 0) {
+                    atomicOr(p.err, kErrWaitTimeout);
+                    mc->abort = 1;
+                }
+                break;
+            }
+            const int tile = mc->slot_tile[ss];
+            if (tile < 0) break;
+            const int64_t row0 = static_cast<int64_t>(tile) * kTcTile;
+            const int rows = static_cast<int>(min(static_cast<int64_t>(kTcTile), p.V - row0));
+            const float *sc = scores + ss * NQ * kTcTile;
+#pragma unroll 1
+            for (int j = 0; j < 4; ++j) {
+                const int q = 4 * sel + j;
+                if (q >= p.nq) break;
+                uint64_t *buf = bufs + q * kTcCap;
+                int cnt = cnt_s[j];
+                if (cnt > kTcCap - kTcTile) cnt = compact_candidates(buf, cnt, p.k, &tau_s[j], lane);
+                const uint64_t tau = tau_s[j];
+                for (int rb = 0; rb < rows; rb += 32) {
+                    const int r = rb + lane;
+                    const uint64_t key =
+                        (r < rows) ? make_key(sc[q * kTcTile + r], static_cast<uint32_t>(row0 + r)) : 0;
+                    const bool in = key > tau;
+                    const unsigned m = __ballot_sync(0xFFFFFFFFu, in);
+                    if (in) buf[cnt + __popc(m & lt_mask)] = key;
+                    cnt += __popc(m);
+                }
+                __syncwarp();
+                if (lane == 0) cnt_s[j] = cnt;
+                __syncwarp();
+            }
+            if (lane == 0) mbar_arrive(&sempty[ss]);
+        }
+#pragma unroll 1
+        for (int j = 0; j < 4; ++j) {
+            const int q = 4 * sel + j;
+            if (q >= p.nq) break;
+            uint64_t *buf = bufs + q * kTcCap;
+            const int cnt = compact_candidates(buf, cnt_s[j], p.k, &tau_s[j], lane);
+            uint64_t *dst = p.cand + (static_cast<size_t>(q) * G + cta) * p.k;
+            for (int e = lane; e < p.k; e += 32) dst[e] = e < cnt ? buf[e] : 0ull;
+        }
+    }
+
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after_sync();
+        tmem_dealloc(tmem, Sh::kTmemCols);
+    }
+}
+
+}  // namespace vie
