@@ -363,7 +363,8 @@ def main(argv=None):
     else:
         step_us = total_ms * 1e3 / K
     value = step_us / world
-    launches_per_step = -(-b // 8)  # one fused launch per query group of up to 8
+    plan = head.plan(b, k)
+    launches_per_step = plan.launches
 
     line = {
         "metric": METRIC, "value": round(value, 3), "unit": UNIT, "n_gpus": world,
@@ -373,7 +374,9 @@ def main(argv=None):
         "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": peaks["hbm_gbs"],
                      "unit": "GB/s", "frac": round(achieved / peaks["hbm_gbs"], 4),
                      "traffic": traffic, "peak_source": peak_src,
-                     "kernel": "stream_topk_kernel", "kernel_us": round(kern_us, 3),
+                     "kernel": "stream_topk_kernel" if plan.path == 0 else
+                               "tc_topk_kernel (step: prep + projection + merge)",
+                     "kernel_us": round(kern_us, 3),
                      "algorithmic_bytes_per_launch": alg_bytes,
                      "frac_of_nominal_8tbs": round(achieved / NOMINAL_HBM_GBS, 4),
                      "w_only_gbs": round(w_bytes / (kern_us * 1e-6) / 1e9, 1),

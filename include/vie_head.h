@@ -95,6 +95,17 @@ vie_status vie_head_destroy(vie_head *head);
 /* Fills *props (host) with the handle's facts. */
 vie_status vie_head_get_props(const vie_head *head, vie_head_props *props);
 
+/* How a vie_head_topk / vie_head_topk_sparse call of this size runs. */
+typedef struct {
+    int32_t path;     /* 0: streaming CUDA-core kernel, 1: tensor-core kernel  */
+    int32_t groups;   /* query groups, one pass over W_out each               */
+    int32_t launches; /* kernel launches the call enqueues                    */
+} vie_topk_plan;
+
+/* Fills *plan (host) for a call with this batch and k; the same argument
+ * checks as vie_head_topk.  Nothing is enqueued. */
+vie_status vie_head_plan(const vie_head *head, int32_t batch, int32_t k, vie_topk_plan *plan);
+
 /*
  * vie_head_topk - exact top-k of z = W_out h for a batch of queries
  * (Section 3: output projection followed by top-k selection, computed by

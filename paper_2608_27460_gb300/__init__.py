@@ -35,7 +35,7 @@ STATUS_NAMES = {0: "VIE_OK", 1: "VIE_ERR_INVALID_ARG", 2: "VIE_ERR_UNSUPPORTED",
                 3: "VIE_ERR_CUDA", 4: "VIE_ERR_OOM", 5: "VIE_ERR_DEVICE"}
 
 # Every entry point of include/vie_head.h.
-EXPORTS = ("vie_head_create", "vie_head_destroy", "vie_head_get_props", "vie_head_topk",
+EXPORTS = ("vie_head_create", "vie_head_destroy", "vie_head_get_props", "vie_head_plan", "vie_head_topk",
            "vie_head_topk_sparse", "vie_head_topk_noalloc", "vie_scatter_sparse_logits", "vie_device_status", "vie_head_device_status",
            "vie_last_error")
 
@@ -51,6 +51,10 @@ class vie_head_props(ctypes.Structure):
     _fields_ = [("V", ctypes.c_int64), ("d", ctypes.c_int32), ("d_pad", ctypes.c_int32),
                 ("ctas", ctypes.c_int32), ("device", ctypes.c_int32),
                 ("weight_bytes", ctypes.c_int64), ("scratch_bytes", ctypes.c_int64)]
+
+
+class vie_topk_plan(ctypes.Structure):
+    _fields_ = [("path", ctypes.c_int32), ("groups", ctypes.c_int32), ("launches", ctypes.c_int32)]
 
 
 _lib = None
@@ -78,6 +82,7 @@ def load(path: str | None = None, build_if_missing: bool = True):
             "vie_head_create": ([P, I64, I32, ctypes.c_int, ctypes.POINTER(P)], ctypes.c_int),
             "vie_head_destroy": ([P], ctypes.c_int),
             "vie_head_get_props": ([P, ctypes.POINTER(vie_head_props)], ctypes.c_int),
+            "vie_head_plan": ([P, I32, I32, ctypes.POINTER(vie_topk_plan)], ctypes.c_int),
             "vie_head_topk": ([P, P, I32, I32, P, P, P], ctypes.c_int),
             "vie_head_topk_sparse": ([P, P, I32, I32, P, P, P, P], ctypes.c_int),
             "vie_head_topk_noalloc": ([P, I64, I32, P, I32, I32, P, P, P], ctypes.c_int),
@@ -117,6 +122,14 @@ def vie_head_get_props(head: int):
     props = vie_head_props()
     st = load().vie_head_get_props(head, ctypes.byref(props))
     return st, props
+
+
+def vie_head_plan(head: int, batch: int, k: int):
+    """Returns (status, vie_topk_plan): path (0 streaming, 1 tensor core),
+    query groups and kernel launches of a top-k call of this size."""
+    plan = vie_topk_plan()
+    st = load().vie_head_plan(head, batch, k, ctypes.byref(plan))
+    return st, plan
 
 
 def vie_head_topk(head: int, h: int, batch: int, k: int, out_idx: int, out_logits: int,
@@ -208,6 +221,11 @@ class Head:
         check(vie_head_topk(self.handle, h.data_ptr(), b, k, out_idx.data_ptr(),
                             out_logits.data_ptr(), _stream_ptr(stream)))
         return out_idx, out_logits
+
+    def plan(self, batch: int, k: int):
+        st, pl = vie_head_plan(self.handle, batch, k)
+        check(st)
+        return pl
 
     def topk_sparse(self, h, k: int, out_idx=None, out_logits=None, out_sparse=None, stream=None):
         """Top-k and the sparse [batch, V] logit tensor in one launch."""

@@ -336,6 +336,28 @@ vie_status vie_head_get_props(const vie_head *head, vie_head_props *props) {
     return VIE_OK;
 }
 
+// The launch plan of a top-k call (path, query groups, launches).
+static bool use_tc(const vie_head *head, int32_t batch, int32_t k) {
+    return head->tc_ready && batch >= knobs().tc_min_batch && k <= vie::kTcMaxK &&
+           head->d_pad >= 64;
+}
+
+static vie_topk_plan make_plan(const vie_head *head, int32_t batch, int32_t k) {
+    vie_topk_plan pl;
+    if (use_tc(head, batch, k)) {
+        const int nqt = batch <= 8 ? 8 : (batch <= 16 ? 16 : 32);
+        pl.path = 1;
+        pl.groups = (batch + nqt - 1) / nqt;
+        pl.launches = 3 * pl.groups;  // hi/lo prep, projection + per-CTA top-k, merge
+    } else {
+        const int cap = nb_cap_for(head->d_pad, pick_mm(k));
+        pl.path = 0;
+        pl.groups = (batch + cap - 1) / cap;
+        pl.launches = pl.groups;
+    }
+    return pl;
+}
+
 // Batches on the tensor cores: per group of up to 32 queries, the hi/lo
 // query matrix, the tcgen05 projection with per-CTA top-k, and the merge.
 static vie_status run_topk_tc(const char *fn, vie_head *head, const float *h, int32_t batch,
@@ -400,8 +422,7 @@ static vie_status run_topk(const char *fn, vie_head *head, const float *h, int32
 
     const int mm = pick_mm(k);
     cudaStream_t s = static_cast<cudaStream_t>(stream);
-    if (head->tc_ready && batch >= knobs().tc_min_batch && k <= vie::kTcMaxK && head->d_pad >= 64)
-        return run_topk_tc(fn, head, h, batch, k, out_idx, out_logits, sparse, s);
+    if (use_tc(head, batch, k)) return run_topk_tc(fn, head, h, batch, k, out_idx, out_logits, sparse, s);
     const int cap = nb_cap_for(head->d_pad, mm);
     for (int q0 = 0; q0 < batch; q0 += cap) {
         const int nq = batch - q0 < cap ? batch - q0 : cap;
@@ -434,6 +455,19 @@ static vie_status run_topk(const char *fn, vie_head *head, const float *h, int32
         const cudaError_t e = vie::launch_stream_topk(nb, mm, shp.r, p, head->G, shp.smem, s);
         if (e != cudaSuccess) return fail_cuda(e, fn);
     }
+    return VIE_OK;
+}
+
+vie_status vie_head_plan(const vie_head *head, int32_t batch, int32_t k, vie_topk_plan *plan) {
+    if (head == nullptr || plan == nullptr)
+        return fail(VIE_ERR_INVALID_ARG, "vie_head_plan: NULL argument");
+    if (batch < 1 || batch > VIE_BATCH_MAX)
+        return fail(VIE_ERR_INVALID_ARG, "vie_head_plan: batch=%d outside [1, %d]", batch,
+                    VIE_BATCH_MAX);
+    if (k < 1 || k > VIE_K_MAX || static_cast<int64_t>(k) > head->V)
+        return fail(VIE_ERR_INVALID_ARG, "vie_head_plan: k=%d outside [1, min(V=%lld, %d)]", k,
+                    static_cast<long long>(head->V), VIE_K_MAX);
+    *plan = make_plan(head, batch, k);
     return VIE_OK;
 }
 

@@ -2,6 +2,8 @@
 // the tcgen05 projection + per-CTA top-k, and the per-query merge.
 #include <cuda_bf16.h>
 
+#include <utility>
+
 #include "vie_launch.h"
 #include "vie_tc_topk.cuh"
 
@@ -11,6 +13,7 @@ namespace vie {
 // rows of absent queries and columns >= d are zero.
 __global__ void prep_queries_kernel(const float *__restrict__ h, int nq, int d, int d_pad,
                                     int n_rows, __nv_bfloat16 *__restrict__ hB) {
+    griddep_launch_dependents();  // the projection kernel may start its prologue now
     const int64_t n = static_cast<int64_t>(n_rows) * d_pad;
     for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < n;
          i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
@@ -33,6 +36,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     MiscSmem *ms = reinterpret_cast<MiscSmem *>(smem);
     unsigned char *ws = smem + 256;
     const int q = blockIdx.x;
+    griddep_wait();  // the lists come from the projection kernel
     if (q == 0 && threadIdx.x == 0) *next_tile = 0;
     if (*reinterpret_cast<const volatile uint32_t *>(err) & kErrWaitTimeout) return;
     merge_queries(cand + static_cast<size_t>(q) * G * k, 1, G, k, V, ws, ws_bytes, ms,
@@ -41,6 +45,24 @@ __global__ void __launch_bounds__(kThreads, 1)
 }
 
 namespace {
+
+// Launch with programmatic stream serialisation (the kernel calls
+// griddep_wait before it touches what the previous kernel wrote).
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, uint32_t smem,
+                       cudaStream_t stream, Args &&...args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kern, std::forward<Args>(args)...);
+}
 
 template <int NQ>
 cudaError_t launch_tc_one(const CUtensorMap &mapW, const CUtensorMap &mapH, const TcParams &p,
@@ -56,8 +78,8 @@ cudaError_t launch_tc_one(const CUtensorMap &mapW, const CUtensorMap &mapH, cons
         if (e != cudaSuccess) return e;
         configured[dev] = true;
     }
-    tc_topk_kernel<NQ><<<grid, TcShape<NQ>::kThreads, smem, stream>>>(mapW, mapH, p);
-    return cudaGetLastError();
+    return launch_pdl(tc_topk_kernel<NQ>, dim3(grid), dim3(TcShape<NQ>::kThreads), smem, stream, mapW,
+                      mapH, p);
 }
 
 template <int NQ>
@@ -132,9 +154,8 @@ cudaError_t launch_merge_lists(const uint64_t *cand, int nq, int G, int k, int64
         configured[dev] = true;
     }
     const uint32_t smem = merge_kernel_smem(G, k);
-    merge_lists_kernel<<<nq, kThreads, smem, stream>>>(cand, G, k, V, out_idx, out_logits, sparse,
-                                                        next_tile, err, smem - 256u);
-    return cudaGetLastError();
+    return launch_pdl(merge_lists_kernel, dim3(nq), dim3(kThreads), smem, stream, cand, G, k, V,
+                      out_idx, out_logits, sparse, next_tile, err, smem - 256u);
 }
 
 }  // namespace vie

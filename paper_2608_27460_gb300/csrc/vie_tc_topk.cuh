@@ -18,7 +18,7 @@
 //   warps 2-5    epilogue: tcgen05.ld of the 128 x N accumulator (warp w
 //                owns TMEM lanes 32*(w%4)..), hi + lo per query, logits into
 //                a score ring laid out [query][row];
-//   warps 6..    selectors, four queries each: per query a shared buffer
+//   warps 6..    selectors, one query each (two when NQ = 32): per query a shared buffer
 //                of candidates above a threshold tau; when it passes half
 //                full, a warp-wide bitonic sort keeps the best k and raises
 //                tau (a few sorts per query instead of one insert per key).
@@ -60,7 +60,8 @@ struct TcParams {
 template <int NQ>
 struct TcShape {
     static constexpr int N = 2 * NQ;
-    static constexpr int kSelWarps = NQ / 4;
+    static constexpr int kQPW = NQ >= 32 ? 2 : 1;  // queries per selector warp
+    static constexpr int kSelWarps = NQ / kQPW;
     static constexpr int kWarps = 6 + kSelWarps;
     static constexpr int kThreads = 32 * kWarps;
     static constexpr int kStageA = kTcTile * kTcKBlock * 2;  // 16 KB per K-block of W
@@ -226,6 +227,7 @@ __global__ void __launch_bounds__(TcShape<NQ>::kThreads, 1)
     __syncthreads();
     tc_fence_after_sync();
     const uint32_t tmem = mc->tmem_base;
+    if (tid == 0) griddep_launch_dependents();  // the merge kernel may be scheduled
 
     if (warp == 0) {
         // ---------------- TMA producer ----------------
@@ -265,6 +267,7 @@ __global__ void __launch_bounds__(TcShape<NQ>::kThreads, 1)
                     for (int i = 0; i < nin; ++i)
                         tma_load_2d(st + i * Sh::kStageA, &mapW, (kb0 + i) * kTcKBlock, tile * kTcTile,
                                     &full[s], pol);
+                    if (it == 0) griddep_wait();  // the hi/lo query matrix comes from the prep kernel
                     for (int i = 0; i < nin; ++i)
                         tma_load_2d(st + KPS * Sh::kStageA + i * Sh::kStageB, &mapH,
                                     (kb0 + i) * kTcKBlock, 0, &full[s], pol);
@@ -390,6 +393,7 @@ __global__ void __launch_bounds__(TcShape<NQ>::kThreads, 1)
     } else {
         // ---------------- selectors ----------------
         const int sel = warp - 6;
+        griddep_wait();  // writes below must follow the previous kernel on the stream
         if (p.sparse != nullptr) {
             // this CTA's fixed slice of every sparse row = -inf (values come later)
             const float ninf = __uint_as_float(0xFF800000u);
@@ -403,9 +407,10 @@ __global__ void __launch_bounds__(TcShape<NQ>::kThreads, 1)
         }
         // per query of this warp: candidate count and threshold, in shared
         // memory next to its buffer (only this warp touches them)
-        int *cnt_s = reinterpret_cast<int *>(bufs + NQ * kTcCap) + 4 * sel;
-        uint64_t *tau_s = reinterpret_cast<uint64_t *>(bufs + NQ * kTcCap) + NQ / 2 + 4 * sel;
-        if (lane < 4) {
+        constexpr int QPW = Sh::kQPW;
+        int *cnt_s = reinterpret_cast<int *>(bufs + NQ * kTcCap) + QPW * sel;
+        uint64_t *tau_s = reinterpret_cast<uint64_t *>(bufs + NQ * kTcCap) + NQ / 2 + QPW * sel;
+        if (lane < QPW) {
             cnt_s[lane] = 0;
             tau_s[lane] = 0;
         }
@@ -426,8 +431,8 @@ __global__ void __launch_bounds__(TcShape<NQ>::kThreads, 1)
             const int rows = static_cast<int>(min(static_cast<int64_t>(kTcTile), p.V - row0));
             const float *sc = scores + ss * NQ * kTcTile;
 #pragma unroll 1
-            for (int j = 0; j < 4; ++j) {
-                const int q = 4 * sel + j;
+            for (int j = 0; j < QPW; ++j) {
+                const int q = QPW * sel + j;
                 if (q >= p.nq) break;
                 uint64_t *buf = bufs + q * kTcCap;
                 int cnt = cnt_s[j];
@@ -449,8 +454,8 @@ __global__ void __launch_bounds__(TcShape<NQ>::kThreads, 1)
             if (lane == 0) mbar_arrive(&sempty[ss]);
         }
 #pragma unroll 1
-        for (int j = 0; j < 4; ++j) {
-            const int q = 4 * sel + j;
+        for (int j = 0; j < QPW; ++j) {
+            const int q = QPW * sel + j;
             if (q >= p.nq) break;
             uint64_t *buf = bufs + q * kTcCap;
             const int cnt = compact_candidates(buf, cnt_s[j], p.k, &tau_s[j], lane);
