@@ -34,7 +34,14 @@ METRIC = "output-head µs/decode-step at batch 1; achieved HBM GB/s vs 8 TB/s pe
 UNIT = "us/step"
 NOMINAL_HBM_GBS = 8000.0
 PROFILE_DIR = os.path.join(ROOT, "profiles")
-KERNEL_SOURCES = ["vie_stream_topk.cuh", "vie_device.cuh", "vie_stream_topk_inst.cuh"]
+# Sources each profiled kernel is built from: a committed ncu summary names
+# the digest of these files, and its traffic figure is used only while the
+# digest still matches.
+KERNEL_SOURCES = {
+    "stream_topk": ["vie_stream_topk.cuh", "vie_device.cuh", "vie_stream_topk_inst.cuh"],
+    "tc_topk": ["vie_tc_topk.cuh", "vie_tc_topk.cu", "vie_tcgen05.cuh", "vie_device.cuh",
+                "vie_stream_topk.cuh"],
+}
 
 
 def parse_args(argv=None):
@@ -66,9 +73,9 @@ def dist_env():
     return rank, world, local
 
 
-def kernel_source_digest() -> str:
+def kernel_source_digest(kernel: str = "stream_topk") -> str:
     h = hashlib.sha256()
-    for f in KERNEL_SOURCES:
+    for f in KERNEL_SOURCES[kernel]:
         with open(os.path.join(ROOT, "paper_2608_27460_gb300", "csrc", f), "rb") as fh:
             h.update(fh.read())
     return h.hexdigest()[:16]
@@ -82,10 +89,10 @@ def measured_peaks():
     return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}, "fallback"
 
 
-def profiled_traffic(workload: str, batch: int, k: int):
+def profiled_traffic(kernel: str, workload: str, batch: int, k: int):
     """dram bytes per launch of the projection kernel from a committed ncu
     summary, if it was taken on the current kernel source; else None."""
-    path = os.path.join(PROFILE_DIR, f"stream_topk_{workload}_b{batch}_k{k}.md")
+    path = os.path.join(PROFILE_DIR, f"{kernel}_{workload}_b{batch}_k{k}.md")
     if not os.path.exists(path):
         return None, None
     text = open(path).read()
@@ -93,7 +100,7 @@ def profiled_traffic(workload: str, batch: int, k: int):
     m_b = re.search(r"dram_bytes_per_launch:\s*([0-9]+)", text)
     if not m_src or not m_b:
         return None, path
-    if m_src.group(1) != kernel_source_digest():
+    if m_src.group(1) != kernel_source_digest(kernel):
         return None, path
     return int(m_b.group(1)), path
 
@@ -357,13 +364,14 @@ def main(argv=None):
     w_bytes = shape.V * props.d_pad * 2
     alg_bytes = w_bytes + b * shape.d * 4 + b * k * 8
     achieved = alg_bytes / (kern_us * 1e-6) / 1e9
-    traffic, prof_path = profiled_traffic(args.workload, b, k)
+    plan = head.plan(b, k)
+    kernel = "stream_topk" if plan.path == 0 else "tc_topk"
+    traffic, prof_path = profiled_traffic(kernel, args.workload, b, k)
     if flush is not None:
         step_us = statistics.mean(kern_ms) * 1e3  # the flush between steps is not head time
     else:
         step_us = total_ms * 1e3 / K
     value = step_us / world
-    plan = head.plan(b, k)
     launches_per_step = plan.launches
 
     line = {
@@ -376,6 +384,7 @@ def main(argv=None):
                      "traffic": traffic, "peak_source": peak_src,
                      "kernel": "stream_topk_kernel" if plan.path == 0 else
                                "tc_topk_kernel (step: prep + projection + merge)",
+                     "profile": os.path.relpath(prof_path, ROOT) if prof_path else None,
                      "kernel_us": round(kern_us, 3),
                      "algorithmic_bytes_per_launch": alg_bytes,
                      "frac_of_nominal_8tbs": round(achieved / NOMINAL_HBM_GBS, 4),
@@ -387,6 +396,19 @@ def main(argv=None):
         "gpu_launches": K * launches_per_step,
         "clocks": ClockSampler.summarize(clocks, t_wall0, t_wall1),
     }
+    if plan.path == 1:
+        # the batched path against the bf16 tensor-core roofline as well:
+        # algorithmic flops 2*V*d*b; the MMAs issue 2*V*d_pad*(2 rows per
+        # query: hi and lo halves of h) over the padded query group
+        alg_flops = 2.0 * shape.V * shape.d * b
+        nq_tile = 8 if b <= 8 else (16 if b <= 16 else 32)
+        issued = 2.0 * shape.V * props.d_pad * 2 * nq_tile * plan.groups
+        tf = alg_flops / (kern_us * 1e-6) / 1e12
+        line["roofline_tensor"] = {
+            "bound": "tensor", "achieved": round(tf, 2), "peak": peaks["bf16_tflops"],
+            "unit": "TFLOP/s", "frac": round(tf / peaks["bf16_tflops"], 5),
+            "issued_mma_tflops": round(issued / (kern_us * 1e-6) / 1e12, 2),
+            "peak_source": peak_src}
     if not args.no_cpu_baseline and world == 1:
         us, n, threads, results = cpu_oracle_sample(W, h, k, args.cpu_seconds, b)
         line["cpu_baseline"] = {"value": round(us, 1), "unit": UNIT, "cores": threads, "kind": "oracle",
