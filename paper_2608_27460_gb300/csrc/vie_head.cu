@@ -146,13 +146,13 @@ int env_int(const char *name, int dflt) {
 //   VIE_STAGE_MIN_KB     smallest weight stage worth one bulk copy (48)
 //   VIE_STATIC_PCT       share of the chunks assigned statically, in % (85)
 //   VIE_TC_MIN_BATCH     smallest batch sent to the tensor-core path (2)
-//   VIE_TC_KPS           K-blocks of 64 columns per tensor-core ring stage (2)
+//   VIE_TC_KPS           K-blocks of 64 columns per tensor-core ring stage (4)
 struct Knobs {
     int stage_min_bytes, static_pct, tc_min_batch, tc_kps;
 };
 const Knobs &knobs() {
     static const Knobs k = {env_int("VIE_STAGE_MIN_KB", 48) * 1024, env_int("VIE_STATIC_PCT", 85),
-                            env_int("VIE_TC_MIN_BATCH", 2), env_int("VIE_TC_KPS", 2)};
+                            env_int("VIE_TC_MIN_BATCH", 2), env_int("VIE_TC_KPS", 4)};
     return k;
 }
 

@@ -4,7 +4,7 @@
 //
 // h is fp32; tcgen05 kind::f16 needs both operands in bf16, so each query
 // enters as two bf16 columns hi = rn(h), lo = rn(h - hi) and its logit is the
-// sum of the two accumulator columns (residual error <= 2^-18 |h| per term).
+// sum of the two accumulator columns (residual error <= 2^-16 |h| per term).
 // N = 2 * NQ accumulator columns per tile.
 //
 // One persistent CTA per SM walks 128-row tiles of W (round robin, then an
@@ -20,8 +20,8 @@
 //                a score ring laid out [query][row];
 //   warps 6..    selectors, one query each (two when NQ = 32): per query a shared buffer
 //                of candidates above a threshold tau; when it passes half
-//                full, a warp-wide bitonic sort keeps the best k and raises
-//                tau (a few sorts per query instead of one insert per key).
+//                full, a warp-wide bisection keeps the best k (unsorted) and
+//                raises tau; one bitonic sort of the final k per query.
 // Each CTA writes its per-query lists; a separate merge kernel (one CTA per
 // query) merges them.  All waits are bounded.
 #pragma once
@@ -136,37 +136,87 @@ __device__ __forceinline__ void warp_sort_desc(uint64_t (&v)[PER], int lane) {
     }
 }
 
-// Keeps the best min(k, cnt) of the cnt keys in buf (sorted descending at
-// buf[0..)), returns the new count; *tau becomes the k-th key once k are
-// held.  Out of line: one copy of the sorting network serves every call.
-static __device__ __noinline__ int compact_candidates(uint64_t *buf, int cnt, int k, uint64_t *tau,
-                                               int lane) {
+// Keeps the k largest of the cnt (> k) nonzero keys in buf, unsorted at
+// buf[0..k), and returns k; *tau becomes a bound T <= the k-th key such that
+// exactly k keys are >= T.  T is found by bisection: first on the high words
+// (the logit order), then, only if several keys tie on the k-th high word,
+// on the low words (the row order) among the tied keys.  Out of line and
+// loop-based: a few hundred instructions, and little code next to the
+// latency-critical producer and MMA loops.
+static __device__ __noinline__ int keep_best(uint64_t *buf, int cnt, int k, uint64_t *tau, int lane) {
     constexpr int PER = kTcCap / 32;
+    uint64_t v[PER];
+#pragma unroll
+    for (int j = 0; j < PER; ++j) {
+        const int e = j * 32 + lane;
+        v[j] = e < cnt ? buf[e] : 0ull;  // 0 is below every key
+    }
+    uint32_t th = 0;
+#pragma unroll 1
+    for (int bit = 31; bit >= 0; --bit) {
+        const uint32_t c = th | (1u << bit);
+        int n = 0;
+#pragma unroll
+        for (int j = 0; j < PER; ++j) n += static_cast<uint32_t>(v[j] >> 32) >= c ? 1 : 0;
+        if (static_cast<int>(__reduce_add_sync(0xFFFFFFFFu, n)) >= k) th = c;
+    }
+    int n_gt = 0, n_ge = 0;
+#pragma unroll
+    for (int j = 0; j < PER; ++j) {
+        const uint32_t hi = static_cast<uint32_t>(v[j] >> 32);
+        n_gt += hi > th ? 1 : 0;
+        n_ge += hi >= th ? 1 : 0;
+    }
+    n_gt = static_cast<int>(__reduce_add_sync(0xFFFFFFFFu, n_gt));
+    n_ge = static_cast<int>(__reduce_add_sync(0xFFFFFFFFu, n_ge));
+    uint32_t tl = 0;
+    if (n_ge > k) {
+        // ties on the k-th logit: the (k - n_gt) largest low words among them
+        const int need = k - n_gt;
+#pragma unroll 1
+        for (int bit = 31; bit >= 0; --bit) {
+            const uint32_t c = tl | (1u << bit);
+            int n = 0;
+#pragma unroll
+            for (int j = 0; j < PER; ++j)
+                n += (static_cast<uint32_t>(v[j] >> 32) == th && static_cast<uint32_t>(v[j]) >= c) ? 1 : 0;
+            if (static_cast<int>(__reduce_add_sync(0xFFFFFFFFu, n)) >= need) tl = c;
+        }
+    }
+    const uint64_t T = (static_cast<uint64_t>(th) << 32) | tl;
+    __syncwarp();
+    const unsigned lt_mask = (1u << lane) - 1u;
+    int base = 0;
+#pragma unroll
+    for (int j = 0; j < PER; ++j) {
+        const bool in = v[j] >= T;
+        const unsigned m = __ballot_sync(0xFFFFFFFFu, in);
+        if (in) buf[base + __popc(m & lt_mask)] = v[j];
+        base += __popc(m);
+    }
+    if (lane == 0) *tau = T;
+    __syncwarp();
+    return k;
+}
+
+// The final list of one query: the best min(k, cnt) keys of buf, sorted
+// descending, written to dst[0..k) (zeros after them).
+static __device__ __noinline__ void write_sorted_list(uint64_t *buf, int cnt, int k, uint64_t *tau,
+                                                      uint64_t *dst, int lane) {
+    if (cnt > k) cnt = keep_best(buf, cnt, k, tau, lane);
+    constexpr int PER = kTcMaxK / 32;  // cnt <= k <= kTcMaxK
     uint64_t v[PER];
 #pragma unroll
     for (int j = 0; j < PER; ++j) {
         const int e = lane * PER + j;
         v[j] = e < cnt ? buf[e] : 0ull;
     }
-    __syncwarp();
     warp_sort_desc<PER>(v, lane);
-    const int keep = cnt < k ? cnt : k;
 #pragma unroll
     for (int j = 0; j < PER; ++j) {
         const int e = lane * PER + j;
-        if (e < keep) buf[e] = v[j];
+        if (e < k) dst[e] = v[j];
     }
-    if (keep == k) {
-        uint64_t x = 0;
-        const int slot = (k - 1) % PER;
-#pragma unroll
-        for (int j = 0; j < PER; ++j)
-            if (j == slot) x = v[j];
-        x = shfl_u64(x, (k - 1) / PER);
-        if (lane == 0) *tau = x;
-    }
-    __syncwarp();
-    return keep;
 }
 
 template <int NQ>
@@ -436,7 +486,7 @@ __global__ void __launch_bounds__(TcShape<NQ>::kThreads, 1)
                 if (q >= p.nq) break;
                 uint64_t *buf = bufs + q * kTcCap;
                 int cnt = cnt_s[j];
-                if (cnt > kTcCap - kTcTile) cnt = compact_candidates(buf, cnt, p.k, &tau_s[j], lane);
+                if (cnt > kTcCap - kTcTile) cnt = keep_best(buf, cnt, p.k, &tau_s[j], lane);
                 const uint64_t tau = tau_s[j];
                 for (int rb = 0; rb < rows; rb += 32) {
                     const int r = rb + lane;
@@ -457,10 +507,8 @@ __global__ void __launch_bounds__(TcShape<NQ>::kThreads, 1)
         for (int j = 0; j < QPW; ++j) {
             const int q = QPW * sel + j;
             if (q >= p.nq) break;
-            uint64_t *buf = bufs + q * kTcCap;
-            const int cnt = compact_candidates(buf, cnt_s[j], p.k, &tau_s[j], lane);
-            uint64_t *dst = p.cand + (static_cast<size_t>(q) * G + cta) * p.k;
-            for (int e = lane; e < p.k; e += 32) dst[e] = e < cnt ? buf[e] : 0ull;
+            write_sorted_list(bufs + q * kTcCap, cnt_s[j], p.k, &tau_s[j],
+                              p.cand + (static_cast<size_t>(q) * G + cta) * p.k, lane);
         }
     }
 
