@@ -38,6 +38,10 @@ __device__ uint32_t g_dev_err = 0;
 
 constexpr int kMaxSmem = 232448;  // 227 KB opt-in dynamic shared memory per CTA
 constexpr int kMaxNB = 8;
+// The tensor-core path keeps [32][G][k <= 128] lists and [32][G][4] heads in
+// the same scratch as the streaming path's [kMaxNB][G][VIE_K_MAX] lists.
+static_assert((vie::kTcHRows / 2) * (vie::kTcMaxK + vie::kTcMergeE) <= kMaxNB * VIE_K_MAX,
+              "tensor-core lists must fit the candidate scratch");
 constexpr int kMaxHBytes = 64 * 1024;  // shared-memory budget for staged queries
 
 }  // namespace
@@ -50,7 +54,8 @@ struct vie_head {
     int G;
     uint16_t *W;        // [V, d_pad] bf16 bits
     uint64_t *cand;     // [kMaxNB][G][VIE_K_MAX] ranking keys
-    uint32_t *words;    // [0] completion ticket, [1] device flag word, [2] chunk pool counter
+    uint32_t *words;    // [0] completion ticket, [1] device flag word, [2] chunk pool counter,
+                        // [3] merging CTAs done (tensor-core path)
     int64_t scratch_bytes;
     // tensor-core path (batches): hi/lo bf16 query matrix and TMA descriptors
     void *hB;             // [kTcHRows][d_pad] bf16
@@ -348,7 +353,7 @@ static vie_topk_plan make_plan(const vie_head *head, int32_t batch, int32_t k) {
         const int nqt = batch <= 8 ? 8 : (batch <= 16 ? 16 : 32);
         pl.path = 1;
         pl.groups = (batch + nqt - 1) / nqt;
-        pl.launches = 3 * pl.groups;  // hi/lo prep, projection + per-CTA top-k, merge
+        pl.launches = 2 * pl.groups;  // hi/lo prep; projection, per-CTA top-k and merge
     } else {
         const int cap = nb_cap_for(head->d_pad, pick_mm(k));
         pl.path = 0;
@@ -359,7 +364,7 @@ static vie_topk_plan make_plan(const vie_head *head, int32_t batch, int32_t k) {
 }
 
 // Batches on the tensor cores: per group of up to 32 queries, the hi/lo
-// query matrix, the tcgen05 projection with per-CTA top-k, and the merge.
+// query matrix, then the tcgen05 projection with per-CTA top-k and the merge.
 static vie_status run_topk_tc(const char *fn, vie_head *head, const float *h, int32_t batch,
                               int32_t k, int32_t *out_idx, float *out_logits, float *sparse,
                               cudaStream_t s) {
@@ -388,16 +393,16 @@ static vie_status run_topk_tc(const char *fn, vie_head *head, const float *h, in
         p.stages = stages;
         p.kb_per_stage = kps;
         p.static_tiles = static_cast<int32_t>(static_cast<int64_t>(n_tiles) * pct / 100 / head->G);
-        p.cand = head->cand;
+        p.cand = head->cand;  // [32][G][k <= 128] keys, then the lists' heads
+        p.heads = head->cand + static_cast<size_t>(vie::kTcHRows / 2) * head->G * vie::kTcMaxK;
+        p.ticket = head->words;
         p.next_tile = head->words + 2;
+        p.merged = head->words + 3;
         p.err = head->words + 1;
+        p.out_idx = out_idx + static_cast<int64_t>(q0) * k;
+        p.out_logits = out_logits + static_cast<int64_t>(q0) * k;
         p.sparse = sparse != nullptr ? sparse + static_cast<int64_t>(q0) * head->V : nullptr;
         e = vie::launch_tc_topk(nqt, head->mapW, mapH, p, head->G, smem, s);
-        if (e != cudaSuccess) return fail_cuda(e, fn);
-        e = vie::launch_merge_lists(head->cand, nq, head->G, k, head->V,
-                                    out_idx + static_cast<int64_t>(q0) * k,
-                                    out_logits + static_cast<int64_t>(q0) * k, p.sparse,
-                                    head->words + 2, head->words + 1, s);
         if (e != cudaSuccess) return fail_cuda(e, fn);
     }
     return VIE_OK;

@@ -40,9 +40,4 @@ cudaError_t launch_tc_topk(int nq_tmpl, const CUtensorMap &mapW, const CUtensorM
 cudaError_t launch_prep_queries(const float *h, int nq, int d, int d_pad, int n_rows, void *hB,
                                 int sms, cudaStream_t stream);
 
-// One CTA per query: merges the per-CTA lists of nq queries.
-cudaError_t launch_merge_lists(const uint64_t *cand, int nq, int G, int k, int64_t V,
-                               int32_t *out_idx, float *out_logits, float *sparse,
-                               uint32_t *next_tile, const uint32_t *err, cudaStream_t stream);
-
 }  // namespace vie

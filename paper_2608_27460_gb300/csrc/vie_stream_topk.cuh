@@ -158,7 +158,8 @@ struct WarpList {
 };
 
 // --------------------------------------------------------------------------
-// Block-wide helpers for the merge (all kThreads threads call them).
+// Block-wide helpers for the merge: every thread of the CTA calls them, for
+// any block size of at least 32 threads (merge_queries: at least kThreads).
 
 struct SmemKeys {
     const uint64_t *p;
@@ -182,9 +183,9 @@ __device__ uint64_t block_radix_threshold(Keys keys, int n, int k, uint64_t lo, 
     uint64_t prefix = 0, mask = 0;
     int remaining = k;
     for (int shift = 56; shift >= 0; shift -= 8) {
-        for (int i = tid; i < 256; i += kThreads) hist[i] = 0;
+        for (int i = tid; i < 256; i += static_cast<int>(blockDim.x)) hist[i] = 0;
         __syncthreads();
-        for (int i = tid; i < n; i += kThreads) {
+        for (int i = tid; i < n; i += static_cast<int>(blockDim.x)) {
             const uint64_t x = keys[i];
             if (x >= lo && x != 0 && (x & mask) == prefix)
                 atomicAdd(&hist[(x >> shift) & 255u], 1u);
@@ -262,7 +263,7 @@ __device__ inline void block_topk_to_output(const uint64_t *keys, int n, int k, 
         const uint64_t T = block_radix_threshold(SmemKeys{keys}, n, k, 1, hist, ms);
         if (tid == 0) ms->n_win = 0;
         __syncthreads();
-        for (int i = tid; i < n; i += kThreads) {
+        for (int i = tid; i < n; i += static_cast<int>(blockDim.x)) {
             const uint64_t x = keys[i];
             if (x >= T) win[atomicAdd(&ms->n_win, 1)] = x;
         }
@@ -270,7 +271,7 @@ __device__ inline void block_topk_to_output(const uint64_t *keys, int n, int k, 
         src = win;
         m = k;
     }
-    for (int i = tid; i < m; i += kThreads) {
+    for (int i = tid; i < m; i += static_cast<int>(blockDim.x)) {
         const uint64_t x = src[i];
         const int rank = rank_among(src, m, x);
         if (rank < k) {
@@ -302,14 +303,14 @@ __device__ void merge_lists(Keys lists, int G, int k, const MergeBufs &mb, MiscS
     uint64_t tau = 0;
     const bool have_pref = P <= kMergePrefixCap;
     if (have_pref) {
-        for (int i = tid; i < P; i += kThreads) {
+        for (int i = tid; i < P; i += static_cast<int>(blockDim.x)) {
             const int c = i / J, j = i - c * J;
             mb.pref[i] = lists[c * k + j];
         }
         if (tid == 0) ms->tau = 0;
         __syncthreads();
         if (P <= kRankCountMax) {
-            for (int i = tid; i < P; i += kThreads) {
+            for (int i = tid; i < P; i += static_cast<int>(blockDim.x)) {
                 const uint64_t x = mb.pref[i];
                 if (x != 0 && rank_among(mb.pref, P, x) == k - 1) ms->tau = x;
             }
@@ -325,7 +326,7 @@ __device__ void merge_lists(Keys lists, int G, int k, const MergeBufs &mb, MiscS
     //    first J entries are in the prefix buffer, deeper entries are read
     //    eight at a time with independent loads.
     const uint64_t lo = tau > 0 ? tau : 1;
-    for (int c = tid; c < G; c += kThreads) {
+    for (int c = tid; c < G; c += static_cast<int>(blockDim.x)) {
         int n = 0;
         if (have_pref)
             while (n < J && mb.pref[c * J + n] >= lo) ++n;
@@ -365,7 +366,7 @@ __device__ void merge_lists(Keys lists, int G, int k, const MergeBufs &mb, MiscS
     const int M = ms->n_cand;
     if (M <= kMergeCandCap) {
         // 3a. gather the candidates, exact top-k among them
-        for (int c = tid; c < G; c += kThreads)
+        for (int c = tid; c < G; c += static_cast<int>(blockDim.x))
             for (int j = 0; j < mb.counts[c]; ++j)
                 mb.cands[mb.offsets[c] + j] =
                     (have_pref && j < J) ? mb.pref[c * J + j] : lists[c * k + j];
@@ -376,7 +377,7 @@ __device__ void merge_lists(Keys lists, int G, int k, const MergeBufs &mb, MiscS
         const uint64_t T = block_radix_threshold(lists, G * k, k, lo, mb.hist, ms);
         if (tid == 0) ms->n_win = 0;
         __syncthreads();
-        for (int i = tid; i < G * k; i += kThreads) {
+        for (int i = tid; i < G * k; i += static_cast<int>(blockDim.x)) {
             const uint64_t x = lists[i];
             if (x >= T && x >= lo) mb.win[atomicAdd(&ms->n_win, 1)] = x;
         }
@@ -403,7 +404,7 @@ __device__ inline bool merge_fast_query(const uint64_t *fe, const uint32_t *hv, 
         ms->n_cand = 0;
         ms->overflow = 0;
     }
-    for (int i = tid; i < kFastE * kThreads / 2; i += kThreads) rank_part[i] = 0;  // M <= G * kFastE
+    for (int i = tid; i < kFastE * kThreads / 2; i += static_cast<int>(blockDim.x)) rank_part[i] = 0;  // M <= G * kFastE
     __syncthreads();
     // tau: thread pair (2c, 2c+1) counts the heads >= head c, half each
     {
@@ -452,7 +453,7 @@ __device__ inline bool merge_fast_query(const uint64_t *fe, const uint32_t *hv, 
     // slice of the candidates; partial counts meet in shared memory
     constexpr int kRankSplit = 5;
     const int per = (M + kRankSplit - 1) / kRankSplit;
-    for (int t = tid; t < M * kRankSplit; t += kThreads) {
+    for (int t = tid; t < M * kRankSplit; t += static_cast<int>(blockDim.x)) {
         const int i = t % M, part = t / M;
         const uint64_t x = cands[i];
         const int j0 = part * per, j1 = min(M, j0 + per);
@@ -462,7 +463,7 @@ __device__ inline bool merge_fast_query(const uint64_t *fe, const uint32_t *hv, 
         if (r) atomicAdd(&rank_part[i], r);
     }
     __syncthreads();
-    for (int i = tid; i < M; i += kThreads) {
+    for (int i = tid; i < M; i += static_cast<int>(blockDim.x)) {
         const int rank = rank_part[i];
         if (rank < k) {
             const uint64_t x = cands[i];
@@ -482,7 +483,7 @@ __device__ inline bool merge_fast_query(const uint64_t *fe, const uint32_t *hv, 
 // Small k: one pass of independent L2 loads fetches the first kFastE
 // entries of every list of every query (thread c: list c), then each query
 // is merged in shared memory; a query the fast merge cannot settle is merged
-// in full.  Called by all kThreads threads of one CTA.
+// in full.  Called by every thread of one CTA of at least kThreads threads.
 __device__ inline void merge_queries(const uint64_t *cand, int nq, int G, int k, int64_t V,
                                      unsigned char *ws, uint32_t merge_bytes, MiscSmem *ms,
                                      int32_t *out_idx, float *out_logits, float *sparse) {
@@ -542,10 +543,10 @@ __device__ inline void merge_queries(const uint64_t *cand, int nq, int G, int k,
             if ((reinterpret_cast<uintptr_t>(src) & 15u) == 0) {
                 const ulonglong2 *src2 = reinterpret_cast<const ulonglong2 *>(src);
                 ulonglong2 *dst2 = reinterpret_cast<ulonglong2 *>(staged);
-                for (int i = tid; i < (n_all >> 1); i += kThreads) dst2[i] = __ldcg(src2 + i);
+                for (int i = tid; i < (n_all >> 1); i += static_cast<int>(blockDim.x)) dst2[i] = __ldcg(src2 + i);
                 if ((n_all & 1) && tid == 0) staged[n_all - 1] = __ldcg(src + n_all - 1);
             } else {
-                for (int i = tid; i < n_all; i += kThreads) staged[i] = __ldcg(src + i);
+                for (int i = tid; i < n_all; i += static_cast<int>(blockDim.x)) staged[i] = __ldcg(src + i);
             }
             __syncthreads();
             merge_lists(SmemKeys{staged}, G, k, mb, ms, oi, ol, sp);

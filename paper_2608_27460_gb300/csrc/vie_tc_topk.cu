@@ -1,5 +1,5 @@
-// vie_tc_topk.cu - launchers of the tensor-core head: hi/lo query prep,
-// the tcgen05 projection + per-CTA top-k, and the per-query merge.
+// vie_tc_topk.cu - launchers of the tensor-core head: hi/lo query prep, and
+// the tcgen05 projection with per-CTA top-k and the merge in its last CTA.
 #include <cuda_bf16.h>
 
 #include <utility>
@@ -23,25 +23,6 @@ __global__ void prep_queries_kernel(const float *__restrict__ h, int nq, int d, 
         const __nv_bfloat16 hi = __float2bfloat16_rn(x);
         hB[i] = (r & 1) ? __float2bfloat16_rn(x - __bfloat162float(hi)) : hi;
     }
-}
-
-// One CTA per query: merges the G per-CTA lists of query blockIdx.x.  Runs
-// after tc_topk_kernel on the same stream; re-arms the tile pool counter.
-__global__ void __launch_bounds__(kThreads, 1)
-    merge_lists_kernel(const uint64_t *cand, int G, int k, int64_t V, int32_t *out_idx,
-                       float *out_logits, float *sparse, uint32_t *next_tile, const uint32_t *err,
-                       uint32_t ws_bytes) {
-    extern __shared__ __align__(1024) unsigned char tc_smem[];
-    unsigned char *smem = tc_smem;
-    MiscSmem *ms = reinterpret_cast<MiscSmem *>(smem);
-    unsigned char *ws = smem + 256;
-    const int q = blockIdx.x;
-    griddep_wait();  // the lists come from the projection kernel
-    if (q == 0 && threadIdx.x == 0) *next_tile = 0;
-    if (*reinterpret_cast<const volatile uint32_t *>(err) & kErrWaitTimeout) return;
-    merge_queries(cand + static_cast<size_t>(q) * G * k, 1, G, k, V, ws, ws_bytes, ms,
-                  out_idx + static_cast<size_t>(q) * k, out_logits + static_cast<size_t>(q) * k,
-                  sparse != nullptr ? sparse + static_cast<int64_t>(q) * V : nullptr);
 }
 
 namespace {
@@ -129,33 +110,6 @@ cudaError_t launch_prep_queries(const float *h, int nq, int d, int d_pad, int n_
     prep_queries_kernel<<<static_cast<unsigned>(blocks), 256, 0, stream>>>(
         h, nq, d, d_pad, n_rows, static_cast<__nv_bfloat16 *>(hB));
     return cudaGetLastError();
-}
-
-uint32_t merge_kernel_smem(int G, int k) {
-    const uint32_t stage = static_cast<uint32_t>(G) * k * 8;
-    const uint32_t fast = static_cast<uint32_t>(G) * (kFastE * 8 + 4) + 64;
-    const uint32_t ws = SmemLayout::merge_fixed_bytes() + (stage > fast ? stage : fast);
-    const uint32_t cap = 232448u - 256u;
-    return 256u + (ws < cap ? ws : cap);
-}
-
-cudaError_t launch_merge_lists(const uint64_t *cand, int nq, int G, int k, int64_t V,
-                               int32_t *out_idx, float *out_logits, float *sparse,
-                               uint32_t *next_tile, const uint32_t *err, cudaStream_t stream) {
-    static bool configured[64] = {};
-    int dev = 0;
-    cudaError_t e = cudaGetDevice(&dev);
-    if (e != cudaSuccess) return e;
-    if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
-    if (!configured[dev]) {
-        e = cudaFuncSetAttribute(merge_lists_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 232448);
-        if (e != cudaSuccess) return e;
-        configured[dev] = true;
-    }
-    const uint32_t smem = merge_kernel_smem(G, k);
-    return launch_pdl(merge_lists_kernel, dim3(nq), dim3(kThreads), smem, stream, cand, G, k, V,
-                      out_idx, out_logits, sparse, next_tile, err, smem - 256u);
 }
 
 }  // namespace vie

@@ -22,8 +22,8 @@
 //                of candidates above a threshold tau; when it passes half
 //                full, a warp-wide bisection keeps the best k (unsorted) and
 //                raises tau; one bitonic sort of the final k per query.
-// Each CTA writes its per-query lists; a separate merge kernel (one CTA per
-// query) merges them.  All waits are bounded.
+// Each CTA writes its per-query lists and takes a completion ticket; the
+// last CTAs to finish merge them, one query each.  All waits are bounded.
 #pragma once
 
 #include <cuda.h>
@@ -42,6 +42,8 @@ constexpr int kTcHRows = 64;       // rows of the hi/lo query matrix (N <= 64)
 constexpr int kTcCap = 256;        // candidate buffer per query (>= k + one tile)
 constexpr int kTcMaxK = kTcCap - kTcTile;  // largest k of this path
 constexpr int kTcMaxKPS = 4;       // K-blocks per stage, at most
+constexpr int kTcMergeE = 4;       // merge: keys per list in the heads area
+constexpr int kTcMaxMergers = 32;  // CTAs that merge, at most (one per query)
 
 struct TcParams {
     int64_t V;
@@ -52,8 +54,13 @@ struct TcParams {
     int32_t static_tiles;    // tiles each CTA owns before drawing from the pool
     int32_t kb_per_stage;    // K-blocks per ring stage (1..kTcMaxKPS)
     uint64_t *cand;          // [NQ][G][k] keys
-    uint32_t *next_tile;     // pool counter (reset by the merge kernel)
+    uint64_t *heads;         // [NQ][G][kTcMergeE]: the first keys of each list
+    uint32_t *ticket;        // CTA completion counter (self-resetting)
+    uint32_t *next_tile;     // pool counter (self-resetting)
+    uint32_t *merged;        // merging CTAs done (self-resetting)
     uint32_t *err;           // device flag word
+    int32_t *out_idx;        // [nq, k]
+    float *out_logits;       // [nq, k]
     float *sparse;           // [nq, V] fp32 or nullptr: slices filled with -inf here
 };
 
@@ -79,6 +86,7 @@ struct TcMisc {
     int stage_tile[kTcMaxStages];  // tile of a stage that starts a tile (-1: end)
     int buf_tile[2];               // tile held by each TMEM accumulator
     int slot_tile[kTcScoreSlots];  // tile of each score slot
+    int merger;                    // m >= 0: this CTA merges queries m, m + X, ...
 };
 
 struct TcSmemLayout {
@@ -200,9 +208,10 @@ static __device__ __noinline__ int keep_best(uint64_t *buf, int cnt, int k, uint
 }
 
 // The final list of one query: the best min(k, cnt) keys of buf, sorted
-// descending, written to dst[0..k) (zeros after them).
+// descending, written to dst[0..k) (zeros after them), and its first
+// kTcMergeE keys also to head[0..kTcMergeE).
 static __device__ __noinline__ void write_sorted_list(uint64_t *buf, int cnt, int k, uint64_t *tau,
-                                                      uint64_t *dst, int lane) {
+                                                      uint64_t *dst, uint64_t *head, int lane) {
     if (cnt > k) cnt = keep_best(buf, cnt, k, tau, lane);
     constexpr int PER = kTcMaxK / 32;  // cnt <= k <= kTcMaxK
     uint64_t v[PER];
@@ -216,6 +225,7 @@ static __device__ __noinline__ void write_sorted_list(uint64_t *buf, int cnt, in
     for (int j = 0; j < PER; ++j) {
         const int e = lane * PER + j;
         if (e < k) dst[e] = v[j];
+        if (e < kTcMergeE) head[e] = v[j];
     }
 }
 
@@ -508,7 +518,8 @@ __global__ void __launch_bounds__(TcShape<NQ>::kThreads, 1)
             const int q = QPW * sel + j;
             if (q >= p.nq) break;
             write_sorted_list(bufs + q * kTcCap, cnt_s[j], p.k, &tau_s[j],
-                              p.cand + (static_cast<size_t>(q) * G + cta) * p.k, lane);
+                              p.cand + (static_cast<size_t>(q) * G + cta) * p.k,
+                              p.heads + (static_cast<size_t>(q) * G + cta) * kTcMergeE, lane);
         }
     }
 
@@ -516,6 +527,79 @@ __global__ void __launch_bounds__(TcShape<NQ>::kThreads, 1)
     if (warp == 1) {
         tc_fence_after_sync();
         tmem_dealloc(tmem, Sh::kTmemCols);
+    }
+
+    // ---------------- completion ticket ----------------
+    // bar.sync orders every thread's writes (lists, heads, sparse fill)
+    // before thread 0's release.  The last X CTAs to take a ticket merge: each
+    // waits until every CTA has taken one (an acquire of the final count,
+    // which follows every release), then merges queries m, m + X, ... with the
+    // whole CTA; the last of them to finish re-arms the counters.
+    const int X = min(p.nq, min(G, kTcMaxMergers));
+    if (tid == 0) {
+        const uint32_t ticket = atomic_add_acq_rel_gpu(p.ticket, 1u);
+        const int m = static_cast<int>(ticket) - (G - X);
+        mc->merger = m;
+        if (m >= 0) {
+            const uint64_t t0 = global_timer_ns();
+            while (ld_acquire_gpu(p.ticket) < static_cast<uint32_t>(G)) {
+                if (global_timer_ns() - t0 > kWaitLimitNs) {
+                    atomicOr(p.err, kErrWaitTimeout);
+                    break;
+                }
+                __nanosleep(32);
+            }
+        }
+    }
+    __syncthreads();
+    const int m = mc->merger;
+    if (m < 0) return;
+
+    // ---------------- global merge (last X CTAs) ----------------
+    // Scores, buffers and ring are free now.  Per query: the first kFastE keys
+    // of every list (the heads area) go to shared memory, the fast merge
+    // settles the query from them, or the full merge reads the lists.
+    if ((*reinterpret_cast<volatile uint32_t *>(p.err) & kErrWaitTimeout) == 0u) {
+        static_assert(kTcMergeE == kFastE, "the heads area feeds the fast merge");
+        unsigned char *ws = smem + L.scores;
+        MergeBufs mb;
+        mb.pref = reinterpret_cast<uint64_t *>(ws);
+        mb.cands = mb.pref + kMergePrefixCap;
+        mb.win = mb.cands + kMergeCandCap;
+        mb.counts = reinterpret_cast<int *>(mb.win + 1024);
+        mb.offsets = mb.counts + kMaxLists;
+        mb.hist = reinterpret_cast<uint32_t *>(mb.offsets + kMaxLists);
+        const uint32_t ms_off = (SmemLayout::merge_fixed_bytes() + 15u) & ~15u;
+        MiscSmem *ms = reinterpret_cast<MiscSmem *>(ws + ms_off);
+        uint64_t *fe = reinterpret_cast<uint64_t *>(ws + ms_off + ((sizeof(MiscSmem) + 15u) & ~15u));
+        const int G8 = (G + 7) & ~7;
+        uint32_t *hv = reinterpret_cast<uint32_t *>(fe + G * kFastE);
+        const bool fast_ok = p.k <= G && 2 * G <= kThreads;
+        for (int q = m; q < p.nq; q += X) {
+            const unsigned long long *hq =
+                reinterpret_cast<const unsigned long long *>(p.heads) + static_cast<size_t>(q) * G * kFastE;
+            for (int i = tid; i < G8 * kFastE; i += Sh::kThreads) {
+                const uint64_t x = i < G * kFastE ? __ldcg(hq + i) : 0ull;
+                if (i < G * kFastE) fe[i] = x;
+                if ((i & (kFastE - 1)) == 0) hv[i / kFastE] = static_cast<uint32_t>(x >> 32);
+            }
+            __syncthreads();
+            int32_t *oi = p.out_idx + static_cast<size_t>(q) * p.k;
+            float *ol = p.out_logits + static_cast<size_t>(q) * p.k;
+            float *sp = p.sparse != nullptr ? p.sparse + static_cast<int64_t>(q) * p.V : nullptr;
+            if (!(fast_ok && merge_fast_query(fe, hv, G, p.k, mb.cands, mb.counts, ms, oi, ol, sp)))
+                merge_lists(GlobalKeys{p.cand + static_cast<size_t>(q) * G * p.k}, G, p.k, mb, ms, oi,
+                            ol, sp);
+            __syncthreads();
+        }
+    }
+    if (tid == 0) {
+        const uint32_t done = atomic_add_acq_rel_gpu(p.merged, 1u);
+        if (done == static_cast<uint32_t>(X - 1)) {
+            *p.ticket = 0;  // re-arm the counters for the next launch
+            *p.next_tile = 0;
+            *p.merged = 0;
+        }
     }
 }
 
