@@ -38,9 +38,10 @@ __device__ uint32_t g_dev_err = 0;
 
 constexpr int kMaxSmem = 232448;  // 227 KB opt-in dynamic shared memory per CTA
 constexpr int kMaxNB = 8;
-// The tensor-core path keeps [32][G][k <= 128] lists and [32][G][4] heads in
+// The tensor-core path keeps [NQ][G][k] lists (NQ * k <= kTcListKeys) and
+// [NQ <= 64][G][4] heads in
 // the same scratch as the streaming path's [kMaxNB][G][VIE_K_MAX] lists.
-static_assert((vie::kTcHRows / 2) * (vie::kTcMaxK + vie::kTcMergeE) <= kMaxNB * VIE_K_MAX,
+static_assert(vie::kTcListKeys + (vie::kTcHRows / 2) * vie::kTcMergeE <= kMaxNB * VIE_K_MAX,
               "tensor-core lists must fit the candidate scratch");
 constexpr int kMaxHBytes = 64 * 1024;  // shared-memory budget for staged queries
 
@@ -61,7 +62,7 @@ struct vie_head {
     void *hB;             // [kTcHRows][d_pad] bf16
     bool tc_ready;
     CUtensorMap mapW;     // W as [V][d_pad], box 128 rows x 64 columns, 128-byte swizzle
-    CUtensorMap mapH[3];  // hB, box 16 / 32 / 64 rows x 64 columns
+    CUtensorMap mapH[4];  // hB, box 16 / 32 / 64 / 128 rows x 64 columns
 };
 
 // ---------------------------------------------------------------------------
@@ -312,7 +313,7 @@ vie_status vie_head_create(const void *W_out, int64_t V, int32_t d, vie_dtype dt
     const uint64_t pitch = static_cast<uint64_t>(hd->d_pad) * 2;
     hd->tc_ready = make_map_bf16(&hd->mapW, hd->W, static_cast<uint64_t>(V), hd->d_pad, pitch,
                                  vie::kTcTile);
-    for (int i = 0; i < 3 && hd->tc_ready; ++i)
+    for (int i = 0; i < 4 && hd->tc_ready; ++i)
         hd->tc_ready = make_map_bf16(&hd->mapH[i], hd->hB, vie::kTcHRows, hd->d_pad, pitch, 16u << i);
     *out = hd;
     return VIE_OK;
@@ -342,15 +343,24 @@ vie_status vie_head_get_props(const vie_head *head, vie_head_props *props) {
 }
 
 // The launch plan of a top-k call (path, query groups, launches).
+// Query slots per tensor-core launch: the smallest tile that holds the batch;
+// 64 (one pass over W for up to 64 queries) only where k fits its lists.
+static int tc_group(int32_t batch, int32_t k) {
+    if (batch <= 8) return 8;
+    if (batch <= 16) return 16;
+    if (batch <= 32 || k > vie::tc_max_k(64)) return 32;
+    return 64;
+}
+
 static bool use_tc(const vie_head *head, int32_t batch, int32_t k) {
-    return head->tc_ready && batch >= knobs().tc_min_batch && k <= vie::kTcMaxK &&
+    return head->tc_ready && batch >= knobs().tc_min_batch && k <= vie::tc_max_k(32) &&
            head->d_pad >= 64;
 }
 
 static vie_topk_plan make_plan(const vie_head *head, int32_t batch, int32_t k) {
     vie_topk_plan pl;
     if (use_tc(head, batch, k)) {
-        const int nqt = batch <= 8 ? 8 : (batch <= 16 ? 16 : 32);
+        const int nqt = tc_group(batch, k);
         pl.path = 1;
         pl.groups = (batch + nqt - 1) / nqt;
         pl.launches = 2 * pl.groups;  // hi/lo prep; projection, per-CTA top-k and merge
@@ -368,7 +378,7 @@ static vie_topk_plan make_plan(const vie_head *head, int32_t batch, int32_t k) {
 static vie_status run_topk_tc(const char *fn, vie_head *head, const float *h, int32_t batch,
                               int32_t k, int32_t *out_idx, float *out_logits, float *sparse,
                               cudaStream_t s) {
-    const int nqt = batch <= 8 ? 8 : (batch <= 16 ? 16 : 32);
+    const int nqt = tc_group(batch, k);
     int stages = 0;
     uint32_t smem = 0;
     int kps = knobs().tc_kps;
@@ -379,7 +389,7 @@ static vie_status run_topk_tc(const char *fn, vie_head *head, const float *h, in
     const int n_tiles = static_cast<int>((head->V + vie::kTcTile - 1) / vie::kTcTile);
     int pct = knobs().static_pct;
     pct = pct < 0 ? 0 : (pct > 100 ? 100 : pct);
-    const CUtensorMap &mapH = head->mapH[nqt == 8 ? 0 : (nqt == 16 ? 1 : 2)];
+    const CUtensorMap &mapH = head->mapH[nqt == 8 ? 0 : (nqt == 16 ? 1 : (nqt == 32 ? 2 : 3))];
     for (int q0 = 0; q0 < batch; q0 += nqt) {
         const int nq = batch - q0 < nqt ? batch - q0 : nqt;
         cudaError_t e = vie::launch_prep_queries(h + static_cast<int64_t>(q0) * head->d, nq, head->d,
@@ -393,8 +403,8 @@ static vie_status run_topk_tc(const char *fn, vie_head *head, const float *h, in
         p.stages = stages;
         p.kb_per_stage = kps;
         p.static_tiles = static_cast<int32_t>(static_cast<int64_t>(n_tiles) * pct / 100 / head->G);
-        p.cand = head->cand;  // [32][G][k <= 128] keys, then the lists' heads
-        p.heads = head->cand + static_cast<size_t>(vie::kTcHRows / 2) * head->G * vie::kTcMaxK;
+        p.cand = head->cand;  // [NQ][G][k] keys (NQ * k <= kTcListKeys), then the heads
+        p.heads = head->cand + static_cast<size_t>(vie::kTcListKeys) * head->G;
         p.ticket = head->words;
         p.next_tile = head->words + 2;
         p.merged = head->words + 3;

@@ -30,6 +30,8 @@ struct TcParams;
 // Ring depth and dynamic shared memory of the tensor-core kernel for query
 // groups of nq_tmpl (8, 16 or 32) and kps K-blocks per stage; false if
 // unsupported.
+// Largest k the tensor-core kernel with nq_tmpl query slots handles.
+int tc_max_k(int nq_tmpl);
 bool tc_shape(int nq_tmpl, int kps, int *stages, uint32_t *smem);
 
 // Launches tc_topk_kernel<nq_tmpl>.

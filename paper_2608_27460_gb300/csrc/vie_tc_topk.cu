@@ -79,6 +79,8 @@ bool tc_shape(int nq_tmpl, int kps, int *stages, uint32_t *smem) {
                  stage_bytes = TcShape<16>::kStageBytes; break;
         case 32: score_bytes = TcShape<32>::kScoreBytes; buf_bytes = TcShape<32>::kBufBytes;
                  stage_bytes = TcShape<32>::kStageBytes; break;
+        case 64: score_bytes = TcShape<64>::kScoreBytes; buf_bytes = TcShape<64>::kBufBytes;
+                 stage_bytes = TcShape<64>::kStageBytes; break;
         default: return false;
     }
     for (int s = kTcMaxStages; s >= 2; --s) {
@@ -92,12 +94,23 @@ bool tc_shape(int nq_tmpl, int kps, int *stages, uint32_t *smem) {
     return false;
 }
 
+int tc_max_k(int nq_tmpl) {
+    switch (nq_tmpl) {
+        case 8: return TcShape<8>::kMaxK;
+        case 16: return TcShape<16>::kMaxK;
+        case 32: return TcShape<32>::kMaxK;
+        case 64: return TcShape<64>::kMaxK;
+        default: return 0;
+    }
+}
+
 cudaError_t launch_tc_topk(int nq_tmpl, const CUtensorMap &mapW, const CUtensorMap &mapH,
                            const TcParams &p, int grid, uint32_t smem, cudaStream_t stream) {
     switch (nq_tmpl) {
         case 8: return launch_tc_one<8>(mapW, mapH, p, grid, smem, stream);
         case 16: return launch_tc_one<16>(mapW, mapH, p, grid, smem, stream);
         case 32: return launch_tc_one<32>(mapW, mapH, p, grid, smem, stream);
+        case 64: return launch_tc_one<64>(mapW, mapH, p, grid, smem, stream);
         default: return cudaErrorInvalidValue;
     }
 }

@@ -18,10 +18,11 @@
 //   warps 2-5    epilogue: tcgen05.ld of the 128 x N accumulator (warp w
 //                owns TMEM lanes 32*(w%4)..), hi + lo per query, logits into
 //                a score ring laid out [query][row];
-//   warps 6..    selectors, one query each (two when NQ = 32): per query a shared buffer
-//                of candidates above a threshold tau; when it passes half
-//                full, a warp-wide bisection keeps the best k (unsorted) and
-//                raises tau; one bitonic sort of the final k per query.
+//   warps 6..    selectors, one query each (two when NQ = 32, four when
+//                NQ = 64): per query a shared buffer of candidates above a
+//                threshold tau; when fewer than 32 slots are left, a
+//                warp-wide bisection keeps the best k (unsorted) and raises
+//                tau; one bitonic sort of the final k per query.
 // Each CTA writes its per-query lists and takes a completion ticket; the
 // last CTAs to finish merge them, one query each.  All waits are bounded.
 #pragma once
@@ -38,9 +39,9 @@ constexpr int kTcTile = 128;       // rows per tile (MMA M)
 constexpr int kTcKBlock = 64;      // bf16 columns per K-block (one 128-byte swizzle row)
 constexpr int kTcScoreSlots = 4;   // score ring depth
 constexpr int kTcMaxStages = 16;
-constexpr int kTcHRows = 64;       // rows of the hi/lo query matrix (N <= 64)
-constexpr int kTcCap = 256;        // candidate buffer per query (>= k + one tile)
-constexpr int kTcMaxK = kTcCap - kTcTile;  // largest k of this path
+constexpr int kTcHRows = 128;      // rows of the hi/lo query matrix (N <= 128)
+constexpr int kTcMaxK = 128;       // largest k of this path
+constexpr int kTcListKeys = 4096;  // keys of the per-CTA lists per CTA: NQ * k <= this
 constexpr int kTcMaxKPS = 4;       // K-blocks per stage, at most
 constexpr int kTcMergeE = 4;       // merge: keys per list in the heads area
 constexpr int kTcMaxMergers = 32;  // CTAs that merge, at most (one per query)
@@ -67,17 +68,22 @@ struct TcParams {
 template <int NQ>
 struct TcShape {
     static constexpr int N = 2 * NQ;
-    static constexpr int kQPW = NQ >= 32 ? 2 : 1;  // queries per selector warp
+    static constexpr int kQPW = NQ >= 64 ? 4 : (NQ >= 32 ? 2 : 1);  // queries per selector warp
     static constexpr int kSelWarps = NQ / kQPW;
     static constexpr int kWarps = 6 + kSelWarps;
     static constexpr int kThreads = 32 * kWarps;
     static constexpr int kStageA = kTcTile * kTcKBlock * 2;  // 16 KB per K-block of W
     static constexpr int kStageB = N * kTcKBlock * 2;        // N x 128 B per K-block of H
     static constexpr int kStageBytes = kStageA + kStageB;    // per K-block; a multiple of 1024
-    static constexpr int kTmemCols = (2 * N <= 32) ? 32 : (2 * N <= 64 ? 64 : 128);
-    static constexpr int kSlots = NQ >= 32 ? 2 : kTcScoreSlots;  // score ring depth
+    static constexpr int kTmemCols = (2 * N <= 32) ? 32 : (2 * N <= 64 ? 64 : (2 * N <= 128 ? 128 : 256));
+    static constexpr int kSlots = NQ >= 64 ? 1 : (NQ >= 32 ? 2 : kTcScoreSlots);  // score ring depth
     static constexpr int kScoreBytes = kSlots * NQ * kTcTile * 4;
-    static constexpr int kBufBytes = NQ * kTcCap * 8 + NQ * 12;  // buffers, counts, thresholds
+    // candidate buffer per query: compacted to k whenever fewer than 32 slots
+    // (one row block) are left, so k <= kCap - 32
+    static constexpr int kCap = NQ >= 64 ? 128 : 256;
+    static constexpr int kMaxK0 = kCap - 32 < kTcMaxK ? kCap - 32 : kTcMaxK;
+    static constexpr int kMaxK = kMaxK0 < kTcListKeys / NQ ? kMaxK0 : kTcListKeys / NQ;  // largest k
+    static constexpr int kBufBytes = NQ * kCap * 8 + NQ * 12;  // buffers, counts, thresholds
 };
 
 struct TcMisc {
@@ -144,15 +150,15 @@ __device__ __forceinline__ void warp_sort_desc(uint64_t (&v)[PER], int lane) {
     }
 }
 
-// Keeps the k largest of the cnt (> k) nonzero keys in buf, unsorted at
+// Keeps the k largest of the cnt (k < cnt <= 32 * PER) nonzero keys in buf, unsorted at
 // buf[0..k), and returns k; *tau becomes a bound T <= the k-th key such that
 // exactly k keys are >= T.  T is found by bisection: first on the high words
 // (the logit order), then, only if several keys tie on the k-th high word,
 // on the low words (the row order) among the tied keys.  Out of line and
 // loop-based: a few hundred instructions, and little code next to the
 // latency-critical producer and MMA loops.
+template <int PER>
 static __device__ __noinline__ int keep_best(uint64_t *buf, int cnt, int k, uint64_t *tau, int lane) {
-    constexpr int PER = kTcCap / 32;
     uint64_t v[PER];
 #pragma unroll
     for (int j = 0; j < PER; ++j) {
@@ -207,12 +213,13 @@ static __device__ __noinline__ int keep_best(uint64_t *buf, int cnt, int k, uint
     return k;
 }
 
-// The final list of one query: the best min(k, cnt) keys of buf, sorted
-// descending, written to dst[0..k) (zeros after them), and its first
-// kTcMergeE keys also to head[0..kTcMergeE).
+// The final list of one query: the best min(k, cnt) keys of buf (cnt <=
+// 32 * CAP_PER), sorted descending, written to dst[0..k) (zeros after them),
+// and its first kTcMergeE keys also to head[0..kTcMergeE).
+template <int CAP_PER>
 static __device__ __noinline__ void write_sorted_list(uint64_t *buf, int cnt, int k, uint64_t *tau,
                                                       uint64_t *dst, uint64_t *head, int lane) {
-    if (cnt > k) cnt = keep_best(buf, cnt, k, tau, lane);
+    if (cnt > k) cnt = keep_best<CAP_PER>(buf, cnt, k, tau, lane);
     constexpr int PER = kTcMaxK / 32;  // cnt <= k <= kTcMaxK
     uint64_t v[PER];
 #pragma unroll
@@ -418,6 +425,40 @@ __global__ void __launch_bounds__(TcShape<NQ>::kThreads, 1)
             tc_fence_after_sync();
             const int tile = mc->buf_tile[b];
             const int ss = ti % Sh::kSlots, su = ti / Sh::kSlots;
+            if constexpr (N > 64) {
+                // wide tiles: wait for the score slot first, then drain the
+                // accumulator 32 columns (16 queries) at a time
+                if (ti >= Sh::kSlots && !mbar_wait(&sempty[ss], (su - 1) & 1, abort_flag)) {
+                    if (lane == 0) {
+                        atomicOr(p.err, kErrWaitTimeout);
+                        mc->abort = 1;
+                    }
+                    break;
+                }
+                if (tile >= 0) {
+                    const uint32_t tb = tmem + (static_cast<uint32_t>(32 * qw) << 16) + b * N;
+                    float *sc = scores + ss * NQ * kTcTile;
+#pragma unroll
+                    for (int c = 0; c < N / 16; c += 2) {
+                        uint32_t r[2][16];
+                        tmem_ld_32x32b_x16(tb + 16 * c, r[0]);
+                        tmem_ld_32x32b_x16(tb + 16 * (c + 1), r[1]);
+                        tmem_wait_ld();
+#pragma unroll
+                        for (int qq = 0; qq < 16; ++qq)
+                            sc[(8 * c + qq) * kTcTile + row] = __uint_as_float(r[qq / 8][(2 * qq) % 16]) +
+                                                               __uint_as_float(r[qq / 8][(2 * qq) % 16 + 1]);
+                    }
+                }
+                tc_fence_before_sync();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&tempty[b]);
+                if (warp == 2 && lane == 0) mc->slot_tile[ss] = tile;
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&sfull[ss]);
+                if (tile < 0) break;
+                continue;
+            }
             float lg[NQ];
             if (tile >= 0) {
                 const uint32_t tb = tmem + (static_cast<uint32_t>(32 * qw) << 16) + b * N;
@@ -468,8 +509,9 @@ __global__ void __launch_bounds__(TcShape<NQ>::kThreads, 1)
         // per query of this warp: candidate count and threshold, in shared
         // memory next to its buffer (only this warp touches them)
         constexpr int QPW = Sh::kQPW;
-        int *cnt_s = reinterpret_cast<int *>(bufs + NQ * kTcCap) + QPW * sel;
-        uint64_t *tau_s = reinterpret_cast<uint64_t *>(bufs + NQ * kTcCap) + NQ / 2 + QPW * sel;
+        constexpr int CAP = Sh::kCap, CAP_PER = CAP / 32;
+        int *cnt_s = reinterpret_cast<int *>(bufs + NQ * CAP) + QPW * sel;
+        uint64_t *tau_s = reinterpret_cast<uint64_t *>(bufs + NQ * CAP) + NQ / 2 + QPW * sel;
         if (lane < QPW) {
             cnt_s[lane] = 0;
             tau_s[lane] = 0;
@@ -494,11 +536,14 @@ __global__ void __launch_bounds__(TcShape<NQ>::kThreads, 1)
             for (int j = 0; j < QPW; ++j) {
                 const int q = QPW * sel + j;
                 if (q >= p.nq) break;
-                uint64_t *buf = bufs + q * kTcCap;
+                uint64_t *buf = bufs + q * CAP;
                 int cnt = cnt_s[j];
-                if (cnt > kTcCap - kTcTile) cnt = keep_best(buf, cnt, p.k, &tau_s[j], lane);
-                const uint64_t tau = tau_s[j];
+                uint64_t tau = tau_s[j];
                 for (int rb = 0; rb < rows; rb += 32) {
+                    if (cnt > CAP - 32) {  // room for one more row block
+                        cnt = keep_best<CAP_PER>(buf, cnt, p.k, &tau_s[j], lane);
+                        tau = tau_s[j];
+                    }
                     const int r = rb + lane;
                     const uint64_t key =
                         (r < rows) ? make_key(sc[q * kTcTile + r], static_cast<uint32_t>(row0 + r)) : 0;
@@ -517,7 +562,7 @@ __global__ void __launch_bounds__(TcShape<NQ>::kThreads, 1)
         for (int j = 0; j < QPW; ++j) {
             const int q = QPW * sel + j;
             if (q >= p.nq) break;
-            write_sorted_list(bufs + q * kTcCap, cnt_s[j], p.k, &tau_s[j],
+            write_sorted_list<CAP_PER>(bufs + q * CAP, cnt_s[j], p.k, &tau_s[j],
                               p.cand + (static_cast<size_t>(q) * G + cta) * p.k,
                               p.heads + (static_cast<size_t>(q) * G + cta) * kTcMergeE, lane);
         }

@@ -18,7 +18,11 @@ def test_plan_selects_paths(vie):
         assert (p.path, p.groups, p.launches) == (0, 1, 1)
         p = head.plan(2, 50)
         assert (p.path, p.groups, p.launches) == (1, 1, 2)
-        p = head.plan(40, 50)  # 32 + 8 queries
+        p = head.plan(40, 50)  # one 64-query group: one pass over W
+        assert (p.path, p.groups, p.launches) == (1, 1, 2)
+        p = head.plan(40, 65)  # k above the 64-query tile's lists: 32 + 8
+        assert (p.path, p.groups, p.launches) == (1, 2, 4)
+        p = head.plan(100, 50)  # 64 + 36
         assert (p.path, p.groups, p.launches) == (1, 2, 4)
         p = head.plan(4, 129)  # above the tensor-core path's k
         assert p.path == 0
@@ -27,7 +31,10 @@ def test_plan_selects_paths(vie):
 @pytest.mark.parametrize("V,d,batch,k", [
     (20011, 512, 3, 128),    # largest k of the tensor-core path
     (20011, 512, 3, 129),    # smallest k above it (streaming path)
-    (30011, 256, 40, 50),    # two query groups, two queries per selector warp
+    (30011, 256, 40, 50),    # 64-query tile, four queries per selector warp
+    (30011, 256, 64, 64),    # full 64-query tile at its largest k
+    (30011, 256, 40, 65),    # two 32-query groups, two queries per selector warp
+    (20011, 1152, 100, 50),  # 64 + 36 queries
     (30011, 256, 32, 1),     # greedy, full group of 32
     (50021, 1024, 17, 77),
 ])
@@ -45,7 +52,7 @@ def _crowded(V, d, batch, rows, seed):
     return synth.f32_to_bf16_bits(f), h
 
 
-@pytest.mark.parametrize("batch,k", [(1, 50), (4, 50), (4, 128), (20, 50)])
+@pytest.mark.parametrize("batch,k", [(1, 50), (4, 50), (4, 128), (20, 50), (40, 50)])
 @pytest.mark.parametrize("where", ["head", "tail"])
 def test_crowded_winners_take_the_full_merge(vie, batch, k, where):
     V, d = 40009, 256
@@ -56,13 +63,13 @@ def test_crowded_winners_take_the_full_merge(vie, batch, k, where):
 
 
 def test_all_rows_equal_full_groups(vie):
-    """Every logit equal, 20 queries (32-query group): every query leaves the
-    warp merge for the full merge, which ranks by index."""
+    """Every logit equal, in 32- and 64-query tiles: every query leaves the
+    fast merge for the full merge, which ranks by index."""
     V, d = 30011, 64
     row = synth.f32_to_bf16_bits(np.full(d, 0.25, np.float32))
     W = np.tile(row, (V, 1))
-    h = np.ones((20, d), np.float32)
-    for k in (1, 128):
+    for b, k in ((20, 1), (20, 128), (48, 64)):
+        h = np.ones((b, d), np.float32)
         idx, val = run_head(vie, W, h, k)
-        np.testing.assert_array_equal(idx, np.tile(np.arange(k, dtype=np.int32), (20, 1)))
+        np.testing.assert_array_equal(idx, np.tile(np.arange(k, dtype=np.int32), (b, 1)))
         assert np.all(val == np.float32(0.25 * d))
