@@ -142,6 +142,31 @@ vie_status vie_head_topk_sparse(vie_head *head, const float *h, int32_t batch, i
                                 vie_stream stream);
 
 /*
+ * vie_head_topk_host - one whole decode step for a caller whose queries and
+ * results live in host memory: copies h in, runs vie_head_topk_sparse (or
+ * vie_head_topk when out_sparse is NULL), copies the top-k out and waits for
+ * it.  The paper has no counterpart: it is the end-to-end form of the call.
+ *
+ *   h_host       host, fp32, row-major [batch, d].  Page-locked memory
+ *                (cudaMallocHost / cudaHostRegister) keeps the copies
+ *                asynchronous; pageable memory works, staged by the driver.
+ *   idx_host     host, int32 [batch, k];  logits_host  host, fp32 [batch, k].
+ *   out_sparse   device, fp32 [batch, V] (4-byte aligned), or NULL.
+ *   batch, k, stream: as for vie_head_topk.
+ *
+ * The queries and the top-k pass through device buffers owned by the handle:
+ * allocated by the first call that needs them (larger ones by a later call
+ * that needs more, VIE_ERR_OOM if that fails), freed by vie_head_destroy.  The
+ * call synchronises `stream` before it returns, so the host outputs are
+ * ready; a device-side problem is reported by the next
+ * vie_head_device_status, as for vie_head_topk.  At most one call per handle
+ * at a time, as for vie_head_topk.
+ */
+vie_status vie_head_topk_host(vie_head *head, const float *h_host, int32_t batch, int32_t k,
+                              int32_t *idx_host, float *logits_host, float *out_sparse,
+                              vie_stream stream);
+
+/*
  * vie_scatter_sparse_logits - the sparse full-vocabulary logit tensor of
  * Section 3: out[b, v] = -inf (bit pattern 0xFF800000) for every v, then
  * out[b, idx[b, j]] = logits[b, j] for j < k (values copied bit for bit).

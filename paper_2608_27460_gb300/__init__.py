@@ -36,8 +36,8 @@ STATUS_NAMES = {0: "VIE_OK", 1: "VIE_ERR_INVALID_ARG", 2: "VIE_ERR_UNSUPPORTED",
 
 # Every entry point of include/vie_head.h.
 EXPORTS = ("vie_head_create", "vie_head_destroy", "vie_head_get_props", "vie_head_plan", "vie_head_topk",
-           "vie_head_topk_sparse", "vie_head_topk_noalloc", "vie_scatter_sparse_logits", "vie_device_status", "vie_head_device_status",
-           "vie_last_error")
+           "vie_head_topk_sparse", "vie_head_topk_host", "vie_head_topk_noalloc", "vie_scatter_sparse_logits",
+           "vie_device_status", "vie_head_device_status", "vie_last_error")
 
 
 class VieError(RuntimeError):
@@ -85,6 +85,7 @@ def load(path: str | None = None, build_if_missing: bool = True):
             "vie_head_plan": ([P, I32, I32, ctypes.POINTER(vie_topk_plan)], ctypes.c_int),
             "vie_head_topk": ([P, P, I32, I32, P, P, P], ctypes.c_int),
             "vie_head_topk_sparse": ([P, P, I32, I32, P, P, P, P], ctypes.c_int),
+            "vie_head_topk_host": ([P, P, I32, I32, P, P, P, P], ctypes.c_int),
             "vie_head_topk_noalloc": ([P, I64, I32, P, I32, I32, P, P, P], ctypes.c_int),
             "vie_scatter_sparse_logits": ([P, P, I32, I32, I64, P, P], ctypes.c_int),
             "vie_device_status": ([P], ctypes.c_int),
@@ -140,6 +141,11 @@ def vie_head_topk(head: int, h: int, batch: int, k: int, out_idx: int, out_logit
 def vie_head_topk_sparse(head: int, h: int, batch: int, k: int, out_idx: int, out_logits: int,
                          out_sparse: int, stream: int = 0) -> int:
     return load().vie_head_topk_sparse(head, h, batch, k, out_idx, out_logits, out_sparse, stream)
+
+
+def vie_head_topk_host(head: int, h_host: int, batch: int, k: int, idx_host: int, logits_host: int,
+                       out_sparse: int = 0, stream: int = 0) -> int:
+    return load().vie_head_topk_host(head, h_host, batch, k, idx_host, logits_host, out_sparse, stream)
 
 
 def vie_head_topk_noalloc(W_out: int, V: int, d: int, h: int, batch: int, k: int, out_idx: int,
@@ -245,6 +251,26 @@ class Head:
         check(vie_head_topk_sparse(self.handle, h.data_ptr(), b, k, out_idx.data_ptr(),
                                    out_logits.data_ptr(), out_sparse.data_ptr(), _stream_ptr(stream)))
         return out_idx, out_logits, out_sparse
+
+    def topk_host(self, h, k: int, out_idx=None, out_logits=None, out_sparse=None, stream=None):
+        """One decode step from host memory: h (CPU float32 [batch, d], best
+        pinned) in, top-k (CPU int32 / float32 [batch, k]) out, ready on
+        return; out_sparse, if given, is a CUDA [batch, V] tensor."""
+        import torch
+        if h.dim() == 1:
+            h = h[None]
+        if h.dtype != torch.float32 or h.is_cuda or h.shape[1] != self.d:
+            raise ValueError(f"h must be a CPU float32 tensor [batch, {self.d}]")
+        h = h.contiguous()
+        b = int(h.shape[0])
+        if out_idx is None:
+            out_idx = torch.empty((b, k), dtype=torch.int32)
+        if out_logits is None:
+            out_logits = torch.empty((b, k), dtype=torch.float32)
+        sp = 0 if out_sparse is None else out_sparse.data_ptr()
+        check(vie_head_topk_host(self.handle, h.data_ptr(), b, k, out_idx.data_ptr(),
+                                 out_logits.data_ptr(), sp, _stream_ptr(stream)))
+        return out_idx, out_logits
 
     def sparse_logits(self, idx, logits, out=None, stream=None):
         """Sparse [batch, V] fp32 tensor: -inf except logits at idx."""

@@ -63,6 +63,11 @@ struct vie_head {
     bool tc_ready;
     CUtensorMap mapW;     // W as [V][d_pad], box 128 rows x 64 columns, 128-byte swizzle
     CUtensorMap mapH[4];  // hB, box 16 / 32 / 64 / 128 rows x 64 columns
+    // vie_head_topk_host: device staging of queries and top-k (grown on demand)
+    float *stage_h;
+    int32_t *stage_idx;
+    float *stage_logits;
+    size_t stage_h_elems, stage_out_elems;
 };
 
 // ---------------------------------------------------------------------------
@@ -325,6 +330,9 @@ vie_status vie_head_destroy(vie_head *head) {
     cudaFree(head->cand);
     cudaFree(head->words);
     cudaFree(head->hB);
+    cudaFree(head->stage_h);
+    cudaFree(head->stage_idx);
+    cudaFree(head->stage_logits);
     delete head;
     return VIE_OK;
 }
@@ -498,6 +506,60 @@ vie_status vie_head_topk_sparse(vie_head *head, const float *h, int32_t batch, i
         return fail(VIE_ERR_INVALID_ARG, "vie_head_topk_sparse: out_sparse is NULL");
     return run_topk("vie_head_topk_sparse", head, h, batch, k, out_idx, out_logits, out_sparse,
                     stream);
+}
+
+vie_status vie_head_topk_host(vie_head *head, const float *h_host, int32_t batch, int32_t k,
+                              int32_t *idx_host, float *logits_host, float *out_sparse,
+                              vie_stream stream) {
+    const char *fn = "vie_head_topk_host";
+    if (head == nullptr) return fail(VIE_ERR_INVALID_ARG, "%s: head is NULL", fn);
+    if (h_host == nullptr || idx_host == nullptr || logits_host == nullptr)
+        return fail(VIE_ERR_INVALID_ARG, "%s: NULL buffer", fn);
+    if (batch < 1 || batch > VIE_BATCH_MAX)
+        return fail(VIE_ERR_INVALID_ARG, "%s: batch=%d outside [1, %d]", fn, batch, VIE_BATCH_MAX);
+    if (k < 1 || k > VIE_K_MAX || static_cast<int64_t>(k) > head->V)
+        return fail(VIE_ERR_INVALID_ARG, "%s: k=%d outside [1, min(V=%lld, %d)]", fn, k,
+                    static_cast<long long>(head->V), VIE_K_MAX);
+    vie_status st = check_device(head);
+    if (st != VIE_OK) return st;
+    const size_t nh = static_cast<size_t>(batch) * head->d, no = static_cast<size_t>(batch) * k;
+    if (head->stage_h_elems < nh) {
+        cudaFree(head->stage_h);
+        head->stage_h = nullptr;
+        head->stage_h_elems = 0;
+        if (cudaMalloc(&head->stage_h, nh * sizeof(float)) != cudaSuccess) {
+            cudaGetLastError();
+            return fail(VIE_ERR_OOM, "%s: cannot allocate %zu bytes of query staging", fn,
+                        nh * sizeof(float));
+        }
+        head->stage_h_elems = nh;
+    }
+    if (head->stage_out_elems < no) {
+        cudaFree(head->stage_idx);
+        cudaFree(head->stage_logits);
+        head->stage_idx = nullptr;
+        head->stage_logits = nullptr;
+        head->stage_out_elems = 0;
+        if (cudaMalloc(&head->stage_idx, no * sizeof(int32_t)) != cudaSuccess ||
+            cudaMalloc(&head->stage_logits, no * sizeof(float)) != cudaSuccess) {
+            cudaGetLastError();
+            return fail(VIE_ERR_OOM, "%s: cannot allocate %zu bytes of output staging", fn,
+                        no * 8);
+        }
+        head->stage_out_elems = no;
+    }
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    cudaError_t e = cudaMemcpyAsync(head->stage_h, h_host, nh * sizeof(float), cudaMemcpyHostToDevice, s);
+    if (e != cudaSuccess) return fail_cuda(e, "vie_head_topk_host: copy of h");
+    st = run_topk(fn, head, head->stage_h, batch, k, head->stage_idx, head->stage_logits, out_sparse,
+                  stream);
+    if (st != VIE_OK) return st;
+    e = cudaMemcpyAsync(idx_host, head->stage_idx, no * sizeof(int32_t), cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess)
+        e = cudaMemcpyAsync(logits_host, head->stage_logits, no * sizeof(float), cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess) return fail_cuda(e, "vie_head_topk_host: copy of the top-k");
+    return VIE_OK;
 }
 
 vie_status vie_scatter_sparse_logits(const int32_t *idx, const float *logits, int32_t batch,

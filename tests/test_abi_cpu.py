@@ -61,6 +61,8 @@ def test_calls_on_null_handle_are_rejected(lib):
     assert vie.vie_head_topk(0, 16, 1, 1, 16, 16) == vie.VIE_ERR_INVALID_ARG
     assert vie.vie_head_get_props(0)[0] == vie.VIE_ERR_INVALID_ARG
     assert vie.vie_head_device_status(0) == vie.VIE_ERR_INVALID_ARG
+    assert vie.vie_head_topk_host(0, 16, 1, 1, 16, 16) == vie.VIE_ERR_INVALID_ARG
+    assert vie.vie_head_plan(0, 1, 1)[0] == vie.VIE_ERR_INVALID_ARG
 
 
 def test_scatter_rejects_bad_arguments_on_host(lib):
