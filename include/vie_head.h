@@ -21,7 +21,8 @@
  *   - Device-side problems (an out-of-range scatter index, a pipeline wait
  *     that ran past its time limit) never trap: the kernel records a flag and
  *     returns, and the next vie_device_status / vie_head_device_status call
- *     reports VIE_ERR_DEVICE.
+ *     reports VIE_ERR_DEVICE.  The outputs of the call that recorded a wait
+ *     time-out are unspecified (every write still stays inside them).
  *   - Logits are fp32.  Ranking is by logit descending; equal logits are
  *     ranked by ascending vocabulary index, and -0.0 ranks as +0.0 (and is
  *     returned as +0.0).  Inputs must be finite; results for NaN or infinite

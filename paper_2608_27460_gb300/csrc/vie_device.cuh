@@ -91,6 +91,22 @@ __device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, volati
     }
 }
 
+// Asynchronous 4-byte copy global -> shared (cp.async), or 4 zero bytes when
+// !real (src is then not read).  Completes at cp_async_wait_all.
+__device__ __forceinline__ void cp_async_4_zfill(void *dst, const void *src, bool real) {
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;" ::"r"(smem_addr(dst)), "l"(src),
+                 "r"(real ? 4 : 0)
+                 : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_all;" ::: "memory"); }
+
+// Barrier `id` (1..15; 0 is __syncthreads) over `count` threads of the CTA,
+// a multiple of 32; every warp that takes part calls it with all lanes.
+__device__ __forceinline__ void named_barrier_sync(int id, int count) {
+    asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(count) : "memory");
+}
+
 // Load with acquire semantics at GPU scope.
 __device__ __forceinline__ uint32_t ld_acquire_gpu(const uint32_t *p) {
     uint32_t v;

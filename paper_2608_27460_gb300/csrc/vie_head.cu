@@ -292,6 +292,7 @@ vie_status vie_head_create(const void *W_out, int64_t V, int32_t d, vie_dtype dt
     hd->scratch_bytes = static_cast<int64_t>(cbytes + 4 * sizeof(uint32_t));
     e = cudaMalloc(&hd->W, wbytes);
     if (e == cudaSuccess) e = cudaMalloc(&hd->cand, cbytes);
+    if (e == cudaSuccess) e = cudaMemset(hd->cand, 0, cbytes);  // empty lists until written
     if (e == cudaSuccess) e = cudaMalloc(&hd->words, 4 * sizeof(uint32_t));
     if (e == cudaSuccess)
         e = cudaMalloc(&hd->hB, static_cast<size_t>(vie::kTcHRows) * hd->d_pad * 2);

@@ -386,6 +386,18 @@ __device__ void merge_lists(Keys lists, int G, int k, const MergeBufs &mb, MiscS
     }
 }
 
+// The zeroed counters merge_fast_query starts from (every thread calls it;
+// callers overlap it with the loads that stage the lists' heads).
+__device__ __forceinline__ void merge_fast_reset(int *rank_part, MiscSmem *ms) {
+    if (threadIdx.x == 0) {
+        ms->tau_v = 0;
+        ms->n_cand = 0;
+        ms->overflow = 0;
+    }
+    for (int i = threadIdx.x; i < kFastE * kThreads / 2; i += static_cast<int>(blockDim.x))
+        rank_part[i] = 0;  // M <= G * kFastE <= kFastE * kThreads / 2
+}
+
 // Latency-lean merge of one query for small k, spread over every warp of
 // the CTA.  fe = the first kFastE keys of each of the G sorted lists, hv =
 // their heads' value bits (padded with 0 to a multiple of 8).  tau = the
@@ -393,19 +405,13 @@ __device__ void merge_lists(Keys lists, int G, int k, const MergeBufs &mb, MiscS
 // >= (tau << 32), so every top-k key is too, and each list contributes its
 // prefix of keys above that bound.  Returns false (writing nothing) if some
 // list might hold more than kFastE such keys or fewer than k heads are
-// real; the caller then merges in full.  Requires 2 * G <= kThreads.
+// real; the caller then merges in full.  Requires 2 * G <= kThreads, and
+// the state merge_fast_reset sets, made visible by a bar.sync.
 __device__ inline bool merge_fast_query(const uint64_t *fe, const uint32_t *hv, int G, int k,
                                         uint64_t *cands, int *rank_part, MiscSmem *ms, int32_t *oi,
                                         float *ol, float *sp) {
     const int tid = threadIdx.x, lane = tid & 31;
     const int G8 = (G + 7) & ~7;
-    if (tid == 0) {
-        ms->tau_v = 0;
-        ms->n_cand = 0;
-        ms->overflow = 0;
-    }
-    for (int i = tid; i < kFastE * kThreads / 2; i += static_cast<int>(blockDim.x)) rank_part[i] = 0;  // M <= G * kFastE
-    __syncthreads();
     // tau: thread pair (2c, 2c+1) counts the heads >= head c, half each
     {
         const int c = tid >> 1, half = tid & 1;
@@ -507,12 +513,15 @@ __device__ inline void merge_queries(const uint64_t *cand, int nq, int G, int k,
         uint32_t *hv = reinterpret_cast<uint32_t *>(fe + nq * G * kFastE);  // [nq][G8]
         const int En = k < kFastE ? k : kFastE;
         for (int q = 0; q < nq; ++q) {
+            uint64_t key[kFastE];
             if (tid < G8) {
-                uint64_t key[kFastE];
                 const unsigned long long *lc = reinterpret_cast<const unsigned long long *>(cand) +
                                                (static_cast<size_t>(q) * G + tid) * k;
 #pragma unroll
                 for (int e = 0; e < kFastE; ++e) key[e] = (tid < G && e < En) ? __ldcg(lc + e) : 0ull;
+            }
+            if (q == 0) merge_fast_reset(mb.counts, ms);  // while the loads are in flight
+            if (tid < G8) {
                 if (tid < G) {
 #pragma unroll
                     for (int e = 0; e < kFastE; ++e) fe[(q * G + tid) * kFastE + e] = key[e];
@@ -525,6 +534,11 @@ __device__ inline void merge_queries(const uint64_t *cand, int nq, int G, int k,
             int32_t *oi = out_idx + static_cast<size_t>(nb) * k;
             float *ol = out_logits + static_cast<size_t>(nb) * k;
             float *sp = sparse != nullptr ? sparse + static_cast<int64_t>(nb) * V : nullptr;
+            if (nb > 0) {  // every thread is done with the previous query's counters
+                __syncthreads();
+                merge_fast_reset(mb.counts, ms);
+                __syncthreads();
+            }
             if (merge_fast_query(fe + nb * G * kFastE, hv + nb * G8, G, k, mb.cands, mb.counts, ms,
                                  oi, ol, sp))
                 fast_done |= 1u << nb;
@@ -597,12 +611,19 @@ __global__ void __launch_bounds__(kThreads, 1) stream_topk_kernel(const StreamTo
         fence_mbar_init();
     }
     // h -> shared memory as [nb][half][chunk][4] so a lane's two float4 loads
-    // of one chunk fall in distinct bank groups; zero pad, zero unused queries.
-    for (int i = tid; i < NB * p.d_pad; i += kThreads) {
-        const int nb = i / p.d_pad, j = i - nb * p.d_pad;
-        const float v = (nb < p.nq && j < p.d) ? p.h[static_cast<int64_t>(nb) * p.d + j] : 0.0f;
-        const int c = j >> 3, e = j & 7;
-        h_s[(nb * 2 + (e >> 2)) * (C * 4) + c * 4 + (e & 3)] = v;
+    // of one chunk fall in distinct bank groups; zero pad, zero unused
+    // queries.  Asynchronous copies by warps 1.. issued before the producer
+    // starts, so h is ahead of the weight stream in the memory queues; those
+    // warps wait for them after the barrier (bar.sync 1 below).
+    if (warp > 0) {
+        for (int i = tid - 32; i < NB * p.d_pad; i += kThreads - 32) {
+            const int nb = i / p.d_pad, j = i - nb * p.d_pad;
+            const bool real = nb < p.nq && j < p.d;
+            const float *src = real ? p.h + static_cast<int64_t>(nb) * p.d + j : p.h;
+            const int c = j >> 3, e = j & 7;
+            cp_async_4_zfill(h_s + (nb * 2 + (e >> 2)) * (C * 4) + c * 4 + (e & 3), src, real);
+        }
+        cp_async_commit();
     }
     __syncthreads();
 
@@ -664,6 +685,8 @@ __global__ void __launch_bounds__(kThreads, 1) stream_topk_kernel(const StreamTo
                 for (int64_t i = tid - 32; i < fn; i += kThreads - 32) row[i] = ninf;
             }
         }
+        cp_async_wait_all();
+        named_barrier_sync(1, kThreads - 32);  // h in shared memory for warps 1..
         if (warp == 1) {
             // ---------------- selector ----------------
             WarpList<MM> list[NB];
@@ -838,9 +861,10 @@ __global__ void __launch_bounds__(kThreads, 1) stream_topk_kernel(const StreamTo
     if (!ms->is_last) return;
 
     // ---------------- global merge (last CTA) ----------------
-    const bool aborted = (*reinterpret_cast<volatile uint32_t *>(p.err) & kErrWaitTimeout) != 0;
-    if (!aborted)
-        merge_queries(p.cand, p.nq, G, p.k, p.V, smem + L.merge, L.total - L.merge, ms, p.out_idx,
+    // Every CTA wrote a full list (valid keys or zeros) even if it gave up on
+    // a wait, so the merge stays in bounds; such a call is reported through
+    // the device flag and its outputs are unspecified.
+    merge_queries(p.cand, p.nq, G, p.k, p.V, smem + L.merge, L.total - L.merge, ms, p.out_idx,
                       p.out_logits, p.sparse);
     if (tid == 0) {
         *p.ticket = 0;  // re-arm both counters for the next launch

@@ -604,7 +604,9 @@ __global__ void __launch_bounds__(TcShape<NQ>::kThreads, 1)
     // Scores, buffers and ring are free now.  Per query: the first kFastE keys
     // of every list (the heads area) go to shared memory, the fast merge
     // settles the query from them, or the full merge reads the lists.
-    if ((*reinterpret_cast<volatile uint32_t *>(p.err) & kErrWaitTimeout) == 0u) {
+    // (every CTA wrote full lists and heads, valid keys or zeros, even if it
+    // gave up on a wait: the merge stays in bounds, the flag reports the call)
+    {
         static_assert(kTcMergeE == kFastE, "the heads area feeds the fast merge");
         unsigned char *ws = smem + L.scores;
         MergeBufs mb;
@@ -625,9 +627,11 @@ __global__ void __launch_bounds__(TcShape<NQ>::kThreads, 1)
                 reinterpret_cast<const unsigned long long *>(p.heads) + static_cast<size_t>(q) * G * kFastE;
             for (int i = tid; i < G8 * kFastE; i += Sh::kThreads) {
                 const uint64_t x = i < G * kFastE ? __ldcg(hq + i) : 0ull;
+                if (i == tid) merge_fast_reset(mb.counts, ms);  // while the first loads are in flight
                 if (i < G * kFastE) fe[i] = x;
                 if ((i & (kFastE - 1)) == 0) hv[i / kFastE] = static_cast<uint32_t>(x >> 32);
             }
+            if (tid >= G8 * kFastE) merge_fast_reset(mb.counts, ms);
             __syncthreads();
             int32_t *oi = p.out_idx + static_cast<size_t>(q) * p.k;
             float *ol = p.out_logits + static_cast<size_t>(q) * p.k;
