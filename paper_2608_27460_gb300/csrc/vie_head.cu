@@ -176,8 +176,9 @@ struct LaunchShape {
 // and ring depth (deepest that fits) for one launch.
 bool pick_shape(int nb, int d_pad, LaunchShape *out) {
     const int row_bytes = d_pad * 2;
+    const int r_max = nb == 1 ? 8 : 4;  // 8 rows per warp only for single-query launches
     int r = 1;
-    while (r < 4 && 8 * r * row_bytes < knobs().stage_min_bytes) r <<= 1;
+    while (r < r_max && 8 * r * row_bytes < knobs().stage_min_bytes) r <<= 1;
     for (int rs = 8 * r; rs >= 1; --rs) {
         for (int s = vie::kMaxStages; s >= 2; --s) {
             const vie::SmemLayout L(nb, d_pad, rs, s, row_bytes);

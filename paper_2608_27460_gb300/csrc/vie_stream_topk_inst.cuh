@@ -46,6 +46,9 @@ cudaError_t launch_width(int mm, int r, const StreamTopkParams &p, int grid, uin
         case 1: return launch_rows<NB, 1>(mm, p, grid, smem, stream);
         case 2: return launch_rows<NB, 2>(mm, p, grid, smem, stream);
         case 4: return launch_rows<NB, 4>(mm, p, grid, smem, stream);
+        case 8:  // narrow rows, one query: 64-row stages
+            if constexpr (NB == 1) return launch_rows<NB, 8>(mm, p, grid, smem, stream);
+            return cudaErrorInvalidValue;
         default: return cudaErrorInvalidValue;
     }
 }
