@@ -81,6 +81,25 @@ def kernel_source_digest(kernel: str = "stream_topk") -> str:
     return h.hexdigest()[:16]
 
 
+def rank_max(x: float, world: int, device="cpu") -> float:
+    """The largest value of x over all ranks (x itself when there is one).
+    A collective: every rank calls it."""
+    if world <= 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_us_per_step(step_us_max: float, world: int) -> float:
+    """Microseconds per decode step of the whole job: N replicas each run
+    the same steps, so in the slowest rank's time per step the job
+    completes N steps."""
+    return step_us_max / world
+
+
 def measured_peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(p):
@@ -318,10 +337,11 @@ def main(argv=None):
     clocks = sampler.stop() if sampler else []
     vie.check(head.device_status())
 
-    if world > 1:
-        t = torch.tensor([total_ms], device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        total_ms = float(t.item())
+    if flush is not None:
+        step_us = statistics.mean(kern_ms) * 1e3  # the flush between steps is not head time
+    else:
+        step_us = total_ms * 1e3 / K
+    step_us = rank_max(step_us, world, dev)  # the slowest rank
 
     # end-to-end through the public API with host buffers: each step is one
     # vie_head_topk_host call, which copies that step's h in from pinned host
@@ -345,7 +365,7 @@ def main(argv=None):
     t_e0 = time.perf_counter()
     for i in range(E):
         e2e_step(i)
-    e2e_us = (time.perf_counter() - t_e0) * 1e6 / E
+    e2e_us = rank_max((time.perf_counter() - t_e0) * 1e6 / E, world, dev)
 
     if rank != 0:
         head.close()
@@ -362,11 +382,7 @@ def main(argv=None):
     plan = head.plan(b, k)
     kernel = "stream_topk" if plan.path == 0 else "tc_topk"
     traffic, prof_path = profiled_traffic(kernel, args.workload, b, k)
-    if flush is not None:
-        step_us = statistics.mean(kern_ms) * 1e3  # the flush between steps is not head time
-    else:
-        step_us = total_ms * 1e3 / K
-    value = step_us / world
+    value = whole_job_us_per_step(step_us, world)
     launches_per_step = plan.launches
 
     line = {
@@ -386,7 +402,7 @@ def main(argv=None):
                      "w_only_gbs": round(w_bytes / (kern_us * 1e-6) / 1e9, 1),
                      "kernel_us_p10_p50_p90": [round(float(np.percentile(kern_ms, q)) * 1e3, 2)
                                                for q in (10, 50, 90)]},
-        "e2e": {"value": round(e2e_us, 3), "unit": UNIT, "h2d_bytes_per_step": b * shape.d * 4,
+        "e2e": {"value": round(whole_job_us_per_step(e2e_us, world), 3), "unit": UNIT, "h2d_bytes_per_step": b * shape.d * 4,
                 "d2h_bytes_per_step": b * k * 8, "api": "vie_head_topk_host (pinned host h in, "
                 "top-k out, synchronised)", "clock": "host wall clock over the steps"},
         "gpu_launches": K * launches_per_step,
