@@ -201,8 +201,8 @@ vie_status vie_scatter_sparse_logits(const int32_t *idx, const float *logits, in
  *   h, batch, k, out_idx, out_logits, stream: as for vie_head_topk.
  *
  * Scratch: one 1 MiB array per device (every GPU that loads the library keeps
- * it until the process exits).  A launch needs 8 * slots * ctas * k bytes of
- * it, where ctas = min(SM count, ceil(V / 64)) and slots = the query group
+ * it until the process exits).  A launch needs 8 * slots * ctas * (k + 4)
+ * bytes of it, where ctas = min(SM count, ceil(V / 64)) and slots = the query group
  * width (the batch rounded up to a power of two, at most 8); larger requests
  * return VIE_ERR_UNSUPPORTED with the sizes in the message.  The call clears
  * the counters at the start of the array with cudaMemsetAsync on `stream`

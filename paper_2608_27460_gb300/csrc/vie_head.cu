@@ -54,7 +54,7 @@ struct vie_head {
     int num_sms;
     int G;
     uint16_t *W;        // [V, d_pad] bf16 bits
-    uint64_t *cand;     // [kMaxNB][G][VIE_K_MAX] ranking keys
+    uint64_t *cand;     // [kMaxNB][G][VIE_K_MAX] ranking keys, then [kMaxNB][G][kFastE] heads
     uint32_t *words;    // [0] completion ticket, [1] device flag word, [2] chunk pool counter,
                         // [3] merging CTAs done (tensor-core path)
     int64_t scratch_bytes;
@@ -156,15 +156,24 @@ int env_int(const char *name, int dflt) {
 // Launch-shape knobs (they change speed, never results):
 //   VIE_STAGE_MIN_KB     smallest weight stage worth one bulk copy (48)
 //   VIE_STATIC_PCT       share of the chunks assigned statically, in % (85)
+//   VIE_POOL_DIV         pool pieces are chunks / this (1)
 //   VIE_TC_MIN_BATCH     smallest batch sent to the tensor-core path (2)
 //   VIE_TC_KPS           K-blocks of 64 columns per tensor-core ring stage (4)
 struct Knobs {
-    int stage_min_bytes, static_pct, tc_min_batch, tc_kps;
+    int stage_min_bytes, static_pct, tc_min_batch, tc_kps, pool_div;
 };
 const Knobs &knobs() {
     static const Knobs k = {env_int("VIE_STAGE_MIN_KB", 48) * 1024, env_int("VIE_STATIC_PCT", 85),
-                            env_int("VIE_TC_MIN_BATCH", 2), env_int("VIE_TC_KPS", 4)};
+                            env_int("VIE_TC_MIN_BATCH", 2), env_int("VIE_TC_KPS", 4),
+                            env_int("VIE_POOL_DIV", 1)};
     return k;
+}
+
+// Rows of a pool piece for stages of rs rows.
+int pool_rows_for(int rs) {
+    int div = knobs().pool_div;
+    div = div < 1 ? 1 : (div > rs ? rs : div);
+    return (rs + div - 1) / div;
 }
 
 struct LaunchShape {
@@ -289,7 +298,8 @@ vie_status vie_head_create(const void *W_out, int64_t V, int32_t d, vie_dtype dt
     hd->G = static_cast<int>(g < 1 ? 1 : g);
 
     const size_t wbytes = static_cast<size_t>(V) * hd->d_pad * 2;
-    const size_t cbytes = static_cast<size_t>(kMaxNB) * hd->G * VIE_K_MAX * sizeof(uint64_t);
+    const size_t cbytes =
+        static_cast<size_t>(kMaxNB) * hd->G * (VIE_K_MAX + vie::kFastE) * sizeof(uint64_t);
     hd->scratch_bytes = static_cast<int64_t>(cbytes + 4 * sizeof(uint32_t));
     e = cudaMalloc(&hd->W, wbytes);
     if (e == cudaSuccess) e = cudaMalloc(&hd->cand, cbytes);
@@ -470,7 +480,9 @@ static vie_status run_topk(const char *fn, vie_head *head, const float *h, int32
         int pct = knobs().static_pct;
         pct = pct < 0 ? 0 : (pct > 100 ? 100 : pct);
         p.static_chunks = static_cast<int32_t>(n_chunks * pct / 100 / head->G);
+        p.pool_rows = pool_rows_for(shp.rs);
         p.cand = head->cand;
+        p.heads = head->cand + static_cast<size_t>(kMaxNB) * head->G * VIE_K_MAX;
         p.ticket = head->words;
         p.err = head->words + 1;
         p.next_chunk = head->words + 2;
@@ -701,12 +713,14 @@ extern "C" vie_status vie_head_topk_noalloc(const void *W_out, int64_t V, int32_
     const int cap = nb_cap_for(d, mm);
     int nb_max = 1;
     while (nb_max < cap && nb_max < batch) nb_max <<= 1;
-    const size_t lists_bytes = static_cast<size_t>(nb_max) * G * k * sizeof(uint64_t);
+    const size_t lists_bytes =
+        static_cast<size_t>(nb_max) * G * (k + vie::kFastE) * sizeof(uint64_t);  // lists, heads
     if (lists_bytes > kNoAllocScratchBytes - kNoAllocCounterBytes)
         return fail(VIE_ERR_UNSUPPORTED,
-                    "%s: needs %zu bytes of scratch (%d query slots x %d CTAs x k=%d x 8), more than "
-                    "the fixed %zu; use vie_head_topk or a smaller batch or k",
-                    fn, lists_bytes, nb_max, G, k, kNoAllocScratchBytes - kNoAllocCounterBytes);
+                    "%s: needs %zu bytes of scratch (%d query slots x %d CTAs x (k=%d + %d) x 8), "
+                    "more than the fixed %zu; use vie_head_topk or a smaller batch or k",
+                    fn, lists_bytes, nb_max, G, k, vie::kFastE,
+                    kNoAllocScratchBytes - kNoAllocCounterBytes);
 
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     uint32_t *counters = reinterpret_cast<uint32_t *>(nd.scratch);
@@ -733,7 +747,9 @@ extern "C" vie_status vie_head_topk_noalloc(const void *W_out, int64_t V, int32_
         int pct = knobs().static_pct;
         pct = pct < 0 ? 0 : (pct > 100 ? 100 : pct);
         p.static_chunks = static_cast<int32_t>(n_chunks * pct / 100 / G);
+        p.pool_rows = pool_rows_for(shp.rs);
         p.cand = reinterpret_cast<uint64_t *>(nd.scratch + kNoAllocCounterBytes);
+        p.heads = p.cand + static_cast<size_t>(nb_max) * G * k;
         p.ticket = counters;
         p.next_chunk = counters + 2;
         p.err = nd.flag;

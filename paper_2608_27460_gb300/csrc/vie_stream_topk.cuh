@@ -50,7 +50,7 @@ constexpr int kMergePrefixCap = 2048;  // keys: first-J prefixes of all lists
 constexpr int kMergeCandCap = 2048;    // keys: gathered candidates
 constexpr int kRankCountMax = 640;     // rank counting below this many keys
 constexpr int kMaxLists = 1024;        // G <= 1024 CTAs
-constexpr int kFastE = 4;              // fast merge: entries read per list
+constexpr int kFastE = 4;              // fast merge: entries read per list (even)
 constexpr int kFastMaxK = 64;          // fast merge: largest k
 
 struct StreamTopkParams {
@@ -63,7 +63,9 @@ struct StreamTopkParams {
     int32_t rows_per_stage;  // RS <= 8 * R: rows of one chunk / weight stage
     int32_t stages;          // S, weight ring depth
     int32_t static_chunks;   // chunks each CTA owns before drawing from the pool
+    int32_t pool_rows;       // rows of a pool piece (<= rows_per_stage)
     uint64_t *cand;          // [NB][G][k] keys
+    uint64_t *heads;         // [NB][G][kFastE]: the first keys of each list
     uint32_t *ticket;        // CTA completion counter (self-resetting)
     uint32_t *next_chunk;    // pool counter (self-resetting)
     uint32_t *err;           // device flag word
@@ -103,8 +105,8 @@ struct MiscSmem {
     unsigned long long prefix;
     unsigned int tau_v;
     int overflow;
-    int chunk_w[kMaxStages];     // chunk id of each weight stage (-1: end)
-    int chunk_s[kScoreStages];   // chunk id of each score stage (-1: end)
+    int chunk_w[kMaxStages];     // first row of each weight stage (-1: end)
+    int chunk_s[kScoreStages];   // first row of each score stage (-1: end)
 };
 
 __device__ __forceinline__ uint32_t atomic_add_acq_rel_gpu(uint32_t *p, uint32_t v) {
@@ -490,7 +492,8 @@ __device__ inline bool merge_fast_query(const uint64_t *fe, const uint32_t *hv, 
 // entries of every list of every query (thread c: list c), then each query
 // is merged in shared memory; a query the fast merge cannot settle is merged
 // in full.  Called by every thread of one CTA of at least kThreads threads.
-__device__ inline void merge_queries(const uint64_t *cand, int nq, int G, int k, int64_t V,
+__device__ inline void merge_queries(const uint64_t *cand, const uint64_t *heads, int nq, int G,
+                                     int k, int64_t V,
                                      unsigned char *ws, uint32_t merge_bytes, MiscSmem *ms,
                                      int32_t *out_idx, float *out_logits, float *sparse) {
     const int tid = threadIdx.x;
@@ -511,14 +514,18 @@ __device__ inline void merge_queries(const uint64_t *cand, int nq, int G, int k,
     if (fast) {
         uint64_t *fe = staged;                                             // [nq][G][E]
         uint32_t *hv = reinterpret_cast<uint32_t *>(fe + nq * G * kFastE);  // [nq][G8]
-        const int En = k < kFastE ? k : kFastE;
         for (int q = 0; q < nq; ++q) {
             uint64_t key[kFastE];
             if (tid < G8) {
-                const unsigned long long *lc = reinterpret_cast<const unsigned long long *>(cand) +
-                                               (static_cast<size_t>(q) * G + tid) * k;
+                // list tid's first keys from the heads area: rows of 32 bytes
+                const ulonglong2 *hq = reinterpret_cast<const ulonglong2 *>(heads) +
+                                       (static_cast<size_t>(q) * G + tid) * (kFastE / 2);
 #pragma unroll
-                for (int e = 0; e < kFastE; ++e) key[e] = (tid < G && e < En) ? __ldcg(lc + e) : 0ull;
+                for (int e = 0; e < kFastE; e += 2) {
+                    const ulonglong2 x = tid < G ? __ldcg(hq + e / 2) : make_ulonglong2(0ull, 0ull);
+                    key[e] = x.x;
+                    key[e + 1] = x.y;
+                }
             }
             if (q == 0) merge_fast_reset(mb.counts, ms);  // while the loads are in flight
             if (tid < G8) {
@@ -571,6 +578,14 @@ __device__ inline void merge_queries(const uint64_t *cand, int nq, int G, int k,
 }
 
 // --------------------------------------------------------------------------
+// Rows of the stage that starts at row0: whole chunks (RS rows) in the
+// round-robin part, pool pieces (RSH rows) behind it, and never past the
+// vocabulary.
+__device__ __forceinline__ int stage_rows(int64_t row0, int64_t pool_row0, int RS, int RSH, int64_t V) {
+    const int64_t len = row0 < pool_row0 ? RS : RSH;
+    return static_cast<int>(min(len, V - row0));
+}
+
 template <int NB, int MM, int R>
 __global__ void __launch_bounds__(kThreads, 1) stream_topk_kernel(const StreamTopkParams p) {
     extern __shared__ __align__(128) unsigned char smem[];
@@ -593,7 +608,8 @@ __global__ void __launch_bounds__(kThreads, 1) stream_topk_kernel(const StreamTo
     const int lane = tid & 31;
     const int G = gridDim.x;
     const int cta = blockIdx.x;
-    const int n_chunks = static_cast<int>((p.V + RS - 1) / RS);
+    const int RSH = p.pool_rows;  // rows of a pool piece
+    const int64_t pool_row0 = static_cast<int64_t>(G) * p.static_chunks * RS;
     const int C = p.d_pad >> 3;  // 16-byte chunks per row
     const int stage_bytes = RS * row_bytes;
 
@@ -633,32 +649,30 @@ __global__ void __launch_bounds__(kThreads, 1) stream_topk_kernel(const StreamTo
             const uint64_t pol = l2_evict_first_policy();
             const unsigned char *W = reinterpret_cast<const unsigned char *>(p.W);
             const int Ns = p.static_chunks;
-            const int pool0 = G * Ns;
             // first draw from the pool, issued early so its latency is hidden
             uint32_t draw = (Ns == 0) ? atomic_add_relaxed_gpu(p.next_chunk, 1u) : 0u;
             int issued = 0;
             bool ok = true;
             for (int t = 0;; ++t) {
-                int chunk;
+                int64_t row0;
                 if (t < Ns) {
-                    chunk = t * G + cta;
+                    row0 = static_cast<int64_t>(t * G + cta) * RS;
                 } else {
-                    chunk = pool0 + static_cast<int>(draw);
-                    if (chunk >= n_chunks) chunk = -1;
+                    row0 = pool_row0 + static_cast<int64_t>(draw) * RSH;
+                    if (row0 >= p.V) row0 = -1;
                 }
                 const int s = t % S, u = t / S;
                 if (t >= S && !mbar_wait(&empty[s], (u - 1) & 1, abort_flag)) {
                     ok = false;
                     break;
                 }
-                ms->chunk_w[s] = chunk;
-                if (chunk < 0) {
+                ms->chunk_w[s] = static_cast<int>(row0);
+                if (row0 < 0) {
                     mbar_arrive(&full[s]);  // closes the stream: no bytes
                     break;
                 }
-                const int64_t row0 = static_cast<int64_t>(chunk) * RS;
-                const int64_t rows = min(static_cast<int64_t>(RS), p.V - row0);
-                const uint32_t bytes = static_cast<uint32_t>(rows * row_bytes);
+                const int rows = stage_rows(row0, pool_row0, RS, RSH, p.V);
+                const uint32_t bytes = static_cast<uint32_t>(rows) * row_bytes;
                 mbar_arrive_expect_tx(&full[s], bytes);
                 bulk_g2s(ring + s * stage_bytes, W + row0 * row_bytes, bytes, &full[s], pol);
                 issued = t + 1;
@@ -707,8 +721,8 @@ __global__ void __launch_bounds__(kThreads, 1) stream_topk_kernel(const StreamTo
                 }
                 const int chunk = ms->chunk_s[s];
                 if (chunk < 0) break;
-                const int64_t row0 = static_cast<int64_t>(chunk) * RS;
-                const int rows = static_cast<int>(min(static_cast<int64_t>(RS), p.V - row0));
+                const int64_t row0 = chunk;
+                const int rows = stage_rows(row0, pool_row0, RS, RSH, p.V);
                 const float *sc = scores + s * RS * NB;
 #pragma unroll
                 for (int nb = 0; nb < NB; ++nb) {
@@ -736,10 +750,12 @@ __global__ void __launch_bounds__(kThreads, 1) stream_topk_kernel(const StreamTo
 #pragma unroll
             for (int nb = 0; nb < NB; ++nb) {
                 uint64_t *dst = p.cand + (static_cast<size_t>(nb) * G + cta) * p.k;
+                uint64_t *head = p.heads + (static_cast<size_t>(nb) * G + cta) * kFastE;
 #pragma unroll
                 for (int s = 0; s < MM; ++s) {
                     const int pos = lane * MM + s;
                     if (pos < p.k) dst[pos] = list[nb].v[s];
+                    if (pos < kFastE) head[pos] = pos < p.k ? list[nb].v[s] : 0ull;
                 }
             }
         } else {
@@ -757,8 +773,8 @@ __global__ void __launch_bounds__(kThreads, 1) stream_topk_kernel(const StreamTo
                 }
                 const int chunk = ms->chunk_w[s];
                 if (chunk < 0) break;
-                const int64_t row0 = static_cast<int64_t>(chunk) * RS;
-                const int rows = static_cast<int>(min(static_cast<int64_t>(RS), p.V - row0));
+                const int64_t row0 = chunk;
+                const int rows = stage_rows(row0, pool_row0, RS, RSH, p.V);
                 const unsigned char *stage = ring + s * stage_bytes;
                 // warp w owns rows w, w + 8, ... (at most R of them) of the stage
                 int rr[R];
@@ -864,7 +880,7 @@ __global__ void __launch_bounds__(kThreads, 1) stream_topk_kernel(const StreamTo
     // Every CTA wrote a full list (valid keys or zeros) even if it gave up on
     // a wait, so the merge stays in bounds; such a call is reported through
     // the device flag and its outputs are unspecified.
-    merge_queries(p.cand, p.nq, G, p.k, p.V, smem + L.merge, L.total - L.merge, ms, p.out_idx,
+    merge_queries(p.cand, p.heads, p.nq, G, p.k, p.V, smem + L.merge, L.total - L.merge, ms, p.out_idx,
                       p.out_logits, p.sparse);
     if (tid == 0) {
         *p.ticket = 0;  // re-arm both counters for the next launch
