@@ -13,6 +13,11 @@ only builds it with gcc and marshals numpy arrays through ctypes.
                        first k rows                               (Sections 2, 3)
   * :func:`scatter` -- sparse full-vocabulary tensor, -inf except the k
                        retrieved logits at their indices          (Section 3)
+  * :func:`sample_sorted`, :func:`sample` -- top-k sampling with temperature,
+                       top-p and min-p on the k candidates, one uniform per
+                       draw                                       (Sections 2-4)
+  * :func:`philox4x32_10`, :func:`uniform` -- the counter-based generator that
+                       gives each (seed, step, query) its uniform
 
 Parity of :func:`topk` against the paper cannot be pinned to printed values
 (the paper prints no worked example); it is pinned instead to hand-worked
@@ -78,6 +83,13 @@ class OracleLib:
         lib.oracle_scatter.restype = ctypes.c_int
         lib.oracle_max_threads.argtypes = []
         lib.oracle_max_threads.restype = ctypes.c_int
+        lib.oracle_philox4x32_10.argtypes = [P, P, P]
+        lib.oracle_philox4x32_10.restype = None
+        lib.oracle_uniform.argtypes = [ctypes.c_uint64, ctypes.c_uint64, ctypes.c_uint32]
+        lib.oracle_uniform.restype = ctypes.c_double
+        D = ctypes.c_double
+        lib.oracle_sample_sorted.argtypes = [P, ctypes.c_int32, D, D, D, D, P, P, P]
+        lib.oracle_sample_sorted.restype = ctypes.c_int
         self.lib = lib
         self.path = path
 
@@ -128,6 +140,42 @@ class OracleLib:
         return out, rc == 0
 
 
+    def philox4x32_10(self, ctr, key):
+        """Philox4x32-10 of a 4-word counter and a 2-word key: 4 uint32 words."""
+        c = np.ascontiguousarray(ctr, dtype=np.uint32)
+        kk = np.ascontiguousarray(key, dtype=np.uint32)
+        out = np.empty(4, dtype=np.uint32)
+        self.lib.oracle_philox4x32_10(_ptr(c), _ptr(kk), _ptr(out))
+        return out
+
+    def uniform(self, seed: int, step: int, q: int) -> float:
+        """The uniform in [0, 1) of query q at decode step `step` under `seed`."""
+        return float(self.lib.oracle_uniform(seed & (2**64 - 1), step & (2**64 - 1), q))
+
+    def sample_sorted(self, z, T: float, top_p: float, min_p: float, u: float):
+        """One draw from sorted candidate logits z: (position j, its
+        probability among the kept candidates, number kept)."""
+        z = np.ascontiguousarray(z, dtype=np.float64)
+        j = ctypes.c_int32()
+        prob = ctypes.c_double()
+        kept = ctypes.c_int32()
+        rc = self.lib.oracle_sample_sorted(_ptr(z), z.shape[0], T, top_p, min_p, u,
+                                           ctypes.byref(j), ctypes.byref(prob), ctypes.byref(kept))
+        if rc != 0:
+            raise ValueError(f"oracle_sample_sorted failed with code {rc}")
+        return j.value, prob.value, kept.value
+
+    def sample(self, z, T: float, top_p: float, min_p: float, seed: int, step: int):
+        """Draws for a batch of sorted candidate rows z [batch, k], query q
+        using uniform(seed, step, q): (positions, probabilities, kept, u)."""
+        z = np.atleast_2d(np.asarray(z, dtype=np.float64))
+        res = [self.sample_sorted(z[q], T, top_p, min_p, self.uniform(seed, step, q))
+               for q in range(z.shape[0])]
+        u = np.array([self.uniform(seed, step, q) for q in range(z.shape[0])])
+        return (np.array([r[0] for r in res], np.int32), np.array([r[1] for r in res]),
+                np.array([r[2] for r in res], np.int32), u)
+
+
 def _default() -> OracleLib:
     global _lib
     with _lock:
@@ -154,3 +202,19 @@ def topk(W_bits, h, k: int, threads: int = 0):
 
 def scatter(idx, logits_f32, V: int):
     return _default().scatter(idx, logits_f32, V)
+
+
+def philox4x32_10(ctr, key):
+    return _default().philox4x32_10(ctr, key)
+
+
+def uniform(seed: int, step: int, q: int) -> float:
+    return _default().uniform(seed, step, q)
+
+
+def sample_sorted(z, T: float, top_p: float, min_p: float, u: float):
+    return _default().sample_sorted(z, T, top_p, min_p, u)
+
+
+def sample(z, T: float, top_p: float, min_p: float, seed: int, step: int):
+    return _default().sample(z, T, top_p, min_p, seed, step)

@@ -26,6 +26,21 @@
  *
  * Rows are independent, so the row loop may run on several OpenMP threads;
  * that changes no arithmetic of any single z_i.
+ *
+ * Top-k sampling (Section 2: top-k sampling restricts the draw to the k most
+ * probable tokens; Section 3: the retrieved logits feed standard logit
+ * processors such as top-p and min-p as a second stage; Section 4 samples
+ * with k = 50).  The paper names no random generator and no processor order;
+ * the readings taken (also listed in the design doc) are:
+ *   - probabilities are the softmax of z / T over the k candidates;
+ *   - top-p and min-p are both defined on that softmax, so each keeps a
+ *     prefix of the candidates (they are sorted by logit) and the kept set is
+ *     the shorter prefix: the two filters commute;
+ *   - the draw is the inverse CDF of the kept probabilities at one uniform u;
+ *   - u comes from the counter-based generator Philox4x32-10 (Salmon, Moraes,
+ *     Dror, Shaw, "Parallel random numbers: as easy as 1, 2, 3", SC 2011):
+ *     counter (step low, step high, query, 0), key (seed low, seed high), the
+ *     top 24 bits of the first output word times 2^-24.
  */
 #include <math.h>
 #include <stdint.h>
@@ -152,3 +167,100 @@ int oracle_max_threads(void) {
     return 1;
 #endif
 }
+
+/* ------------------------------------------------------------------------ */
+/* Philox4x32-10: ten rounds; a round multiplies words 0 and 2 by the two
+ * published constants into 64-bit products and mixes the halves with words
+ * 1 and 3 and the key; the key is bumped by the two published Weyl
+ * constants between rounds. */
+void oracle_philox4x32_10(const uint32_t ctr[4], const uint32_t key[2], uint32_t out[4]) {
+    uint32_t c0 = ctr[0], c1 = ctr[1], c2 = ctr[2], c3 = ctr[3];
+    uint32_t k0 = key[0], k1 = key[1];
+    for (int r = 0; r < 10; ++r) {
+        if (r > 0) {
+            k0 += 0x9E3779B9u;
+            k1 += 0xBB67AE85u;
+        }
+        const uint64_t p0 = (uint64_t)0xD2511F53u * c0;
+        const uint64_t p1 = (uint64_t)0xCD9E8D57u * c2;
+        const uint32_t n0 = (uint32_t)(p1 >> 32) ^ c1 ^ k0;
+        const uint32_t n1 = (uint32_t)p1;
+        const uint32_t n2 = (uint32_t)(p0 >> 32) ^ c3 ^ k1;
+        const uint32_t n3 = (uint32_t)p0;
+        c0 = n0;
+        c1 = n1;
+        c2 = n2;
+        c3 = n3;
+    }
+    out[0] = c0;
+    out[1] = c1;
+    out[2] = c2;
+    out[3] = c3;
+}
+
+/* The uniform of query q at decode step `step` under `seed`, in [0, 1). */
+double oracle_uniform(uint64_t seed, uint64_t step, uint32_t q) {
+    const uint32_t ctr[4] = {(uint32_t)step, (uint32_t)(step >> 32), q, 0u};
+    const uint32_t key[2] = {(uint32_t)seed, (uint32_t)(seed >> 32)};
+    uint32_t out[4];
+    oracle_philox4x32_10(ctr, key, out);
+    return (double)(out[0] >> 8) * (1.0 / 16777216.0);
+}
+
+/*
+ * One draw from the k candidate logits z[0..k), sorted descending:
+ *   s_j = z_j / T;  p_j = exp(s_j - s_0) / sum_i exp(s_i - s_0)
+ *   top-p: n_p = the smallest n >= 1 with sum_{i<n} p_i >= top_p
+ *   min-p: n_m = the number of j with p_j >= min_p * p_0
+ *   n = min(n_p, n_m);  M = sum_{i<n} p_i
+ *   j* = the smallest j < n with sum_{i<=j} p_i > u * M (n - 1 if none)
+ * Writes j*, p_{j*} / M and n.  Requires T > 0, 0 < top_p <= 1,
+ * 0 <= min_p <= 1, 0 <= u < 1.
+ */
+int oracle_sample_sorted(const double *z, int32_t k, double T, double top_p, double min_p,
+                         double u, int32_t *j_out, double *prob_out, int32_t *kept_out) {
+    if (!z || !j_out || !prob_out || !kept_out || k < 1) return ORACLE_EINVAL;
+    if (!(T > 0.0) || !(top_p > 0.0 && top_p <= 1.0) || !(min_p >= 0.0 && min_p <= 1.0) ||
+        !(u >= 0.0 && u < 1.0))
+        return ORACLE_EINVAL;
+    double *p = (double *)malloc(sizeof(double) * (size_t)k);
+    if (!p) return ORACLE_ENOMEM;
+    const double s0 = z[0] / T;
+    double total = 0.0;
+    for (int32_t j = 0; j < k; ++j) {
+        p[j] = exp(z[j] / T - s0);
+        total += p[j];
+    }
+    for (int32_t j = 0; j < k; ++j) p[j] /= total;
+    int32_t n_p = k;
+    double run = 0.0;
+    for (int32_t n = 1; n <= k; ++n) {
+        run += p[n - 1];
+        if (run >= top_p) {
+            n_p = n;
+            break;
+        }
+    }
+    int32_t n_m = 0;
+    for (int32_t j = 0; j < k; ++j)
+        if (p[j] >= min_p * p[0]) ++n_m;
+    const int32_t n = n_p < n_m ? n_p : n_m;
+    double M = 0.0;
+    for (int32_t j = 0; j < n; ++j) M += p[j];
+    const double target = u * M;
+    int32_t js = n - 1;
+    double cum = 0.0;
+    for (int32_t j = 0; j < n; ++j) {
+        cum += p[j];
+        if (cum > target) {
+            js = j;
+            break;
+        }
+    }
+    *j_out = js;
+    *prob_out = p[js] / M;
+    *kept_out = n;
+    free(p);
+    return ORACLE_OK;
+}
+

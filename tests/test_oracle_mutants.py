@@ -11,6 +11,7 @@ import pytest
 
 import oracle as default_oracle
 from test_oracle_pins import PINS
+from test_oracle_sampling import SAMPLING_PINS
 
 SRC = os.path.join(os.path.dirname(default_oracle.__file__), "oracle.c")
 
@@ -30,6 +31,16 @@ MUTANTS = {
     "unsorted_logit_copy": ("logits[(int64_t)b * k + j] = rows[j].z;", "logits[(int64_t)b * k + j] = z[j];"),
     "zero_fill_not_neg_inf": ("row[v] = -INFINITY;", "row[v] = 0.0f;"),
     "no_range_check": ("if (t < 0 || (int64_t)t >= V) {", "if (t < 0) {"),
+    # top-k sampling and its generator
+    "philox_wrong_multiplier": ("(uint64_t)0xD2511F53u * c0", "(uint64_t)0xD2511F55u * c0"),
+    "philox_key_not_bumped": ("k1 += 0xBB67AE85u;", "k1 += 0u;"),
+    "philox_words_swapped": ("const uint32_t n1 = (uint32_t)p1;", "const uint32_t n1 = (uint32_t)p0;"),
+    "uniform_wrong_bits": ("(double)(out[0] >> 8) * (1.0 / 16777216.0)", "(double)(out[1] >> 8) * (1.0 / 16777216.0)"),
+    "temperature_dropped": ("p[j] = exp(z[j] / T - s0);", "p[j] = exp(z[j] - s0);"),
+    "top_p_strict": ("if (run >= top_p) {", "if (run > top_p) {"),
+    "min_p_absolute": ("if (p[j] >= min_p * p[0]) ++n_m;", "if (p[j] >= min_p) ++n_m;"),
+    "draw_at_or_above": ("if (cum > target) {", "if (cum >= target) {"),
+    "prob_not_renormalised": ("*prob_out = p[js] / M;", "*prob_out = p[js];"),
 }
 
 
@@ -42,7 +53,7 @@ def test_pins_catch_planted_mistake(name, tmp_path):
     src.write_text(text.replace(old, new, 1))
     lib = default_oracle.OracleLib(default_oracle.build(True, str(src), str(tmp_path / f"{name}.so")))
     caught = []
-    for pin_name, pin in PINS:
+    for pin_name, pin in PINS + SAMPLING_PINS:
         try:
             pin(lib)
         except (AssertionError, ValueError):
