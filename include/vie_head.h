@@ -168,6 +168,50 @@ vie_status vie_head_topk_host(vie_head *head, const float *h_host, int32_t batch
                               vie_stream stream);
 
 /*
+ * vie_sample_topk - top-k sampling on the k candidates of each query
+ * (Section 2: top-k sampling draws the next token from the k most probable
+ * tokens; Section 3: top-p and min-p act as a second stage on the retrieved
+ * logits; Section 4 samples with k = 50).  Per query, in fp32:
+ *   p_j = softmax of logits[j] / temperature over the k candidates;
+ *   top-p keeps the shortest prefix whose probability reaches top_p (at
+ *   least one candidate); min-p keeps the candidates with p_j >= min_p * p_0;
+ *   the kept set is the shorter prefix of the two;
+ *   the token is the first kept candidate j whose cumulative probability
+ *   exceeds u * (kept mass), where u in [0, 1) is the top 24 bits of the first
+ *   output word of Philox4x32-10 (Salmon et al., SC 2011) at counter
+ *   (step low, step high, query, 0) with key (seed low, seed high), times
+ *   2^-24: the same (seed, step) gives the same draws, a new step new ones.
+ *
+ *   idx, logits  device, int32 / fp32 [batch, k]: candidates sorted by logit,
+ *                best first, as vie_head_topk returns them (4-byte aligned).
+ *   batch >= 1;  1 <= k <= VIE_K_MAX.
+ *   temperature  > 0 and finite;  0 < top_p <= 1;  0 <= min_p <= 1.
+ *   out_token    device, int32 [batch]: the drawn vocabulary index.
+ *   out_prob     device, fp32 [batch]: its probability among the kept
+ *                candidates.
+ *   stream       the stream the work is enqueued on.
+ *
+ * The launch may start while the previous kernel on the stream finishes
+ * (programmatic dependent launch); it reads idx and logits only after that
+ * kernel has completed.  No allocation, no sync.
+ */
+vie_status vie_sample_topk(const int32_t *idx, const float *logits, int32_t batch, int32_t k,
+                           float temperature, float top_p, float min_p, uint64_t seed,
+                           uint64_t step, int32_t *out_token, float *out_prob, vie_stream stream);
+
+/*
+ * vie_head_topk_sample - vie_head_topk_sparse (or vie_head_topk when
+ * out_sparse is NULL) followed by vie_sample_topk on its output: the whole
+ * decode-step head with the next token drawn on the device.  Arguments as for
+ * those two calls; k <= VIE_K_MAX.
+ */
+vie_status vie_head_topk_sample(vie_head *head, const float *h, int32_t batch, int32_t k,
+                                float temperature, float top_p, float min_p, uint64_t seed,
+                                uint64_t step, int32_t *out_idx, float *out_logits,
+                                float *out_sparse, int32_t *out_token, float *out_prob,
+                                vie_stream stream);
+
+/*
  * vie_scatter_sparse_logits - the sparse full-vocabulary logit tensor of
  * Section 3: out[b, v] = -inf (bit pattern 0xFF800000) for every v, then
  * out[b, idx[b, j]] = logits[b, j] for j < k (values copied bit for bit).

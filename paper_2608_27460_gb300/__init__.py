@@ -36,8 +36,9 @@ STATUS_NAMES = {0: "VIE_OK", 1: "VIE_ERR_INVALID_ARG", 2: "VIE_ERR_UNSUPPORTED",
 
 # Every entry point of include/vie_head.h.
 EXPORTS = ("vie_head_create", "vie_head_destroy", "vie_head_get_props", "vie_head_plan", "vie_head_topk",
-           "vie_head_topk_sparse", "vie_head_topk_host", "vie_head_topk_noalloc", "vie_scatter_sparse_logits",
-           "vie_device_status", "vie_head_device_status", "vie_last_error")
+           "vie_head_topk_sparse", "vie_head_topk_host", "vie_sample_topk", "vie_head_topk_sample",
+           "vie_head_topk_noalloc", "vie_scatter_sparse_logits", "vie_device_status",
+           "vie_head_device_status", "vie_last_error")
 
 
 class VieError(RuntimeError):
@@ -78,6 +79,7 @@ def load(path: str | None = None, build_if_missing: bool = True):
                                "(run python -m paper_2608_27460_gb300.build)")
         lib = ctypes.CDLL(p)
         P, I32, I64 = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64
+        F32, U64 = ctypes.c_float, ctypes.c_uint64
         sig = {
             "vie_head_create": ([P, I64, I32, ctypes.c_int, ctypes.POINTER(P)], ctypes.c_int),
             "vie_head_destroy": ([P], ctypes.c_int),
@@ -86,6 +88,9 @@ def load(path: str | None = None, build_if_missing: bool = True):
             "vie_head_topk": ([P, P, I32, I32, P, P, P], ctypes.c_int),
             "vie_head_topk_sparse": ([P, P, I32, I32, P, P, P, P], ctypes.c_int),
             "vie_head_topk_host": ([P, P, I32, I32, P, P, P, P], ctypes.c_int),
+            "vie_sample_topk": ([P, P, I32, I32, F32, F32, F32, U64, U64, P, P, P], ctypes.c_int),
+            "vie_head_topk_sample": ([P, P, I32, I32, F32, F32, F32, U64, U64, P, P, P, P, P, P],
+                                     ctypes.c_int),
             "vie_head_topk_noalloc": ([P, I64, I32, P, I32, I32, P, P, P], ctypes.c_int),
             "vie_scatter_sparse_logits": ([P, P, I32, I32, I64, P, P], ctypes.c_int),
             "vie_device_status": ([P], ctypes.c_int),
@@ -146,6 +151,36 @@ def vie_head_topk_sparse(head: int, h: int, batch: int, k: int, out_idx: int, ou
 def vie_head_topk_host(head: int, h_host: int, batch: int, k: int, idx_host: int, logits_host: int,
                        out_sparse: int = 0, stream: int = 0) -> int:
     return load().vie_head_topk_host(head, h_host, batch, k, idx_host, logits_host, out_sparse, stream)
+
+
+def vie_sample_topk(idx: int, logits: int, batch: int, k: int, temperature: float, top_p: float,
+                    min_p: float, seed: int, step: int, out_token: int, out_prob: int,
+                    stream: int = 0) -> int:
+    return load().vie_sample_topk(idx, logits, batch, k, temperature, top_p, min_p,
+                                  seed & (2**64 - 1), step & (2**64 - 1), out_token, out_prob, stream)
+
+
+def vie_head_topk_sample(head: int, h: int, batch: int, k: int, temperature: float, top_p: float,
+                         min_p: float, seed: int, step: int, out_idx: int, out_logits: int,
+                         out_sparse: int, out_token: int, out_prob: int, stream: int = 0) -> int:
+    return load().vie_head_topk_sample(head, h, batch, k, temperature, top_p, min_p,
+                                       seed & (2**64 - 1), step & (2**64 - 1), out_idx, out_logits,
+                                       out_sparse, out_token, out_prob, stream)
+
+
+def sample_topk(idx, logits, temperature: float = 1.0, top_p: float = 1.0, min_p: float = 0.0,
+                seed: int = 0, step: int = 0, out_token=None, out_prob=None, stream=None):
+    """Top-k sampling on CUDA candidates (int32 / float32 [batch, k], sorted
+    best first): returns (token int32 [batch], probability float32 [batch])."""
+    import torch
+    b, k = int(idx.shape[0]), int(idx.shape[1])
+    if out_token is None:
+        out_token = torch.empty((b,), dtype=torch.int32, device=idx.device)
+    if out_prob is None:
+        out_prob = torch.empty((b,), dtype=torch.float32, device=idx.device)
+    check(vie_sample_topk(idx.data_ptr(), logits.data_ptr(), b, k, temperature, top_p, min_p, seed,
+                          step, out_token.data_ptr(), out_prob.data_ptr(), _stream_ptr(stream)))
+    return out_token, out_prob
 
 
 def vie_head_topk_noalloc(W_out: int, V: int, d: int, h: int, batch: int, k: int, out_idx: int,
@@ -271,6 +306,26 @@ class Head:
         check(vie_head_topk_host(self.handle, h.data_ptr(), b, k, out_idx.data_ptr(),
                                  out_logits.data_ptr(), sp, _stream_ptr(stream)))
         return out_idx, out_logits
+
+    def topk_sample(self, h, k: int, temperature: float = 1.0, top_p: float = 1.0,
+                    min_p: float = 0.0, seed: int = 0, step: int = 0, out_sparse=None, stream=None):
+        """Top-k of W h, then one draw per query: (idx, logits, token, prob)."""
+        import torch
+        if h.dim() == 1:
+            h = h[None]
+        if h.dtype != torch.float32 or not h.is_cuda or h.shape[1] != self.d:
+            raise ValueError(f"h must be a CUDA float32 tensor [batch, {self.d}]")
+        h = h.contiguous()
+        b = int(h.shape[0])
+        idx = torch.empty((b, k), dtype=torch.int32, device=h.device)
+        val = torch.empty((b, k), dtype=torch.float32, device=h.device)
+        tok = torch.empty((b,), dtype=torch.int32, device=h.device)
+        prob = torch.empty((b,), dtype=torch.float32, device=h.device)
+        sp = 0 if out_sparse is None else out_sparse.data_ptr()
+        check(vie_head_topk_sample(self.handle, h.data_ptr(), b, k, temperature, top_p, min_p, seed,
+                                   step, idx.data_ptr(), val.data_ptr(), sp, tok.data_ptr(),
+                                   prob.data_ptr(), _stream_ptr(stream)))
+        return idx, val, tok, prob
 
     def sparse_logits(self, idx, logits, out=None, stream=None):
         """Sparse [batch, V] fp32 tensor: -inf except logits at idx."""

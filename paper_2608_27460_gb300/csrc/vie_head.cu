@@ -4,6 +4,7 @@
 #include <cuda_runtime.h>
 
 #include <climits>
+#include <cmath>
 #include <cstdarg>
 #include <cstdint>
 #include <cstdio>
@@ -520,6 +521,51 @@ vie_status vie_head_topk_sparse(vie_head *head, const float *h, int32_t batch, i
         return fail(VIE_ERR_INVALID_ARG, "vie_head_topk_sparse: out_sparse is NULL");
     return run_topk("vie_head_topk_sparse", head, h, batch, k, out_idx, out_logits, out_sparse,
                     stream);
+}
+
+vie_status vie_sample_topk(const int32_t *idx, const float *logits, int32_t batch, int32_t k,
+                           float temperature, float top_p, float min_p, uint64_t seed,
+                           uint64_t step, int32_t *out_token, float *out_prob, vie_stream stream) {
+    const char *fn = "vie_sample_topk";
+    if (idx == nullptr || logits == nullptr || out_token == nullptr || out_prob == nullptr)
+        return fail(VIE_ERR_INVALID_ARG, "%s: NULL buffer", fn);
+    if (batch < 1) return fail(VIE_ERR_INVALID_ARG, "%s: batch=%d < 1", fn, batch);
+    if (k < 1 || k > VIE_K_MAX)
+        return fail(VIE_ERR_INVALID_ARG, "%s: k=%d outside [1, %d]", fn, k, VIE_K_MAX);
+    if (!(temperature > 0.0f) || !std::isfinite(temperature))
+        return fail(VIE_ERR_INVALID_ARG, "%s: temperature=%g must be positive and finite", fn,
+                    static_cast<double>(temperature));
+    if (!(top_p > 0.0f && top_p <= 1.0f))
+        return fail(VIE_ERR_INVALID_ARG, "%s: top_p=%g outside (0, 1]", fn, static_cast<double>(top_p));
+    if (!(min_p >= 0.0f && min_p <= 1.0f))
+        return fail(VIE_ERR_INVALID_ARG, "%s: min_p=%g outside [0, 1]", fn, static_cast<double>(min_p));
+    if ((reinterpret_cast<uintptr_t>(idx) | reinterpret_cast<uintptr_t>(logits) |
+         reinterpret_cast<uintptr_t>(out_token) | reinterpret_cast<uintptr_t>(out_prob)) & 3u)
+        return fail(VIE_ERR_INVALID_ARG, "%s: buffers must be 4-byte aligned", fn);
+    const cudaError_t e = vie::launch_sample_topk(idx, logits, batch, k, temperature, top_p, min_p,
+                                                  seed, step, out_token, out_prob,
+                                                  static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return fail_cuda(e, fn);
+    return VIE_OK;
+}
+
+vie_status vie_head_topk_sample(vie_head *head, const float *h, int32_t batch, int32_t k,
+                                float temperature, float top_p, float min_p, uint64_t seed,
+                                uint64_t step, int32_t *out_idx, float *out_logits,
+                                float *out_sparse, int32_t *out_token, float *out_prob,
+                                vie_stream stream) {
+    const char *fn = "vie_head_topk_sample";
+    if (out_token == nullptr || out_prob == nullptr)
+        return fail(VIE_ERR_INVALID_ARG, "%s: NULL buffer", fn);
+    if (!(temperature > 0.0f) || !std::isfinite(temperature) || !(top_p > 0.0f && top_p <= 1.0f) ||
+        !(min_p >= 0.0f && min_p <= 1.0f))
+        return fail(VIE_ERR_INVALID_ARG, "%s: temperature=%g top_p=%g min_p=%g out of range", fn,
+                    static_cast<double>(temperature), static_cast<double>(top_p),
+                    static_cast<double>(min_p));
+    vie_status st = run_topk(fn, head, h, batch, k, out_idx, out_logits, out_sparse, stream);
+    if (st != VIE_OK) return st;
+    return vie_sample_topk(out_idx, out_logits, batch, k, temperature, top_p, min_p, seed, step,
+                           out_token, out_prob, stream);
 }
 
 vie_status vie_head_topk_host(vie_head *head, const float *h_host, int32_t batch, int32_t k,

@@ -30,6 +30,11 @@ struct TcParams;
 // Ring depth and dynamic shared memory of the tensor-core kernel for query
 // groups of nq_tmpl (8, 16 or 32) and kps K-blocks per stage; false if
 // unsupported.
+// Top-k sampling: one draw per query from its k sorted candidates.
+cudaError_t launch_sample_topk(const int32_t *idx, const float *logits, int batch, int k, float T,
+                               float top_p, float min_p, uint64_t seed, uint64_t step,
+                               int32_t *out_token, float *out_prob, cudaStream_t stream);
+
 // Largest k the tensor-core kernel with nq_tmpl query slots handles.
 int tc_max_k(int nq_tmpl);
 bool tc_shape(int nq_tmpl, int kps, int *stages, uint32_t *smem);

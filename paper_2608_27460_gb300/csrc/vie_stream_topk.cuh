@@ -625,6 +625,7 @@ __global__ void __launch_bounds__(kThreads, 1) stream_topk_kernel(const StreamTo
         ms->abort = 0;
         ms->is_last = 0;
         fence_mbar_init();
+        griddep_launch_dependents();  // a kernel launched after this one may be scheduled now
     }
     // h -> shared memory as [nb][half][chunk][4] so a lane's two float4 loads
     // of one chunk fall in distinct bank groups; zero pad, zero unused

@@ -106,13 +106,5 @@ __device__ __forceinline__ void tmem_wait_ld() {
     asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
 
-// Programmatic dependent launch: a kernel launched with programmatic stream
-// serialisation may start while the previous kernel on the stream still
-// runs; griddep_wait() blocks until that kernel has finished and its writes
-// are visible, griddep_launch_dependents() lets the next kernel start early.
-__device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
-__device__ __forceinline__ void griddep_launch_dependents() {
-    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-}
 
 }  // namespace vie

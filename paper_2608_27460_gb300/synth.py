@@ -134,3 +134,24 @@ def make_head(shape: HeadShape, seed: int = 0, n_queries: int = 16, planted_frac
     h, rows = make_queries(W, n_queries, seed + 1000 + offset, planted_frac=plant,
                            dup_src=meta["dup_src"])
     return W, h, meta, rows
+
+
+def make_candidates(batch: int, k: int, V: int, seed: int, spread: float = 3.0,
+                    ties: float = 0.0):
+    """Candidate rows for top-k sampling, shaped like a head's output:
+    distinct vocabulary indices per row (int32 [batch, k]) and fp32 logits
+    [batch, k] sorted best first, drawn N(0, spread^2); with ties > 0 about
+    that share of the logits repeats its neighbour's value exactly."""
+    rng = np.random.default_rng(seed)
+    idx = np.stack([rng.choice(V, size=k, replace=False) for _ in range(batch)]).astype(np.int32)
+    z = rng.normal(0.0, spread, size=(batch, k)).astype(np.float32)
+    if ties > 0 and k > 1:
+        rep = rng.random((batch, k)) < ties
+        rep[:, 0] = False
+        z = np.sort(z, axis=1)[:, ::-1].copy()
+        for b in range(batch):
+            for j in range(1, k):
+                if rep[b, j]:
+                    z[b, j] = z[b, j - 1]
+    z = np.sort(z, axis=1)[:, ::-1].astype(np.float32, order="C", copy=True)
+    return idx, z

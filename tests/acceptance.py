@@ -80,3 +80,45 @@ def check_batch(idx, val, z, k):
         if e:
             out[q] = e
     return out
+
+
+def check_draw(z, T, top_p, min_p, u, j, prob, tol=None):
+    """Acceptance of one top-k draw made in fp32: z the query's candidate
+    logits (sorted, best first), u its uniform, j the position drawn and
+    prob its reported probability.  The reference is the oracle's fp64
+    definition; where a decision lies within `tol` of a boundary (the
+    top-p or min-p cut, or the CDF crossing u * M) every outcome reachable
+    by moving that boundary by tol is accepted.  Returns a list of problems
+    (empty when the draw is acceptable)."""
+    import oracle
+    z = np.asarray(z, dtype=np.float64)
+    k = z.shape[0]
+    if tol is None:
+        tol = 1e-6 + 2e-7 * k
+    s = z / T
+    e = np.exp(s - s[0])
+    p = e / e.sum()
+    C = np.cumsum(p)
+    ok_n = set()
+    for tp_try in (top_p - tol, top_p, top_p + tol):
+        n_p = next((n for n in range(1, k + 1) if C[n - 1] >= min(tp_try, 1.0)), k)
+        for mp_try in (min_p - tol, min_p, min_p + tol):
+            n_m = int(np.sum(p >= max(mp_try, 0.0) * p[0]))
+            ok_n.add(max(1, min(n_p, n_m)))
+    ok_j = {}
+    for n in ok_n:
+        M = C[n - 1]
+        for ut in (u - tol, u, u + tol):
+            ut = min(max(ut, 0.0), 1.0 - 1e-12)
+            jj = next((i for i in range(n) if C[i] > ut * M), n - 1)
+            ok_j.setdefault(jj, []).append(p[jj] / M)
+    problems = []
+    if j not in ok_j:
+        problems.append(f"position {j} not drawable (acceptable {sorted(ok_j)})")
+    elif min(abs(prob - q) for q in ok_j[j]) > 1e-5 + 1e-4 * max(ok_j[j]):
+        problems.append(f"probability {prob} vs {ok_j[j]}")
+    # the oracle itself must be among the accepted outcomes
+    jo, po, _ = oracle.sample_sorted(z, T, top_p, min_p, u)
+    if jo not in ok_j:
+        problems.append(f"oracle draw {jo} outside the accepted set {sorted(ok_j)}")
+    return problems

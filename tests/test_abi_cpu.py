@@ -75,6 +75,28 @@ def test_scatter_rejects_bad_arguments_on_host(lib):
     assert vie.vie_scatter_sparse_logits(p + 2, p, 1, 1, 8, p) == vie.VIE_ERR_INVALID_ARG
 
 
+def test_sampling_rejects_bad_arguments_on_host(lib):
+    p = 0x10000
+    ok = dict(temperature=1.0, top_p=1.0, min_p=0.0)
+    def call(idx=p, logits=p, batch=1, k=50, out_token=p, out_prob=p, **kw):
+        a = dict(ok, **kw)
+        return vie.vie_sample_topk(idx, logits, batch, k, a["temperature"], a["top_p"], a["min_p"],
+                                   0, 0, out_token, out_prob)
+    assert call(idx=0) == vie.VIE_ERR_INVALID_ARG
+    assert call(out_prob=0) == vie.VIE_ERR_INVALID_ARG
+    assert call(batch=0) == vie.VIE_ERR_INVALID_ARG
+    assert call(k=0) == vie.VIE_ERR_INVALID_ARG
+    assert call(k=vie.VIE_K_MAX + 1) == vie.VIE_ERR_INVALID_ARG
+    assert call(temperature=0.0) == vie.VIE_ERR_INVALID_ARG
+    assert call(temperature=float("inf")) == vie.VIE_ERR_INVALID_ARG
+    assert call(top_p=0.0) == vie.VIE_ERR_INVALID_ARG
+    assert call(top_p=1.5) == vie.VIE_ERR_INVALID_ARG
+    assert call(min_p=-0.1) == vie.VIE_ERR_INVALID_ARG
+    assert call(min_p=1.1) == vie.VIE_ERR_INVALID_ARG
+    assert call(logits=p + 2) == vie.VIE_ERR_INVALID_ARG
+    assert vie.vie_head_topk_sample(0, p, 1, 50, 1.0, 1.0, 0.0, 0, 0, p, p, 0, p, p) == vie.VIE_ERR_INVALID_ARG
+
+
 def test_product_path_does_not_import_the_oracle():
     pkg = os.path.join(ROOT, "paper_2608_27460_gb300")
     for dirpath, _, files in os.walk(pkg):
