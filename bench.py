@@ -58,6 +58,9 @@ def parse_args(argv=None):
     ap.add_argument("--cpu-seconds", type=float, default=15.0, help="oracle sample budget")
     ap.add_argument("--e2e-steps", type=int, default=200)
     ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--sample", action="store_true",
+                    help="each step also draws the next token on the device (temperature 0.8, "
+                         "top-p 0.9, min-p 0.05, Philox keyed by the step)")
     ap.add_argument("--l2", choices=["flush", "resident"], default="flush",
                     help="flush: read a 256 MB buffer between timed steps (evicts W_out from L2 "
                          "with clean lines, like the other layers of a decode step would) and time "
@@ -227,6 +230,8 @@ def run_reference(args, rank, world):
         q0 = (i * args.batch) % (len(h) - args.batch + 1)
         idx, val = oracle.topk(W, h[q0:q0 + args.batch], args.k, threads=threads)
         oracle.scatter(idx, val.astype(np.float32), V)
+        if args.sample:
+            oracle.sample(val, 0.8, 0.9, 0.05, args.seed, i)
 
     for i in range(args.warmup):
         step(i)
@@ -251,7 +256,8 @@ def run_reference(args, rank, world):
 
 
 def workload_config(args, shape):
-    return {"workload": f"{shape.name}-shaped head, batch {args.batch}, k {args.k}",
+    return {"workload": f"{shape.name}-shaped head, batch {args.batch}, k {args.k}"
+                        + (", then a top-k draw" if getattr(args, "sample", False) else ""),
             "V": shape.V, "d": shape.d, "batch": args.batch, "k": args.k,
             "weights": "bf16 (fp32 accumulation)",
             "l2": ("flushed between timed steps (256 MB read); value = mean of per-step CUDA "
@@ -292,11 +298,22 @@ def main(argv=None):
     stream = torch.cuda.current_stream(dev)
     sptr = int(stream.cuda_stream)
     starts = [(i * b) % (nq - b + 1) for i in range(nq)]
+    tok = torch.empty((b,), dtype=torch.int32, device=dev)
+    prob = torch.empty((b,), dtype=torch.float32, device=dev)
+    SAMPLING = (0.8, 0.9, 0.05)  # temperature, top-p, min-p
+
+    def head_call(i):
+        q0 = starts[i % nq]
+        if args.sample:
+            vie.check(vie.vie_head_topk_sample(head.handle, hd[q0].data_ptr(), b, k, *SAMPLING,
+                                               args.seed, i, idx.data_ptr(), val.data_ptr(),
+                                               sparse.data_ptr(), tok.data_ptr(), prob.data_ptr(), sptr))
+        else:
+            vie.check(vie.vie_head_topk_sparse(head.handle, hd[q0].data_ptr(), b, k, idx.data_ptr(),
+                                               val.data_ptr(), sparse.data_ptr(), sptr))
 
     def step(i):
-        q0 = starts[i % nq]
-        vie.check(vie.vie_head_topk_sparse(head.handle, hd[q0].data_ptr(), b, k, idx.data_ptr(),
-                                           val.data_ptr(), sparse.data_ptr(), sptr))
+        head_call(i)
 
     sampler = ClockSampler(gpu_id_for_smi(local)) if rank == 0 else None
     if sampler:
@@ -324,8 +341,7 @@ def main(argv=None):
         if flush is not None:
             torch.sum(flush, dim=0, out=flush_sink)  # reads 256 MB: W_out leaves L2
         ev_a[i].record(stream)
-        vie.check(vie.vie_head_topk_sparse(head.handle, hd[q0].data_ptr(), b, k, idx.data_ptr(),
-                                           val.data_ptr(), sparse.data_ptr(), sptr))
+        head_call(i)
         ev_b[i].record(stream)
     end.record(stream)
     torch.cuda.synchronize()
@@ -383,7 +399,24 @@ def main(argv=None):
     kernel = "stream_topk" if plan.path == 0 else "tc_topk"
     traffic, prof_path = profiled_traffic(kernel, args.workload, b, k)
     value = whole_job_us_per_step(step_us, world)
-    launches_per_step = plan.launches
+    launches_per_step = plan.launches + (1 if args.sample else 0)
+    sample_info = None
+    if args.sample:
+        # the sampling kernel alone, on this step's candidates, back to back
+        sa, sb = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        for i in range(20):
+            vie.check(vie.vie_sample_topk(idx.data_ptr(), val.data_ptr(), b, k, *SAMPLING, args.seed, i,
+                                          tok.data_ptr(), prob.data_ptr(), sptr))
+        sa.record(stream)
+        for i in range(200):
+            vie.check(vie.vie_sample_topk(idx.data_ptr(), val.data_ptr(), b, k, *SAMPLING, args.seed, i,
+                                          tok.data_ptr(), prob.data_ptr(), sptr))
+        sb.record(stream)
+        torch.cuda.synchronize()
+        sample_info = {"temperature": SAMPLING[0], "top_p": SAMPLING[1], "min_p": SAMPLING[2],
+                       "draw": "inverse CDF at a Philox4x32-10 uniform keyed by (seed, step, query)",
+                       "sample_kernel_us_back_to_back": round(sa.elapsed_time(sb) * 1e3 / 200, 3),
+                       "step": "head (top-k and sparse tensor) then the draw, one call, PDL-chained"}
 
     line = {
         "metric": METRIC, "value": round(value, 3), "unit": UNIT, "n_gpus": world,
@@ -406,6 +439,7 @@ def main(argv=None):
                 "d2h_bytes_per_step": b * k * 8, "api": "vie_head_topk_host (pinned host h in, "
                 "top-k out, synchronised)", "clock": "host wall clock over the steps"},
         "gpu_launches": K * launches_per_step,
+        **({"sampling": sample_info} if sample_info else {}),
         "clocks": ClockSampler.summarize(clocks, t_wall0, t_wall1),
     }
     if plan.path == 1:
