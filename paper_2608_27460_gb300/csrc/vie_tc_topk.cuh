@@ -44,7 +44,7 @@ constexpr int kTcMaxK = 128;       // largest k of this path
 constexpr int kTcListKeys = 4096;  // keys of the per-CTA lists per CTA: NQ * k <= this
 constexpr int kTcMaxKPS = 4;       // K-blocks per stage, at most
 constexpr int kTcMergeE = 4;       // merge: keys per list in the heads area
-constexpr int kTcMaxMergers = 32;  // CTAs that merge, at most (one per query)
+constexpr int kTcMaxMergers = 64;  // CTAs that merge, at most (one per query)
 
 struct TcParams {
     int64_t V;
@@ -558,21 +558,27 @@ __global__ void __launch_bounds__(TcShape<NQ>::kThreads, 1)
             }
             if (lane == 0) mbar_arrive(&sempty[ss]);
         }
-#pragma unroll 1
-        for (int j = 0; j < QPW; ++j) {
-            const int q = QPW * sel + j;
-            if (q >= p.nq) break;
-            write_sorted_list<CAP_PER>(bufs + q * CAP, cnt_s[j], p.k, &tau_s[j],
-                              p.cand + (static_cast<size_t>(q) * G + cta) * p.k,
-                              p.heads + (static_cast<size_t>(q) * G + cta) * kTcMergeE, lane);
-        }
     }
 
+    // Every warp is free now: warp w sorts and writes the lists of queries
+    // w, w + kWarps, ... (each query's buffer, count and bound are in shared
+    // memory, next to one another).
     __syncthreads();
     if (warp == 1) {
         tc_fence_after_sync();
         tmem_dealloc(tmem, Sh::kTmemCols);
     }
+    {
+        constexpr int CAP = Sh::kCap, CAP_PER = CAP / 32;
+        int *cnt_all = reinterpret_cast<int *>(bufs + NQ * CAP);
+        uint64_t *tau_all = reinterpret_cast<uint64_t *>(bufs + NQ * CAP) + NQ / 2;
+#pragma unroll 1
+        for (int q = warp; q < p.nq; q += Sh::kWarps)
+            write_sorted_list<CAP_PER>(bufs + q * CAP, cnt_all[q], p.k, &tau_all[q],
+                                       p.cand + (static_cast<size_t>(q) * G + cta) * p.k,
+                                       p.heads + (static_cast<size_t>(q) * G + cta) * kTcMergeE, lane);
+    }
+    __syncthreads();
 
     // ---------------- completion ticket ----------------
     // bar.sync orders every thread's writes (lists, heads, sparse fill)
