@@ -18,6 +18,8 @@ only builds it with gcc and marshals numpy arrays through ctypes.
                        draw                                       (Sections 2-4)
   * :func:`philox4x32_10`, :func:`uniform` -- the counter-based generator that
                        gives each (seed, step, query) its uniform
+  * :func:`quantize_e4m3`, :func:`logits_e4m3`, :func:`topk_e4m3` -- the head
+                       on rows stored as e4m3 codes with one fp32 scale each
 
 Parity of :func:`topk` against the paper cannot be pinned to printed values
 (the paper prints no worked example); it is pinned instead to hand-worked
@@ -90,6 +92,18 @@ class OracleLib:
         D = ctypes.c_double
         lib.oracle_sample_sorted.argtypes = [P, ctypes.c_int32, D, D, D, D, P, P, P]
         lib.oracle_sample_sorted.restype = ctypes.c_int
+        lib.oracle_e4m3_to_double.argtypes = [ctypes.c_uint8]
+        lib.oracle_e4m3_to_double.restype = ctypes.c_double
+        lib.oracle_f32_to_e4m3.argtypes = [ctypes.c_float]
+        lib.oracle_f32_to_e4m3.restype = ctypes.c_uint8
+        lib.oracle_quantize_e4m3.argtypes = [P, ctypes.c_int64, ctypes.c_int32, P, P]
+        lib.oracle_quantize_e4m3.restype = ctypes.c_int
+        lib.oracle_logits_e4m3.argtypes = [P, P, ctypes.c_int64, ctypes.c_int32, P, ctypes.c_int32,
+                                           P, ctypes.c_int32]
+        lib.oracle_logits_e4m3.restype = ctypes.c_int
+        lib.oracle_topk_e4m3.argtypes = [P, P, ctypes.c_int64, ctypes.c_int32, P, ctypes.c_int32,
+                                         ctypes.c_int32, P, P, ctypes.c_int32]
+        lib.oracle_topk_e4m3.restype = ctypes.c_int
         self.lib = lib
         self.path = path
 
@@ -176,6 +190,54 @@ class OracleLib:
                 np.array([r[2] for r in res], np.int32), u)
 
 
+    def e4m3_to_double(self, code: int) -> float:
+        """Exact value of one e4m3 code (NaN for 0x7f / 0xff)."""
+        return float(self.lib.oracle_e4m3_to_double(int(code) & 0xFF))
+
+    def f32_to_e4m3(self, x: float) -> int:
+        """Nearest e4m3 code of an fp32 value (ties to even, saturated at 448)."""
+        return int(self.lib.oracle_f32_to_e4m3(float(np.float32(x))))
+
+    def quantize_e4m3(self, W_bits: np.ndarray):
+        """Per-row e4m3 quantisation of bf16 rows: (codes uint8 [V, d], scales fp32 [V])."""
+        W_bits = np.ascontiguousarray(W_bits, dtype=np.uint16)
+        V, d = W_bits.shape
+        q = np.empty((V, d), dtype=np.uint8)
+        sc = np.empty(V, dtype=np.float32)
+        rc = self.lib.oracle_quantize_e4m3(_ptr(W_bits), V, d, _ptr(q), _ptr(sc))
+        if rc != 0:
+            raise ValueError(f"oracle_quantize_e4m3 failed with code {rc}")
+        return q, sc
+
+    def logits_e4m3(self, q: np.ndarray, scale: np.ndarray, h: np.ndarray, threads: int = 0):
+        """fp64 logits [batch, V] of the quantised head."""
+        q = np.ascontiguousarray(q, dtype=np.uint8)
+        scale = np.ascontiguousarray(scale, dtype=np.float32)
+        V, d = q.shape
+        h = np.ascontiguousarray(np.asarray(h, dtype=np.float32).reshape(-1, d))
+        out = np.empty((h.shape[0], V), dtype=np.float64)
+        rc = self.lib.oracle_logits_e4m3(_ptr(q), _ptr(scale), V, d, _ptr(h), h.shape[0], _ptr(out),
+                                         threads or self.max_threads())
+        if rc != 0:
+            raise ValueError(f"oracle_logits_e4m3 failed with code {rc}")
+        return out
+
+    def topk_e4m3(self, q: np.ndarray, scale: np.ndarray, h: np.ndarray, k: int, threads: int = 0):
+        """Exact top-k of the quantised head: (idx int32 [batch,k], logits fp64 [batch,k])."""
+        q = np.ascontiguousarray(q, dtype=np.uint8)
+        scale = np.ascontiguousarray(scale, dtype=np.float32)
+        V, d = q.shape
+        h = np.ascontiguousarray(np.asarray(h, dtype=np.float32).reshape(-1, d))
+        b = h.shape[0]
+        idx = np.empty((b, k), dtype=np.int32)
+        val = np.empty((b, k), dtype=np.float64)
+        rc = self.lib.oracle_topk_e4m3(_ptr(q), _ptr(scale), V, d, _ptr(h), b, k, _ptr(idx), _ptr(val),
+                                       threads or self.max_threads())
+        if rc != 0:
+            raise ValueError(f"oracle_topk_e4m3 failed with code {rc}")
+        return idx, val
+
+
 def _default() -> OracleLib:
     global _lib
     with _lock:
@@ -218,3 +280,16 @@ def sample_sorted(z, T: float, top_p: float, min_p: float, u: float):
 
 def sample(z, T: float, top_p: float, min_p: float, seed: int, step: int):
     return _default().sample(z, T, top_p, min_p, seed, step)
+
+
+def quantize_e4m3(W_bits):
+    return _default().quantize_e4m3(W_bits)
+
+
+def logits_e4m3(q, scale, h, threads: int = 0):
+    return _default().logits_e4m3(q, scale, h, threads)
+
+
+def topk_e4m3(q, scale, h, k: int, threads: int = 0):
+    return _default().topk_e4m3(q, scale, h, k, threads)
+

@@ -41,6 +41,16 @@
  *     Dror, Shaw, "Parallel random numbers: as easy as 1, 2, 3", SC 2011):
  *     counter (step low, step high, query, 0), key (seed low, seed high), the
  *     top 24 bits of the first output word times 2^-24.
+ *
+ * Quantised output embedding (Section 4 names weight quantisation as a
+ * bandwidth-saving technique orthogonal to the method).  Readings: each row
+ * of W_out is stored as 8-bit floats of the e4m3 format (1 sign bit, 4
+ * exponent bits with bias 7, 3 mantissa bits, subnormals, no infinities,
+ * largest finite value 448) times one fp32 scale per row,
+ *   scale_i = max_j |w_ij| / 448 in fp32 (1 for an all-zero row),
+ *   q_ij = e4m3(w_ij / scale_i), the fp32 quotient rounded to the nearest
+ *          e4m3 value, ties to even, magnitudes past 448 saturated;
+ * and the head computes z_i = scale_i * sum_j e4m3(q_ij) * h_j.
  */
 #include <math.h>
 #include <stdint.h>
@@ -262,5 +272,110 @@ int oracle_sample_sorted(const double *z, int32_t k, double T, double top_p, dou
     *kept_out = n;
     free(p);
     return ORACLE_OK;
+}
+
+/* ------------------------------------------------------------------------ */
+/* e4m3 code -> value, exactly.  Code 0x7f / 0xff is NaN. */
+double oracle_e4m3_to_double(uint8_t c) {
+    const int sgn = (c >> 7) & 1, E = (c >> 3) & 15, M = c & 7;
+    double v;
+    if (E == 15 && M == 7) return NAN;
+    if (E == 0)
+        v = ldexp((double)M, -9);              /* subnormal: M * 2^-9 */
+    else
+        v = ldexp(1.0 + M / 8.0, E - 7);       /* normal: (1 + M/8) * 2^(E-7) */
+    return sgn ? -v : v;
+}
+
+/* fp32 value -> nearest e4m3 code, ties to even, magnitudes past 448 to 448. */
+uint8_t oracle_f32_to_e4m3(float x) {
+    const int sgn = signbit(x) ? 1 : 0;
+    const double a = fabs((double)x);
+    if (a >= 448.0) return (uint8_t)((sgn << 7) | (15 << 3) | 6);
+    if (a < ldexp(1.0, -6)) {
+        /* subnormal range: a multiple of 2^-9 (8 * 2^-9 is the least normal) */
+        const double m = rint(ldexp(a, 9));    /* rint: to nearest, ties to even */
+        return (uint8_t)((sgn << 7) | (int)m);  /* m = 8 gives exponent field 1 */
+    }
+    int e;
+    frexp(a, &e);                              /* a = f * 2^e, f in [0.5, 1) */
+    e -= 1;                                    /* a = (1 + t) * 2^e, t in [0, 1) */
+    double m = rint((ldexp(a, -e) - 1.0) * 8.0);
+    if (m == 8.0) {
+        m = 0.0;
+        e += 1;
+    }
+    if (e > 8 || (e == 8 && m > 6.0)) return (uint8_t)((sgn << 7) | (15 << 3) | 6);
+    return (uint8_t)((sgn << 7) | ((e + 7) << 3) | (int)m);
+}
+
+/* Quantise bf16 rows W [V, d] to e4m3 codes q [V, d] and fp32 scales [V]. */
+int oracle_quantize_e4m3(const uint16_t *W, int64_t V, int32_t d, uint8_t *q, float *scale) {
+    if (!W || !q || !scale || V < 1 || d < 1) return ORACLE_EINVAL;
+    for (int64_t i = 0; i < V; ++i) {
+        const uint16_t *wi = W + i * (int64_t)d;
+        float amax = 0.0f;
+        for (int32_t j = 0; j < d; ++j) {
+            const float a = fabsf((float)oracle_bf16_to_double(wi[j]));
+            if (a > amax) amax = a;
+        }
+        const float s = amax > 0.0f ? amax / 448.0f : 1.0f;
+        scale[i] = s;
+        for (int32_t j = 0; j < d; ++j)
+            q[i * (int64_t)d + j] = oracle_f32_to_e4m3((float)oracle_bf16_to_double(wi[j]) / s);
+    }
+    return ORACLE_OK;
+}
+
+/* z[b*V + i] = scale_i * sum_j e4m3(q_ij) * h[b, j] in fp64. */
+int oracle_logits_e4m3(const uint8_t *q, const float *scale, int64_t V, int32_t d,
+                       const float *h, int32_t batch, double *z, int32_t nthreads) {
+    if (!q || !scale || !h || !z || V < 1 || d < 1 || batch < 1) return ORACLE_EINVAL;
+    if (nthreads < 1) nthreads = 1;
+    for (int32_t b = 0; b < batch; ++b) {
+        const float *hb = h + (int64_t)b * d;
+        double *zb = z + (int64_t)b * V;
+#pragma omp parallel for num_threads(nthreads) schedule(static)
+        for (int64_t i = 0; i < V; ++i) {
+            const uint8_t *qi = q + i * (int64_t)d;
+            double acc = 0.0;
+            for (int32_t j = 0; j < d; ++j) acc += oracle_e4m3_to_double(qi[j]) * (double)hb[j];
+            zb[i] = (double)scale[i] * acc;
+        }
+    }
+    return ORACLE_OK;
+}
+
+/* Exhaustive MIPS over the quantised rows: the same full sort as oracle_topk
+ * on z_i = scale_i * sum_j e4m3(q_ij) * h_j. */
+int oracle_topk_e4m3(const uint8_t *q, const float *scale, int64_t V, int32_t d, const float *h,
+                     int32_t batch, int32_t k, int32_t *idx, double *logits, int32_t nthreads) {
+    if (!q || !scale || !h || !idx || !logits || V < 1 || d < 1 || batch < 1 || k < 1 ||
+        (int64_t)k > V)
+        return ORACLE_EINVAL;
+    double *z = (double *)malloc(sizeof(double) * (size_t)V);
+    scored_row *rows = (scored_row *)malloc(sizeof(scored_row) * (size_t)V);
+    if (!z || !rows) {
+        free(z);
+        free(rows);
+        return ORACLE_ENOMEM;
+    }
+    int rc = ORACLE_OK;
+    for (int32_t b = 0; b < batch && rc == ORACLE_OK; ++b) {
+        rc = oracle_logits_e4m3(q, scale, V, d, h + (int64_t)b * d, 1, z, nthreads);
+        if (rc != ORACLE_OK) break;
+        for (int64_t i = 0; i < V; ++i) {
+            rows[i].z = z[i];
+            rows[i].i = i;
+        }
+        qsort(rows, (size_t)V, sizeof(scored_row), by_logit_desc_index_asc);
+        for (int32_t j = 0; j < k; ++j) {
+            idx[(int64_t)b * k + j] = (int32_t)rows[j].i;
+            logits[(int64_t)b * k + j] = rows[j].z;
+        }
+    }
+    free(z);
+    free(rows);
+    return rc;
 }
 

@@ -12,6 +12,7 @@ import pytest
 import oracle as default_oracle
 from test_oracle_pins import PINS
 from test_oracle_sampling import SAMPLING_PINS
+from test_oracle_fp8 import FP8_PINS
 
 SRC = os.path.join(os.path.dirname(default_oracle.__file__), "oracle.c")
 
@@ -41,6 +42,13 @@ MUTANTS = {
     "min_p_absolute": ("if (p[j] >= min_p * p[0]) ++n_m;", "if (p[j] >= min_p) ++n_m;"),
     "draw_at_or_above": ("if (cum > target) {", "if (cum >= target) {"),
     "prob_not_renormalised": ("*prob_out = p[js] / M;", "*prob_out = p[js];"),
+    # the quantised head
+    "e4m3_truncated": ("double m = rint((ldexp(a, -e) - 1.0) * 8.0);", "double m = floor((ldexp(a, -e) - 1.0) * 8.0);"),
+    "e4m3_bias_off": ("return (uint8_t)((sgn << 7) | ((e + 7) << 3) | (int)m);", "return (uint8_t)((sgn << 7) | ((e + 8) << 3) | (int)m);"),
+    "e4m3_subnormal_step": ("const double m = rint(ldexp(a, 9));", "const double m = rint(ldexp(a, 8));"),
+    "e4m3_decode_bias": ("v = ldexp(1.0 + M / 8.0, E - 7);", "v = ldexp(1.0 + M / 8.0, E - 8);"),
+    "scale_wrong_range": ("const float s = amax > 0.0f ? amax / 448.0f : 1.0f;", "const float s = amax > 0.0f ? amax / 240.0f : 1.0f;"),
+    "logits_scale_dropped": ("zb[i] = (double)scale[i] * acc;", "zb[i] = acc;"),
 }
 
 
@@ -53,7 +61,7 @@ def test_pins_catch_planted_mistake(name, tmp_path):
     src.write_text(text.replace(old, new, 1))
     lib = default_oracle.OracleLib(default_oracle.build(True, str(src), str(tmp_path / f"{name}.so")))
     caught = []
-    for pin_name, pin in PINS + SAMPLING_PINS:
+    for pin_name, pin in PINS + SAMPLING_PINS + FP8_PINS:
         try:
             pin(lib)
         except (AssertionError, ValueError):
