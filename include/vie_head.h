@@ -89,6 +89,35 @@ typedef struct {
 vie_status vie_head_create(const void *W_out, int64_t V, int32_t d, vie_dtype dtype,
                            vie_head **out);
 
+/*
+ * vie_head_create_e4m3 - a head whose rows are stored as 8-bit floats: the
+ * paper names weight quantisation as a bandwidth saving orthogonal to its
+ * method (Section 4); this is that variant of the exact head, streaming half
+ * the bytes of the bf16 head per decode step.
+ *
+ *   W_out   device, bf16, row-major [V, d], 2-byte aligned (as for
+ *           vie_head_create); quantised on the device before the call returns.
+ *   V, d    as for vie_head_create.
+ *
+ * Row i is stored as e4m3 codes (1 sign, 4 exponent bits with bias 7, 3
+ * mantissa bits, largest finite value 448) and one fp32 scale:
+ *   scale_i = max_j |w_ij| / 448 in fp32 (1 for an all-zero row);
+ *   q_ij = w_ij / scale_i in fp32, rounded to the nearest e4m3 value (ties
+ *          to even, saturated at +-448);
+ * and every top-k call on the handle (vie_head_topk, _sparse, _host,
+ * _sample) computes z_i = scale_i * sum_j e4m3(q_ij) * h_j with fp32
+ * accumulation, then the same exact top-k.  Such a handle always uses the
+ * streaming CUDA-core kernel (vie_head_plan reports path 0).  Same errors as
+ * vie_head_create.
+ */
+vie_status vie_head_create_e4m3(const void *W_out, int64_t V, int32_t d, vie_head **out);
+
+/* Copies an e4m3 handle's codes (device uint8 [V, d], row-major) and scales
+ * (device fp32 [V]) to caller buffers, asynchronously on `stream`.
+ * VIE_ERR_INVALID_ARG for a bf16 handle or NULL arguments. */
+vie_status vie_head_export_e4m3(const vie_head *head, uint8_t *codes, float *scales,
+                                vie_stream stream);
+
 /* Frees the padded copy and the scratch.  NULL is accepted.  The caller must
  * make sure no work using the handle is still running (synchronise first). */
 vie_status vie_head_destroy(vie_head *head);

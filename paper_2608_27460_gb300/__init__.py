@@ -37,6 +37,7 @@ STATUS_NAMES = {0: "VIE_OK", 1: "VIE_ERR_INVALID_ARG", 2: "VIE_ERR_UNSUPPORTED",
 # Every entry point of include/vie_head.h.
 EXPORTS = ("vie_head_create", "vie_head_destroy", "vie_head_get_props", "vie_head_plan", "vie_head_topk",
            "vie_head_topk_sparse", "vie_head_topk_host", "vie_sample_topk", "vie_head_topk_sample",
+           "vie_head_create_e4m3", "vie_head_export_e4m3",
            "vie_head_topk_noalloc", "vie_scatter_sparse_logits", "vie_device_status",
            "vie_head_device_status", "vie_last_error")
 
@@ -83,6 +84,8 @@ def load(path: str | None = None, build_if_missing: bool = True):
         sig = {
             "vie_head_create": ([P, I64, I32, ctypes.c_int, ctypes.POINTER(P)], ctypes.c_int),
             "vie_head_destroy": ([P], ctypes.c_int),
+            "vie_head_create_e4m3": ([P, I64, I32, ctypes.POINTER(P)], ctypes.c_int),
+            "vie_head_export_e4m3": ([P, P, P, P], ctypes.c_int),
             "vie_head_get_props": ([P, ctypes.POINTER(vie_head_props)], ctypes.c_int),
             "vie_head_plan": ([P, I32, I32, ctypes.POINTER(vie_topk_plan)], ctypes.c_int),
             "vie_head_topk": ([P, P, I32, I32, P, P, P], ctypes.c_int),
@@ -117,6 +120,17 @@ def vie_head_create(W_out: int, V: int, d: int, dtype: int = VIE_DTYPE_BF16):
     out = ctypes.c_void_p(0)
     st = load().vie_head_create(W_out, V, d, dtype, ctypes.byref(out))
     return st, out.value
+
+
+def vie_head_create_e4m3(W_out: int, V: int, d: int):
+    """Returns (status, handle) of a head stored as e4m3 rows with fp32 scales."""
+    out = ctypes.c_void_p(0)
+    st = load().vie_head_create_e4m3(W_out, V, d, ctypes.byref(out))
+    return st, out.value
+
+
+def vie_head_export_e4m3(head: int, codes: int, scales: int, stream: int = 0) -> int:
+    return load().vie_head_export_e4m3(head, codes, scales, stream)
 
 
 def vie_head_destroy(head: int) -> int:
@@ -224,7 +238,9 @@ class Head:
     bf16 bit patterns).  The head keeps its own padded copy, so ``W`` may be
     freed afterwards."""
 
-    def __init__(self, W):
+    def __init__(self, W, storage: str = "bf16"):
+        """W: bf16 weights [V, d] on a CUDA device.  storage "bf16" keeps them
+        as they are; "e4m3" quantises each row to e4m3 with an fp32 scale."""
         import torch
         if not W.is_cuda or W.dim() != 2:
             raise ValueError("W must be a 2-D CUDA tensor")
@@ -233,8 +249,14 @@ class Head:
         W = W.contiguous()
         self.V, self.d = int(W.shape[0]), int(W.shape[1])
         self.device = W.device
+        if storage not in ("bf16", "e4m3"):
+            raise ValueError(f"storage must be 'bf16' or 'e4m3', not {storage!r}")
+        self.storage = storage
         with torch.cuda.device(W.device):
-            st, hd = vie_head_create(W.data_ptr(), self.V, self.d, VIE_DTYPE_BF16)
+            if storage == "e4m3":
+                st, hd = vie_head_create_e4m3(W.data_ptr(), self.V, self.d)
+            else:
+                st, hd = vie_head_create(W.data_ptr(), self.V, self.d, VIE_DTYPE_BF16)
         check(st)
         self._h = hd
         st, self.props = vie_head_get_props(hd)
@@ -326,6 +348,14 @@ class Head:
                                    step, idx.data_ptr(), val.data_ptr(), sp, tok.data_ptr(),
                                    prob.data_ptr(), _stream_ptr(stream)))
         return idx, val, tok, prob
+
+    def export_e4m3(self, stream=None):
+        """The e4m3 codes (uint8 [V, d]) and row scales (float32 [V]) of an e4m3 head."""
+        import torch
+        codes = torch.empty((self.V, self.d), dtype=torch.uint8, device=self.device)
+        scales = torch.empty((self.V,), dtype=torch.float32, device=self.device)
+        check(vie_head_export_e4m3(self.handle, codes.data_ptr(), scales.data_ptr(), _stream_ptr(stream)))
+        return codes, scales
 
     def sparse_logits(self, idx, logits, out=None, stream=None):
         """Sparse [batch, V] fp32 tensor: -inf except logits at idx."""

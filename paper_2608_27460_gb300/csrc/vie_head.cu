@@ -1,6 +1,7 @@
 // vie_head.cu - the C ABI declared in include/vie_head.h: argument checks,
 // handle life cycle, launch configuration, weight-layout preparation and
 // the sparse-logit scatter kernel.
+#include <cuda_fp8.h>
 #include <cuda_runtime.h>
 
 #include <climits>
@@ -54,7 +55,8 @@ struct vie_head {
     int32_t d, d_pad;
     int num_sms;
     int G;
-    uint16_t *W;        // [V, d_pad] bf16 bits
+    uint16_t *W;        // [V, d_pad] bf16 bits, or e4m3 codes (bytes) when scale is set
+    float *scale;       // e4m3 heads: fp32 scale per row [V]; nullptr for bf16 heads
     uint64_t *cand;     // [kMaxNB][G][VIE_K_MAX] ranking keys, then [kMaxNB][G][kFastE] heads
     uint32_t *words;    // [0] completion ticket, [1] device flag word, [2] chunk pool counter,
                         // [3] merging CTAs done (tensor-core path)
@@ -70,6 +72,33 @@ struct vie_head {
     float *stage_logits;
     size_t stage_h_elems, stage_out_elems;
 };
+
+// ---------------------------------------------------------------------------
+// Row quantisation to e4m3: one warp per row of bf16 W [V, d] (any 2-byte
+// alignment).  scale = max |w| / 448 in fp32 (1 for a zero row); each code is
+// w / scale rounded to the nearest e4m3 value (ties to even, saturated), the
+// row padded to d_pad (a multiple of 16) with zero codes.
+__global__ void quantize_e4m3_kernel(const uint16_t *__restrict__ src, int64_t V, int d, int d_pad,
+                                     uint8_t *__restrict__ q, float *__restrict__ scale) {
+    const int lane = threadIdx.x & 31;
+    const int64_t warps = static_cast<int64_t>(gridDim.x) * (blockDim.x >> 5);
+    for (int64_t row = blockIdx.x * static_cast<int64_t>(blockDim.x >> 5) + (threadIdx.x >> 5);
+         row < V; row += warps) {
+        const uint16_t *wr = src + row * d;
+        float amax = 0.0f;
+        for (int j = lane; j < d; j += 32)
+            amax = fmaxf(amax, fabsf(__uint_as_float(static_cast<uint32_t>(wr[j]) << 16)));
+#pragma unroll
+        for (int o = 16; o >= 1; o >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xFFFFFFFFu, amax, o));
+        const float sc = amax > 0.0f ? amax / 448.0f : 1.0f;
+        uint8_t *qr = q + row * d_pad;
+        for (int j = lane; j < d_pad; j += 32) {
+            const float x = j < d ? __uint_as_float(static_cast<uint32_t>(wr[j]) << 16) / sc : 0.0f;
+            qr[j] = static_cast<uint8_t>(__nv_cvt_float_to_fp8(x, __NV_SATFINITE, __NV_E4M3));
+        }
+        if (lane == 0) scale[row] = sc;
+    }
+}
 
 // ---------------------------------------------------------------------------
 // Weight-layout preparation: [V, d] (any 2-byte alignment) -> [V, d_pad]
@@ -184,8 +213,7 @@ struct LaunchShape {
 
 // Rows per warp per stage (R), stage rows (8*R, fewer for very wide rows),
 // and ring depth (deepest that fits) for one launch.
-bool pick_shape(int nb, int d_pad, LaunchShape *out) {
-    const int row_bytes = d_pad * 2;
+bool pick_shape(int nb, int d_pad, int row_bytes, LaunchShape *out) {
     const int r_max = nb == 1 ? 8 : 4;  // 8 rows per warp only for single-query launches
     int r = 1;
     while (r < r_max && 8 * r * row_bytes < knobs().stage_min_bytes) r <<= 1;
@@ -253,8 +281,8 @@ extern "C" {
 
 const char *vie_last_error(void) { return g_err; }
 
-vie_status vie_head_create(const void *W_out, int64_t V, int32_t d, vie_dtype dtype,
-                           vie_head **out) {
+static vie_status create_head(const void *W_out, int64_t V, int32_t d, vie_dtype dtype, bool e4m3,
+                              vie_head **out) {
     if (out == nullptr) return fail(VIE_ERR_INVALID_ARG, "vie_head_create: out is NULL");
     *out = nullptr;
     if (W_out == nullptr) return fail(VIE_ERR_INVALID_ARG, "vie_head_create: W_out is NULL");
@@ -291,18 +319,19 @@ vie_status vie_head_create(const void *W_out, int64_t V, int32_t d, vie_dtype dt
     hd->device = dev;
     hd->V = V;
     hd->d = d;
-    hd->d_pad = (d + 7) & ~7;
+    hd->d_pad = e4m3 ? (d + 15) & ~15 : (d + 7) & ~7;  // 16-byte rows either way
     hd->num_sms = sms;
     int64_t g = (V + 63) / 64;
     if (g > sms) g = sms;
     if (g > vie::kMaxLists) g = vie::kMaxLists;
     hd->G = static_cast<int>(g < 1 ? 1 : g);
 
-    const size_t wbytes = static_cast<size_t>(V) * hd->d_pad * 2;
+    const size_t wbytes = static_cast<size_t>(V) * hd->d_pad * (e4m3 ? 1 : 2);
     const size_t cbytes =
         static_cast<size_t>(kMaxNB) * hd->G * (VIE_K_MAX + vie::kFastE) * sizeof(uint64_t);
     hd->scratch_bytes = static_cast<int64_t>(cbytes + 4 * sizeof(uint32_t));
     e = cudaMalloc(&hd->W, wbytes);
+    if (e == cudaSuccess && e4m3) e = cudaMalloc(&hd->scale, static_cast<size_t>(V) * sizeof(float));
     if (e == cudaSuccess) e = cudaMalloc(&hd->cand, cbytes);
     if (e == cudaSuccess) e = cudaMemset(hd->cand, 0, cbytes);  // empty lists until written
     if (e == cudaSuccess) e = cudaMalloc(&hd->words, 4 * sizeof(uint32_t));
@@ -310,7 +339,14 @@ vie_status vie_head_create(const void *W_out, int64_t V, int32_t d, vie_dtype dt
         e = cudaMalloc(&hd->hB, static_cast<size_t>(vie::kTcHRows) * hd->d_pad * 2);
     if (e == cudaSuccess) e = cudaMemset(hd->hB, 0, static_cast<size_t>(vie::kTcHRows) * hd->d_pad * 2);
     if (e == cudaSuccess) e = cudaMemset(hd->words, 0, 4 * sizeof(uint32_t));
-    if (e == cudaSuccess) {
+    if (e == cudaSuccess && e4m3) {
+        int64_t blocks = (V + 7) / 8;  // 8 rows (warps) per block
+        if (blocks > 64LL * sms) blocks = 64LL * sms;
+        quantize_e4m3_kernel<<<static_cast<unsigned>(blocks), 256>>>(
+            static_cast<const uint16_t *>(W_out), V, d, hd->d_pad, reinterpret_cast<uint8_t *>(hd->W),
+            hd->scale);
+        e = cudaGetLastError();
+    } else if (e == cudaSuccess) {
         const int64_t chunks = V * (hd->d_pad >> 3);
         int64_t blocks = (chunks + 255) / 256;
         if (blocks > 32LL * sms) blocks = 32LL * sms;
@@ -322,11 +358,17 @@ vie_status vie_head_create(const void *W_out, int64_t V, int32_t d, vie_dtype dt
     if (e != cudaSuccess) {
         const vie_status st = fail_cuda(e, "vie_head_create");
         cudaFree(hd->W);
+        cudaFree(hd->scale);
         cudaFree(hd->cand);
         cudaFree(hd->words);
         cudaFree(hd->hB);
         delete hd;
         return st;
+    }
+    if (e4m3) {  // e4m3 heads stream through the CUDA-core kernel at every batch size
+        hd->tc_ready = false;
+        *out = hd;
+        return VIE_OK;
     }
     const uint64_t pitch = static_cast<uint64_t>(hd->d_pad) * 2;
     hd->tc_ready = make_map_bf16(&hd->mapW, hd->W, static_cast<uint64_t>(V), hd->d_pad, pitch,
@@ -337,9 +379,38 @@ vie_status vie_head_create(const void *W_out, int64_t V, int32_t d, vie_dtype dt
     return VIE_OK;
 }
 
+vie_status vie_head_create(const void *W_out, int64_t V, int32_t d, vie_dtype dtype,
+                           vie_head **out) {
+    return create_head(W_out, V, d, dtype, false, out);
+}
+
+vie_status vie_head_create_e4m3(const void *W_out, int64_t V, int32_t d, vie_head **out) {
+    return create_head(W_out, V, d, VIE_DTYPE_BF16, true, out);
+}
+
+vie_status vie_head_export_e4m3(const vie_head *head, uint8_t *codes, float *scales,
+                                vie_stream stream) {
+    const char *fn = "vie_head_export_e4m3";
+    if (head == nullptr || codes == nullptr || scales == nullptr)
+        return fail(VIE_ERR_INVALID_ARG, "%s: NULL argument", fn);
+    if (head->scale == nullptr) return fail(VIE_ERR_INVALID_ARG, "%s: not an e4m3 head", fn);
+    vie_status st = check_device(head);
+    if (st != VIE_OK) return st;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    cudaError_t e = cudaMemcpy2DAsync(codes, static_cast<size_t>(head->d), head->W,
+                                      static_cast<size_t>(head->d_pad), static_cast<size_t>(head->d),
+                                      static_cast<size_t>(head->V), cudaMemcpyDeviceToDevice, s);
+    if (e == cudaSuccess)
+        e = cudaMemcpyAsync(scales, head->scale, static_cast<size_t>(head->V) * sizeof(float),
+                            cudaMemcpyDeviceToDevice, s);
+    if (e != cudaSuccess) return fail_cuda(e, fn);
+    return VIE_OK;
+}
+
 vie_status vie_head_destroy(vie_head *head) {
     if (head == nullptr) return VIE_OK;
     cudaFree(head->W);
+    cudaFree(head->scale);
     cudaFree(head->cand);
     cudaFree(head->words);
     cudaFree(head->hB);
@@ -358,7 +429,8 @@ vie_status vie_head_get_props(const vie_head *head, vie_head_props *props) {
     props->d_pad = head->d_pad;
     props->ctas = head->G;
     props->device = head->device;
-    props->weight_bytes = head->V * head->d_pad * 2;
+    props->weight_bytes = head->scale != nullptr ? head->V * head->d_pad + head->V * 4
+                                                 : head->V * head->d_pad * 2;
     props->scratch_bytes = head->scratch_bytes;
     return VIE_OK;
 }
@@ -465,10 +537,11 @@ static vie_status run_topk(const char *fn, vie_head *head, const float *h, int32
         int nb = 1;
         while (nb < nq) nb <<= 1;
         LaunchShape shp;
-        if (!pick_shape(nb, head->d_pad, &shp))
+        if (!pick_shape(nb, head->d_pad, head->d_pad * (head->scale != nullptr ? 1 : 2), &shp))
             return fail(VIE_ERR_UNSUPPORTED, "%s: no shared-memory layout for d=%d", fn, head->d);
         vie::StreamTopkParams p;
         p.W = head->W;
+        p.row_scale = head->scale;
         p.h = h + static_cast<int64_t>(q0) * head->d;
         p.nq = nq;
         p.V = head->V;
@@ -777,10 +850,11 @@ extern "C" vie_status vie_head_topk_noalloc(const void *W_out, int64_t V, int32_
         int nb = 1;
         while (nb < nq) nb <<= 1;
         LaunchShape shp;
-        if (!pick_shape(nb, d, &shp))
+        if (!pick_shape(nb, d, d * 2, &shp))
             return fail(VIE_ERR_UNSUPPORTED, "%s: no shared-memory layout for d=%d", fn, d);
         vie::StreamTopkParams p;
         p.W = static_cast<const uint16_t *>(W_out);
+        p.row_scale = nullptr;
         p.h = h + static_cast<int64_t>(q0) * d;
         p.nq = nq;
         p.V = V;
@@ -811,6 +885,15 @@ extern "C" vie_status vie_head_topk_noalloc(const void *W_out, int64_t V, int32_
 namespace vie {
 cudaError_t launch_stream_topk(int nb, int mm, int r, const StreamTopkParams &p, int grid,
                                uint32_t smem, cudaStream_t stream) {
+    if (p.row_scale != nullptr) {
+        switch (nb) {
+            case 1: return launch_stream_topk_e4m3_nb1(mm, r, p, grid, smem, stream);
+            case 2: return launch_stream_topk_e4m3_nb2(mm, r, p, grid, smem, stream);
+            case 4: return launch_stream_topk_e4m3_nb4(mm, r, p, grid, smem, stream);
+            case 8: return launch_stream_topk_e4m3_nb8(mm, r, p, grid, smem, stream);
+            default: return cudaErrorInvalidValue;
+        }
+    }
     switch (nb) {
         case 1: return launch_stream_topk_nb1(mm, r, p, grid, smem, stream);
         case 2: return launch_stream_topk_nb2(mm, r, p, grid, smem, stream);

@@ -23,6 +23,16 @@ cudaError_t launch_stream_topk_nb4(int mm, int r, const StreamTopkParams &p, int
                                    uint32_t smem, cudaStream_t stream);
 cudaError_t launch_stream_topk_nb8(int mm, int r, const StreamTopkParams &p, int grid,
                                    uint32_t smem, cudaStream_t stream);
+// The same on rows of e4m3 codes with per-row scales (p.row_scale).
+cudaError_t launch_stream_topk_e4m3_nb1(int mm, int r, const StreamTopkParams &p, int grid,
+                                        uint32_t smem, cudaStream_t stream);
+cudaError_t launch_stream_topk_e4m3_nb2(int mm, int r, const StreamTopkParams &p, int grid,
+                                        uint32_t smem, cudaStream_t stream);
+cudaError_t launch_stream_topk_e4m3_nb4(int mm, int r, const StreamTopkParams &p, int grid,
+                                        uint32_t smem, cudaStream_t stream);
+cudaError_t launch_stream_topk_e4m3_nb8(int mm, int r, const StreamTopkParams &p, int grid,
+                                        uint32_t smem, cudaStream_t stream);
+
 
 // ---- tensor-core head (vie_tc_topk.cu) ----
 struct TcParams;

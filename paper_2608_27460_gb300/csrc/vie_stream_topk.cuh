@@ -36,6 +36,9 @@
 // so each fill happens before the value at the same position.
 #pragma once
 
+#include <cuda_fp16.h>
+#include <cuda_fp8.h>
+
 #include <cstdint>
 
 #include "vie_device.cuh"
@@ -54,7 +57,8 @@ constexpr int kFastE = 4;              // fast merge: entries read per list (eve
 constexpr int kFastMaxK = 64;          // fast merge: largest k
 
 struct StreamTopkParams {
-    const uint16_t *W;   // padded [V, d_pad] bf16 bits
+    const uint16_t *W;   // padded [V, d_pad] bf16 bits, or [V, d_pad] e4m3 codes (bytes)
+    const float *row_scale;  // e4m3 rows: fp32 scale per row [V]; nullptr for bf16 rows
     const float *h;      // [nq, d] fp32
     int32_t nq;          // queries in this launch (<= NB)
     int64_t V;
@@ -586,12 +590,29 @@ __device__ __forceinline__ int stage_rows(int64_t row0, int64_t pool_row0, int R
     return static_cast<int>(min(len, V - row0));
 }
 
-template <int NB, int MM, int R>
+// e4m3 x4 (one 32-bit word, element 0 in the low byte) times h.x..h.w into a,
+// in element order; each e4m3 value is exact in fp16 and fp32.
+__device__ __forceinline__ float fma_e4m3x4(uint32_t w, float4 h, float a) {
+    const float2 lo = __half22float2(__half2(__nv_cvt_fp8x2_to_halfraw2(
+        static_cast<__nv_fp8x2_storage_t>(w & 0xFFFFu), __NV_E4M3)));
+    const float2 hi = __half22float2(__half2(__nv_cvt_fp8x2_to_halfraw2(
+        static_cast<__nv_fp8x2_storage_t>(w >> 16), __NV_E4M3)));
+    a = fmaf(lo.x, h.x, a);
+    a = fmaf(lo.y, h.y, a);
+    a = fmaf(hi.x, h.z, a);
+    a = fmaf(hi.y, h.w, a);
+    return a;
+}
+
+// Q8: rows of e4m3 codes (16 per 16-byte chunk) with one fp32 scale per row,
+// logit = scale * sum; otherwise bf16 rows (8 per chunk).
+template <int NB, int MM, int R, bool Q8>
 __global__ void __launch_bounds__(kThreads, 1) stream_topk_kernel(const StreamTopkParams p) {
     extern __shared__ __align__(128) unsigned char smem[];
     const int RS = p.rows_per_stage;  // <= 8 * R
     const int S = p.stages;
-    const int row_bytes = p.d_pad * 2;
+    const int row_bytes = Q8 ? p.d_pad : p.d_pad * 2;
+    constexpr int kEPC = Q8 ? 16 : 8;  // weights per 16-byte chunk
     const SmemLayout L(NB, p.d_pad, RS, S, row_bytes);
     uint64_t *full = reinterpret_cast<uint64_t *>(smem + L.bars);
     uint64_t *empty = full + kMaxStages;
@@ -610,7 +631,7 @@ __global__ void __launch_bounds__(kThreads, 1) stream_topk_kernel(const StreamTo
     const int cta = blockIdx.x;
     const int RSH = p.pool_rows;  // rows of a pool piece
     const int64_t pool_row0 = static_cast<int64_t>(G) * p.static_chunks * RS;
-    const int C = p.d_pad >> 3;  // 16-byte chunks per row
+    const int C = p.d_pad / kEPC;  // 16-byte chunks per row
     const int stage_bytes = RS * row_bytes;
 
     if (tid == 0) {
@@ -627,9 +648,9 @@ __global__ void __launch_bounds__(kThreads, 1) stream_topk_kernel(const StreamTo
         fence_mbar_init();
         griddep_launch_dependents();  // a kernel launched after this one may be scheduled now
     }
-    // h -> shared memory as [nb][half][chunk][4] so a lane's two float4 loads
-    // of one chunk fall in distinct bank groups; zero pad, zero unused
-    // queries.  Asynchronous copies by warps 1.. issued before the producer
+    // h -> shared memory as [nb][part][chunk][4] (2 parts of 4 for bf16 rows,
+    // 4 for e4m3 rows) so a lane's float4 loads of one chunk fall in distinct
+    // bank groups; zero pad, zero unused queries.  Asynchronous copies by warps 1.. issued before the producer
     // starts, so h is ahead of the weight stream in the memory queues; those
     // warps wait for them after the barrier (bar.sync 1 below).
     if (warp > 0) {
@@ -637,8 +658,8 @@ __global__ void __launch_bounds__(kThreads, 1) stream_topk_kernel(const StreamTo
             const int nb = i / p.d_pad, j = i - nb * p.d_pad;
             const bool real = nb < p.nq && j < p.d;
             const float *src = real ? p.h + static_cast<int64_t>(nb) * p.d + j : p.h;
-            const int c = j >> 3, e = j & 7;
-            cp_async_4_zfill(h_s + (nb * 2 + (e >> 2)) * (C * 4) + c * 4 + (e & 3), src, real);
+            const int c = j / kEPC, e = j - c * kEPC;
+            cp_async_4_zfill(h_s + (nb * (kEPC / 4) + (e >> 2)) * (C * 4) + c * 4 + (e & 3), src, real);
         }
         cp_async_commit();
     }
@@ -786,6 +807,9 @@ __global__ void __launch_bounds__(kThreads, 1) stream_topk_kernel(const StreamTo
                 for (int i = 0; i < R; ++i)
 #pragma unroll
                     for (int nb = 0; nb < NB; ++nb) acc[i][nb] = 0.0f;
+                float rscale[R];  // e4m3 rows: their scales, loaded under the FMA loop
+#pragma unroll
+                for (int i = 0; i < R; ++i) rscale[i] = Q8 ? __ldg(p.row_scale + row0 + rr[i]) : 1.0f;
                 if (w < rows) {
                     for (int c = lane; c < C; c += 32) {
                         uint4 wv[R];
@@ -794,22 +818,39 @@ __global__ void __launch_bounds__(kThreads, 1) stream_topk_kernel(const StreamTo
                             wv[i] = *reinterpret_cast<const uint4 *>(stage + rr[i] * row_bytes + c * 16);
 #pragma unroll
                         for (int nb = 0; nb < NB; ++nb) {
-                            const float4 ha = *reinterpret_cast<const float4 *>(
-                                h_s + (nb * 2 + 0) * (C * 4) + c * 4);
-                            const float4 hb = *reinterpret_cast<const float4 *>(
-                                h_s + (nb * 2 + 1) * (C * 4) + c * 4);
+                            if constexpr (Q8) {
+                                const float *hq = h_s + nb * 4 * (C * 4) + c * 4;
+                                const float4 h0 = *reinterpret_cast<const float4 *>(hq);
+                                const float4 h1 = *reinterpret_cast<const float4 *>(hq + 1 * (C * 4));
+                                const float4 h2 = *reinterpret_cast<const float4 *>(hq + 2 * (C * 4));
+                                const float4 h3 = *reinterpret_cast<const float4 *>(hq + 3 * (C * 4));
 #pragma unroll
-                            for (int i = 0; i < R; ++i) {
-                                float a = acc[i][nb];
-                                a = fmaf(bf16_lo(wv[i].x), ha.x, a);
-                                a = fmaf(bf16_hi(wv[i].x), ha.y, a);
-                                a = fmaf(bf16_lo(wv[i].y), ha.z, a);
-                                a = fmaf(bf16_hi(wv[i].y), ha.w, a);
-                                a = fmaf(bf16_lo(wv[i].z), hb.x, a);
-                                a = fmaf(bf16_hi(wv[i].z), hb.y, a);
-                                a = fmaf(bf16_lo(wv[i].w), hb.z, a);
-                                a = fmaf(bf16_hi(wv[i].w), hb.w, a);
-                                acc[i][nb] = a;
+                                for (int i = 0; i < R; ++i) {
+                                    float a = acc[i][nb];
+                                    a = fma_e4m3x4(wv[i].x, h0, a);
+                                    a = fma_e4m3x4(wv[i].y, h1, a);
+                                    a = fma_e4m3x4(wv[i].z, h2, a);
+                                    a = fma_e4m3x4(wv[i].w, h3, a);
+                                    acc[i][nb] = a;
+                                }
+                            } else {
+                                const float4 ha = *reinterpret_cast<const float4 *>(
+                                    h_s + (nb * 2 + 0) * (C * 4) + c * 4);
+                                const float4 hb = *reinterpret_cast<const float4 *>(
+                                    h_s + (nb * 2 + 1) * (C * 4) + c * 4);
+#pragma unroll
+                                for (int i = 0; i < R; ++i) {
+                                    float a = acc[i][nb];
+                                    a = fmaf(bf16_lo(wv[i].x), ha.x, a);
+                                    a = fmaf(bf16_hi(wv[i].x), ha.y, a);
+                                    a = fmaf(bf16_lo(wv[i].y), ha.z, a);
+                                    a = fmaf(bf16_hi(wv[i].y), ha.w, a);
+                                    a = fmaf(bf16_lo(wv[i].z), hb.x, a);
+                                    a = fmaf(bf16_hi(wv[i].z), hb.y, a);
+                                    a = fmaf(bf16_lo(wv[i].w), hb.z, a);
+                                    a = fmaf(bf16_hi(wv[i].w), hb.w, a);
+                                    acc[i][nb] = a;
+                                }
                             }
                         }
                     }
@@ -842,7 +883,8 @@ __global__ void __launch_bounds__(kThreads, 1) stream_topk_kernel(const StreamTo
                         const int r = w + i * kDotWarps;
                         if (r < rows) {
 #pragma unroll
-                            for (int nb = 0; nb < NB; ++nb) sc[r * NB + nb] = acc[i][nb];
+                            for (int nb = 0; nb < NB; ++nb)
+                                sc[r * NB + nb] = Q8 ? acc[i][nb] * rscale[i] : acc[i][nb];
                         }
                     }
                 }

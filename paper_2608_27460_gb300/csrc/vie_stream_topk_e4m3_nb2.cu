@@ -1,0 +1,9 @@
+// Instantiations of the streaming top-k kernel on e4m3 rows for query groups of 2.
+#include "vie_stream_topk_inst.cuh"
+
+namespace vie {
+cudaError_t launch_stream_topk_e4m3_nb2(int mm, int r, const StreamTopkParams &p, int grid,
+                                        uint32_t smem, cudaStream_t stream) {
+    return launch_width<2, true>(mm, r, p, grid, smem, stream);
+}
+}  // namespace vie

@@ -6,7 +6,7 @@
 
 namespace vie {
 
-template <int NB, int MM, int kR>
+template <int NB, int MM, int kR, bool Q8>
 cudaError_t launch_one(const StreamTopkParams &p, int grid, uint32_t smem, cudaStream_t stream) {
     static bool configured[64] = {};
     int dev = 0;
@@ -14,40 +14,40 @@ cudaError_t launch_one(const StreamTopkParams &p, int grid, uint32_t smem, cudaS
     if (e != cudaSuccess) return e;
     if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
     if (!configured[dev]) {
-        e = cudaFuncSetAttribute(stream_topk_kernel<NB, MM, kR>,
+        e = cudaFuncSetAttribute(stream_topk_kernel<NB, MM, kR, Q8>,
                                  cudaFuncAttributeMaxDynamicSharedMemorySize, 232448);
         if (e != cudaSuccess) return e;
         configured[dev] = true;
     }
-    stream_topk_kernel<NB, MM, kR><<<grid, kThreads, smem, stream>>>(p);
+    stream_topk_kernel<NB, MM, kR, Q8><<<grid, kThreads, smem, stream>>>(p);
     return cudaGetLastError();
 }
 
-template <int NB, int R>
+template <int NB, int R, bool Q8>
 cudaError_t launch_rows(int mm, const StreamTopkParams &p, int grid, uint32_t smem,
                         cudaStream_t stream) {
     // Wide lists are only built for narrow query groups (register budget).
     switch (mm) {
-        case 2: return launch_one<NB, 2, R>(p, grid, smem, stream);
+        case 2: return launch_one<NB, 2, R, Q8>(p, grid, smem, stream);
         case 8:
-            if constexpr (NB <= 4) return launch_one<NB, 8, R>(p, grid, smem, stream);
+            if constexpr (NB <= 4) return launch_one<NB, 8, R, Q8>(p, grid, smem, stream);
             return cudaErrorInvalidValue;
         case 32:
-            if constexpr (NB == 1) return launch_one<NB, 32, R>(p, grid, smem, stream);
+            if constexpr (NB == 1) return launch_one<NB, 32, R, Q8>(p, grid, smem, stream);
             return cudaErrorInvalidValue;
         default: return cudaErrorInvalidValue;
     }
 }
 
-template <int NB>
+template <int NB, bool Q8>
 cudaError_t launch_width(int mm, int r, const StreamTopkParams &p, int grid, uint32_t smem,
                          cudaStream_t stream) {
     switch (r) {
-        case 1: return launch_rows<NB, 1>(mm, p, grid, smem, stream);
-        case 2: return launch_rows<NB, 2>(mm, p, grid, smem, stream);
-        case 4: return launch_rows<NB, 4>(mm, p, grid, smem, stream);
+        case 1: return launch_rows<NB, 1, Q8>(mm, p, grid, smem, stream);
+        case 2: return launch_rows<NB, 2, Q8>(mm, p, grid, smem, stream);
+        case 4: return launch_rows<NB, 4, Q8>(mm, p, grid, smem, stream);
         case 8:  // narrow rows, one query: 64-row stages
-            if constexpr (NB == 1) return launch_rows<NB, 8>(mm, p, grid, smem, stream);
+            if constexpr (NB == 1) return launch_rows<NB, 8, Q8>(mm, p, grid, smem, stream);
             return cudaErrorInvalidValue;
         default: return cudaErrorInvalidValue;
     }

@@ -4,6 +4,6 @@
 namespace vie {
 cudaError_t launch_stream_topk_nb8(int mm, int r, const StreamTopkParams &p, int grid,
                                    uint32_t smem, cudaStream_t stream) {
-    return launch_width<8>(mm, r, p, grid, smem, stream);
+    return launch_width<8, false>(mm, r, p, grid, smem, stream);
 }
 }  // namespace vie

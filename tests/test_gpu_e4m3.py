@@ -1,0 +1,99 @@
+"""GPU parity of the e4m3-quantised head (vie_head_create_e4m3): the
+device quantiser gives the oracle's codes and scales bit for bit, and every
+top-k call on the handle matches the oracle's head on those codes
+(z_i = scale_i * sum_j e4m3(q_ij) h_j) under the usual acceptance rule."""
+import numpy as np
+import pytest
+
+import oracle
+from acceptance import check_topk
+from gpu_cases import to_device_bits, workload
+from paper_2608_27460_gb300 import synth
+
+pytestmark = pytest.mark.gpu
+
+
+def _head(vie, W):
+    return vie.Head(to_device_bits(W), storage="e4m3")
+
+
+@pytest.mark.parametrize("V,d", [(3001, 100), (2003, 640), (1009, 1024), (257, 16)])
+def test_quantiser_is_bit_exact(vie, V, d):
+    W, _ = workload(V, d, 1, seed=V + d)
+    W[7] = 0  # an all-zero row
+    oq, osc = oracle.quantize_e4m3(W)
+    with _head(vie, W) as head:
+        codes, scales = head.export_e4m3()
+        np.testing.assert_array_equal(codes.cpu().numpy(), oq)
+        np.testing.assert_array_equal(scales.cpu().numpy().view(np.uint32), osc.view(np.uint32))
+        p = head.props
+        assert p.d_pad == (d + 15) // 16 * 16 and p.weight_bytes == V * p.d_pad + V * 4
+        assert head.plan(16, 50).path == 0  # e4m3 heads stay on the streaming kernel
+
+
+def _parity(vie, W, h, k, reps=1):
+    import torch
+    q, sc = oracle.quantize_e4m3(W)
+    z = oracle.logits_e4m3(q, sc, h)
+    with _head(vie, W) as head:
+        hd = torch.from_numpy(h).cuda()
+        prev = None
+        for _ in range(reps):
+            idx, val = head.topk(hd, k)
+            torch.cuda.synchronize()
+            cur = (idx.cpu().numpy(), val.cpu().numpy())
+            if prev is not None:
+                assert np.array_equal(prev[0], cur[0]) and np.array_equal(prev[1].view(np.uint32),
+                                                                           cur[1].view(np.uint32))
+            prev = cur
+        assert head.device_status() == vie.VIE_OK
+    fails = {q_: e for q_ in range(h.shape[0]) if (e := check_topk(prev[0][q_], prev[1][q_], z[q_], k))}
+    assert not fails, next(iter(fails.items()))
+    return prev, z
+
+
+@pytest.mark.parametrize("V,d,batch,k", [
+    (20011, 640, 1, 50),
+    (20011, 1024, 1, 50),
+    (4099, 100, 3, 50),      # padded rows
+    (33333, 2048, 4, 1),
+    (30011, 512, 8, 64),
+    (30011, 512, 13, 50),    # two query groups
+    (9973, 256, 2, 300),
+    (5000, 1152, 1, 1024),
+])
+def test_e4m3_head_matches_the_oracle(vie, V, d, batch, k):
+    W, h = workload(V, d, batch, seed=V + d + batch)
+    _parity(vie, W, h, k, reps=2)
+
+
+def test_duplicate_rows_tie_by_index(vie):
+    W, h = workload(40009, 640, 4, seed=23, dup_frac=0.05, planted=0.5)
+    (idx, val), _ = _parity(vie, W, h, 50)
+    for q in range(4):
+        for j in range(1, 50):
+            if val[q, j] == val[q, j - 1]:
+                assert idx[q, j] > idx[q, j - 1]
+
+
+@pytest.mark.parametrize("name,batch,k,n", [("qwen3-0.6b", 1, 50, 2), ("gemma3-270m", 1, 50, 2),
+                                            ("llama3.2-1b", 4, 50, 4)])
+def test_e4m3_full_size(vie, name, batch, k, n):
+    shape = synth.HEADS[name]
+    W, h, _, _ = synth.make_head(shape, seed=0, n_queries=n)
+    _parity(vie, W, h[:n], k)
+
+
+def test_host_entry_and_sampling_on_e4m3(vie):
+    import torch
+    W, h = workload(20011, 512, 3, seed=3)
+    with _head(vie, W) as head:
+        ri, rv = head.topk(torch.from_numpy(h).cuda(), 50)
+        gi, gv = head.topk_host(torch.from_numpy(h), 50)
+        torch.cuda.synchronize()
+        np.testing.assert_array_equal(gi.numpy(), ri.cpu().numpy())
+        idx, val, tok, prob = head.topk_sample(torch.from_numpy(h).cuda(), 50, 0.8, 0.9, 0.05, seed=1, step=2)
+        torch.cuda.synchronize()
+        for q in range(3):
+            assert tok[q].item() in idx[q].cpu().numpy()
+        assert head.device_status() == vie.VIE_OK
