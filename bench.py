@@ -39,6 +39,7 @@ PROFILE_DIR = os.path.join(ROOT, "profiles")
 # digest still matches.
 KERNEL_SOURCES = {
     "stream_topk": ["vie_stream_topk.cuh", "vie_device.cuh", "vie_stream_topk_inst.cuh"],
+    "stream_topk_e4m3": ["vie_stream_topk.cuh", "vie_device.cuh", "vie_stream_topk_inst.cuh"],
     "tc_topk": ["vie_tc_topk.cuh", "vie_tc_topk.cu", "vie_tcgen05.cuh", "vie_device.cuh",
                 "vie_stream_topk.cuh"],
 }
@@ -58,6 +59,8 @@ def parse_args(argv=None):
     ap.add_argument("--cpu-seconds", type=float, default=15.0, help="oracle sample budget")
     ap.add_argument("--e2e-steps", type=int, default=200)
     ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--storage", choices=["bf16", "e4m3"], default="bf16",
+                    help="bf16 rows, or e4m3 rows with an fp32 scale each (half the bytes)")
     ap.add_argument("--sample", action="store_true",
                     help="each step also draws the next token on the device (temperature 0.8, "
                          "top-p 0.9, min-p 0.05, Philox keyed by the step)")
@@ -194,19 +197,32 @@ def gpu_id_for_smi(local_rank: int) -> str:
 
 
 # ---------------------------------------------------------------------------
-def cpu_oracle_sample(W, h_pool, k, budget_s, batch):
+def oracle_head(W, storage):
+    """The oracle's top-k for this storage: bf16 rows, or its own e4m3
+    quantisation of them (done once, outside any timing)."""
+    import oracle
+    if storage == "e4m3":
+        q, sc = oracle.quantize_e4m3(W)
+        return (lambda hb, k, threads: oracle.topk_e4m3(q, sc, hb, k, threads=threads),
+                lambda hb: oracle.logits_e4m3(q, sc, hb))
+    return (lambda hb, k, threads: oracle.topk(W, hb, k, threads=threads),
+            lambda hb: oracle.logits(W, hb))
+
+
+def cpu_oracle_sample(W, h_pool, k, budget_s, batch, storage="bf16"):
     """The oracle, as it stands, on host cores: whole decode steps (top-k by
     full sort + sparse tensor) until the time budget is spent."""
     import oracle
     threads = oracle.max_threads()
     V = W.shape[0]
+    topk, _ = oracle_head(W, storage)
     t0 = time.perf_counter()
     n = 0
     results = {}
     while True:
         q0 = (n * batch) % len(h_pool)
         hb = h_pool[q0:q0 + batch]
-        idx, val = oracle.topk(W, hb, k, threads=threads)
+        idx, val = topk(hb, k, threads)
         oracle.scatter(idx, val.astype(np.float32), V)
         results[q0] = (idx, val)
         n += 1
@@ -225,10 +241,11 @@ def run_reference(args, rank, world):
     import oracle
     threads = oracle.max_threads()
     V = W.shape[0]
+    topk, _ = oracle_head(W, args.storage)
 
     def step(i):
         q0 = (i * args.batch) % (len(h) - args.batch + 1)
-        idx, val = oracle.topk(W, h[q0:q0 + args.batch], args.k, threads=threads)
+        idx, val = topk(h[q0:q0 + args.batch], args.k, threads)
         oracle.scatter(idx, val.astype(np.float32), V)
         if args.sample:
             oracle.sample(val, 0.8, 0.9, 0.05, args.seed, i)
@@ -259,7 +276,9 @@ def workload_config(args, shape):
     return {"workload": f"{shape.name}-shaped head, batch {args.batch}, k {args.k}"
                         + (", then a top-k draw" if getattr(args, "sample", False) else ""),
             "V": shape.V, "d": shape.d, "batch": args.batch, "k": args.k,
-            "weights": "bf16 (fp32 accumulation)",
+            "weights": "bf16 (fp32 accumulation)" if getattr(args, "storage", "bf16") == "bf16"
+                       else "e4m3 with an fp32 scale per row, quantised from the bf16 weights "
+                            "(fp32 accumulation)",
             "l2": ("flushed between timed steps (256 MB read); value = mean of per-step CUDA "
                    "events around the head launch" if getattr(args, "l2", "flush") == "flush" else
                    f"inputs larger than L2 (W_out {shape.V * shape.d * 2 / 1e6:.0f} MB vs 129 MB L2), "
@@ -288,7 +307,7 @@ def main(argv=None):
     nq = max(args.queries, args.batch)
     W, h, _, _ = synth.make_head(shape, seed=args.seed + rank * 7919, n_queries=nq)
     Wd = torch.from_numpy(W.view(np.int16)).to(dev)
-    head = vie.Head(Wd)
+    head = vie.Head(Wd, storage=args.storage)
     del Wd
     hd = torch.from_numpy(h).to(dev)
     b, k, V = args.batch, args.k, shape.V
@@ -392,11 +411,12 @@ def main(argv=None):
     props = head.props
     peaks, peak_src = measured_peaks()
     kern_us = statistics.mean(kern_ms) * 1e3
-    w_bytes = shape.V * props.d_pad * 2
+    w_bytes = props.weight_bytes  # bf16: V*d_pad*2; e4m3: V*d_pad + V*4 (codes and scales)
     alg_bytes = w_bytes + b * shape.d * 4 + b * k * 8
     achieved = alg_bytes / (kern_us * 1e-6) / 1e9
     plan = head.plan(b, k)
-    kernel = "stream_topk" if plan.path == 0 else "tc_topk"
+    kernel = ("stream_topk_e4m3" if args.storage == "e4m3" else "stream_topk") if plan.path == 0 \
+        else "tc_topk"
     traffic, prof_path = profiled_traffic(kernel, args.workload, b, k)
     value = whole_job_us_per_step(step_us, world)
     launches_per_step = plan.launches + (1 if args.sample else 0)
@@ -422,12 +442,13 @@ def main(argv=None):
         "metric": METRIC, "value": round(value, 3), "unit": UNIT, "n_gpus": world,
         "steps": K, "warmup": args.warmup, "ms_per_step": round(step_us / 1e3, 6),
         "higher_is_better": False, "scaling": "weak", "vs_baseline": None,
-        "dtype": "f32", "data": "synthetic", "config": workload_config(args, shape),
+        "dtype": "f32" if args.storage == "bf16" else "f32 (e4m3 weights)", "data": "synthetic",
+        "config": workload_config(args, shape),
         "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": peaks["hbm_gbs"],
                      "unit": "GB/s", "frac": round(achieved / peaks["hbm_gbs"], 4),
                      "traffic": traffic, "peak_source": peak_src,
-                     "kernel": "stream_topk_kernel" if plan.path == 0 else
-                               "tc_topk_kernel (step: prep + projection + merge)",
+                     "kernel": ("stream_topk_kernel" + (" (e4m3 rows)" if args.storage == "e4m3" else ""))
+                               if plan.path == 0 else "tc_topk_kernel (step: prep + projection + merge)",
                      "profile": os.path.relpath(prof_path, ROOT) if prof_path else None,
                      "kernel_us": round(kern_us, 3),
                      "algorithmic_bytes_per_launch": alg_bytes,
@@ -447,7 +468,8 @@ def main(argv=None):
         # algorithmic flops 2*V*d*b; the MMAs issue 2*V*d_pad*(2 rows per
         # query: hi and lo halves of h) over the padded query group
         alg_flops = 2.0 * shape.V * shape.d * b
-        nq_tile = 8 if b <= 8 else (16 if b <= 16 else 32)
+        per_group = -(-b // plan.groups)
+        nq_tile = max(8, 1 << (per_group - 1).bit_length())  # the tile the library picked
         issued = 2.0 * shape.V * props.d_pad * 2 * nq_tile * plan.groups
         tf = alg_flops / (kern_us * 1e-6) / 1e12
         line["roofline_tensor"] = {
@@ -456,7 +478,7 @@ def main(argv=None):
             "issued_mma_tflops": round(issued / (kern_us * 1e-6) / 1e12, 2),
             "peak_source": peak_src}
     if not args.no_cpu_baseline and world == 1:
-        us, n, threads, results = cpu_oracle_sample(W, h, k, args.cpu_seconds, b)
+        us, n, threads, results = cpu_oracle_sample(W, h, k, args.cpu_seconds, b, args.storage)
         line["cpu_baseline"] = {"value": round(us, 1), "unit": UNIT, "cores": threads, "kind": "oracle",
                                 "sample": f"{n} decode steps (batch {b}) of the same workload in "
                                           f"{args.cpu_seconds:.0f} s: fp64 projection, full sort, "
@@ -466,10 +488,11 @@ def main(argv=None):
         import oracle
         from acceptance import check_topk
         ok = True
+        logits = oracle_head(W, args.storage)[1]
         for q0 in list(results)[:2]:
             gi, gv = head.topk(hd[q0:q0 + b], k)
             torch.cuda.synchronize()
-            z = oracle.logits(W, h[q0:q0 + b])
+            z = logits(h[q0:q0 + b])
             for q in range(b):
                 ok &= not check_topk(gi.cpu().numpy()[q], gv.cpu().numpy()[q], z[q], k)
         line["parity_sample_ok"] = bool(ok)

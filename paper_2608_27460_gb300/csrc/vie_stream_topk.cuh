@@ -591,7 +591,9 @@ __device__ __forceinline__ int stage_rows(int64_t row0, int64_t pool_row0, int R
 }
 
 // e4m3 x4 (one 32-bit word, element 0 in the low byte) times h.x..h.w into a,
-// in element order; each e4m3 value is exact in fp16 and fp32.
+// in element order; each e4m3 value is exact in fp16 and fp32.  (Decoding by
+// integer shifts into fp32 bits instead took more instructions per weight
+// than these conversions.)
 __device__ __forceinline__ float fma_e4m3x4(uint32_t w, float4 h, float a) {
     const float2 lo = __half22float2(__half2(__nv_cvt_fp8x2_to_halfraw2(
         static_cast<__nv_fp8x2_storage_t>(w & 0xFFFFu), __NV_E4M3)));

@@ -97,3 +97,40 @@ def test_host_entry_and_sampling_on_e4m3(vie):
         for q in range(3):
             assert tok[q].item() in idx[q].cpu().numpy()
         assert head.device_status() == vie.VIE_OK
+
+
+def _wide_range_weights(V, d, seed):
+    """Rows whose magnitudes span 2^-18 .. 1: after the per-row scale they land
+    on every e4m3 binade, subnormal codes and zero included."""
+    rng = np.random.default_rng(seed)
+    mag = np.exp2(rng.uniform(-18.0, 0.0, (V, d)))
+    sign = np.where(rng.random((V, d)) < 0.5, -1.0, 1.0)
+    return synth.f32_to_bf16_bits((sign * mag).astype(np.float32))
+
+
+@pytest.mark.parametrize("hval", [1.0, -0.375, 2.0**40, 2.0**-30, 1.5 * 2.0**70])
+def test_one_hot_queries_give_exact_products(vie, hval):
+    """With h = hval * e_j every logit is one product scale_i * e4m3(q_ij) *
+    hval, which the kernel must return rounded once to fp32: equal, bit for
+    bit, to the oracle's fp64 value rounded to fp32, for normal and subnormal
+    codes alike."""
+    import torch
+    V, d, k = 4096, 48, 1024
+    W = _wide_range_weights(V, d, seed=17)
+    q, sc = oracle.quantize_e4m3(W)
+    assert ((q & 0x78) == 0).mean() > 0.05  # subnormal codes (and zeros) are common
+    cols = [0, 5, 16, 31, 47]
+    h = np.zeros((len(cols), d), np.float32)
+    for r, j in enumerate(cols):
+        h[r, j] = hval
+    z = oracle.logits_e4m3(q, sc, h)
+    with _head(vie, W) as head:
+        idx, val = head.topk(torch.from_numpy(h).cuda(), k)
+        torch.cuda.synchronize()
+        assert head.device_status() == vie.VIE_OK
+    idx, val = idx.cpu().numpy(), val.cpu().numpy()
+    for r in range(len(cols)):
+        want = z[r][idx[r]].astype(np.float32)
+        np.testing.assert_array_equal(val[r].view(np.uint32), want.view(np.uint32))
+        assert not check_topk(idx[r], val[r], z[r], k)
+
