@@ -20,6 +20,9 @@ only builds it with gcc and marshals numpy arrays through ctypes.
                        gives each (seed, step, query) its uniform
   * :func:`quantize_e4m3`, :func:`logits_e4m3`, :func:`topk_e4m3` -- the head
                        on rows stored as e4m3 codes with one fp32 scale each
+  * :func:`recall_hits`, :func:`recall_at_k` -- Recall@k bookkeeping: how
+                       many exact top-k indices an approximate search
+                       returned                                   (Section 4.3)
 
 Parity of :func:`topk` against the paper cannot be pinned to printed values
 (the paper prints no worked example); it is pinned instead to hand-worked
@@ -104,6 +107,8 @@ class OracleLib:
         lib.oracle_topk_e4m3.argtypes = [P, P, ctypes.c_int64, ctypes.c_int32, P, ctypes.c_int32,
                                          ctypes.c_int32, P, P, ctypes.c_int32]
         lib.oracle_topk_e4m3.restype = ctypes.c_int
+        lib.oracle_recall_hits.argtypes = [P, ctypes.c_int32, P, ctypes.c_int32, ctypes.c_int64, P]
+        lib.oracle_recall_hits.restype = ctypes.c_int
         self.lib = lib
         self.path = path
 
@@ -237,6 +242,27 @@ class OracleLib:
             raise ValueError(f"oracle_topk_e4m3 failed with code {rc}")
         return idx, val
 
+    def recall_hits(self, exact: np.ndarray, approx: np.ndarray) -> np.ndarray:
+        """Per query, how many of the exact top-k indices [n, k] are among the
+        approximate candidates [n, m] (a set; negative entries are empty)."""
+        exact = np.ascontiguousarray(np.atleast_2d(exact), dtype=np.int32)
+        approx = np.ascontiguousarray(np.atleast_2d(approx), dtype=np.int32)
+        if exact.shape[0] != approx.shape[0]:
+            raise ValueError("exact and approx must have one row per query each")
+        n, k = exact.shape
+        m = approx.shape[1]
+        hits = np.empty(n, dtype=np.int32)
+        rc = self.lib.oracle_recall_hits(_ptr(exact), k, _ptr(approx), m, n, _ptr(hits))
+        if rc != 0:
+            raise ValueError(f"oracle_recall_hits failed with code {rc}")
+        return hits
+
+    def recall_at_k(self, exact: np.ndarray, approx: np.ndarray) -> float:
+        """Recall@k over the queries: total hits / (n k)."""
+        hits = self.recall_hits(exact, approx)
+        exact = np.atleast_2d(exact)
+        return float(hits.sum()) / (exact.shape[0] * exact.shape[1])
+
 
 def _default() -> OracleLib:
     global _lib
@@ -293,3 +319,10 @@ def logits_e4m3(q, scale, h, threads: int = 0):
 def topk_e4m3(q, scale, h, k: int, threads: int = 0):
     return _default().topk_e4m3(q, scale, h, k, threads)
 
+
+def recall_hits(exact, approx):
+    return _default().recall_hits(exact, approx)
+
+
+def recall_at_k(exact, approx) -> float:
+    return _default().recall_at_k(exact, approx)

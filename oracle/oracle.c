@@ -51,6 +51,14 @@
  *   q_ij = e4m3(w_ij / scale_i), the fp32 quotient rounded to the nearest
  *          e4m3 value, ties to even, magnitudes past 448 saturated;
  * and the head computes z_i = scale_i * sum_j e4m3(q_ij) * h_j.
+ *
+ * Recall@k (Section 4.3: the share of the exact head's top-k tokens that an
+ * approximate search also retrieves, averaged over many hidden states).
+ * Readings: the approximate method hands over m candidate indices per query
+ * (m may differ from k), taken as a set: a repeated candidate counts once and
+ * a negative entry is an empty slot; the hits of a query are the positions
+ * j < k of the exact top-k whose index is among the candidates; Recall@k is
+ * the sum of the hits over the n queries divided by n k.
  */
 #include <math.h>
 #include <stdint.h>
@@ -379,3 +387,24 @@ int oracle_topk_e4m3(const uint8_t *q, const float *scale, int64_t V, int32_t d,
     return rc;
 }
 
+/* ------------------------------------------------------------------------ */
+/* hits[q] = #{ j < k : exact[q, j] >= 0 and exact[q, j] in {approx[q, i] : i < m} } */
+int oracle_recall_hits(const int32_t *exact, int32_t k, const int32_t *approx, int32_t m, int64_t n,
+                       int32_t *hits) {
+    if (!exact || !approx || !hits || k < 1 || m < 1 || n < 1) return ORACLE_EINVAL;
+    for (int64_t q = 0; q < n; ++q) {
+        const int32_t *eq = exact + q * k, *aq = approx + q * m;
+        int32_t h = 0;
+        for (int32_t j = 0; j < k; ++j) {
+            if (eq[j] < 0) continue;
+            for (int32_t i = 0; i < m; ++i) {
+                if (aq[i] == eq[j]) {
+                    ++h;
+                    break;
+                }
+            }
+        }
+        hits[q] = h;
+    }
+    return ORACLE_OK;
+}

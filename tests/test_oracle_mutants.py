@@ -13,6 +13,7 @@ import oracle as default_oracle
 from test_oracle_pins import PINS
 from test_oracle_sampling import SAMPLING_PINS
 from test_oracle_fp8 import FP8_PINS
+from test_oracle_recall import RECALL_PINS
 
 SRC = os.path.join(os.path.dirname(default_oracle.__file__), "oracle.c")
 
@@ -49,6 +50,11 @@ MUTANTS = {
     "e4m3_decode_bias": ("v = ldexp(1.0 + M / 8.0, E - 7);", "v = ldexp(1.0 + M / 8.0, E - 8);"),
     "scale_wrong_range": ("const float s = amax > 0.0f ? amax / 448.0f : 1.0f;", "const float s = amax > 0.0f ? amax / 240.0f : 1.0f;"),
     "logits_scale_dropped": ("zb[i] = (double)scale[i] * acc;", "zb[i] = acc;"),
+    # Recall@k bookkeeping
+    "recall_repeats_counted": ("++h;\n                    break;", "++h;"),
+    "recall_last_candidate_missed": ("for (int32_t i = 0; i < m; ++i) {", "for (int32_t i = 0; i + 1 < m; ++i) {"),
+    "recall_wrong_row_stride": ("*aq = approx + q * m;", "*aq = approx + q * k;"),
+    "recall_empty_slots_match": ("if (eq[j] < 0) continue;", ""),
 }
 
 
@@ -61,7 +67,7 @@ def test_pins_catch_planted_mistake(name, tmp_path):
     src.write_text(text.replace(old, new, 1))
     lib = default_oracle.OracleLib(default_oracle.build(True, str(src), str(tmp_path / f"{name}.so")))
     caught = []
-    for pin_name, pin in PINS + SAMPLING_PINS + FP8_PINS:
+    for pin_name, pin in PINS + SAMPLING_PINS + FP8_PINS + RECALL_PINS:
         try:
             pin(lib)
         except (AssertionError, ValueError):
