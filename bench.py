@@ -64,6 +64,11 @@ def parse_args(argv=None):
     ap.add_argument("--sample", action="store_true",
                     help="each step also draws the next token on the device (temperature 0.8, "
                          "top-p 0.9, min-p 0.05, Philox keyed by the step)")
+    ap.add_argument("--recall", type=int, default=0, metavar="N",
+                    help="also time the exact head as a Recall@k ground truth over N hidden states "
+                         "(Section 4.3 uses 20000 and k = 2) and report the Recall@k of the e4m3 "
+                         "head against it")
+    ap.add_argument("--recall-k", type=int, default=2)
     ap.add_argument("--l2", choices=["flush", "resident"], default="flush",
                     help="flush: read a 256 MB buffer between timed steps (evicts W_out from L2 "
                          "with clean lines, like the other layers of a decode step would) and time "
@@ -207,6 +212,70 @@ def oracle_head(W, storage):
                 lambda hb: oracle.logits_e4m3(q, sc, hb))
     return (lambda hb, k, threads: oracle.topk(W, hb, k, threads=threads),
             lambda hb: oracle.logits(W, hb))
+
+
+def recall_leg(args, vie, shape, W, exact_head, dev):
+    """The exact head as the ground truth of a Recall@k evaluation (Section
+    4.3): exact top-k of N hidden states (vie_head_topk_many), the e4m3 head's
+    top-k of the same states as the approximate head, and the hit counts
+    (vie_recall_hits), each timed with CUDA events on the launching stream."""
+    import torch
+    N, k = args.recall, args.recall_k
+    hq, _ = synth.make_queries(W, N, seed=args.seed + 101)
+    hd = torch.from_numpy(hq).to(dev)
+    own = exact_head is None
+    if own:
+        exact_head = vie.Head(torch.from_numpy(W.view(np.int16)).to(dev))
+    approx_head = vie.Head(torch.from_numpy(W.view(np.int16)).to(dev), storage="e4m3")
+    stream = torch.cuda.current_stream(dev)
+    ei = torch.empty((N, k), dtype=torch.int32, device=dev)
+    ev = torch.empty((N, k), dtype=torch.float32, device=dev)
+    ai = torch.empty((N, k), dtype=torch.int32, device=dev)
+    av = torch.empty((N, k), dtype=torch.float32, device=dev)
+    hits = torch.empty((N,), dtype=torch.int32, device=dev)
+
+    def timed(fn, reps):
+        fn()
+        torch.cuda.synchronize()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(reps):
+            fn()
+        b.record(stream)
+        torch.cuda.synchronize()
+        return a.elapsed_time(b) * 1e3 / reps
+
+    exact_us = timed(lambda: exact_head.topk_many(hd, k, ei, ev, stream), 3)
+    approx_us = timed(lambda: approx_head.topk_many(hd, k, ai, av, stream), 3)
+    recall_us = timed(lambda: vie.recall_hits(ei, ai, hits, stream), 20)
+    vie.check(exact_head.device_status())
+    vie.check(approx_head.device_status())
+    ei_h, ai_h, hits_h = ei.cpu().numpy(), ai.cpu().numpy(), hits.cpu().numpy()
+    # parity: the hit counts against the oracle's on the same lists, and a few
+    # ground-truth rows against the oracle's logits
+    sys.path.insert(0, os.path.join(ROOT, "tests"))
+    import oracle
+    from acceptance import check_topk
+    ok = bool(np.array_equal(hits_h, oracle.recall_hits(ei_h, ai_h)))
+    sample = np.linspace(0, N - 1, 4).astype(int)
+    z = oracle.logits(W, hq[sample])
+    evh = ev.cpu().numpy()
+    ok &= all(not check_topk(ei_h[q], evh[q], z[r], k) for r, q in enumerate(sample))
+    plan = exact_head.plan(min(N, vie.VIE_BATCH_MAX), k)
+    info = {"states": N, "k": k,
+            "ground_truth": "exact bf16 head, vie_head_topk_many (blocks of "
+                            f"{vie.VIE_BATCH_MAX} states, {plan.groups} query groups each)",
+            "ground_truth_us": round(exact_us, 1),
+            "ground_truth_states_per_s": round(N / (exact_us * 1e-6), 1),
+            "approx": "e4m3 head (per-row scales), vie_head_topk_many",
+            "approx_us": round(approx_us, 1),
+            "recall_kernel_us": round(recall_us, 3),
+            f"recall_at_{k}": round(float(hits_h.sum()) / (N * k), 5),
+            "parity_ok": ok}
+    approx_head.close()
+    if own:
+        exact_head.close()
+    return info
 
 
 def cpu_oracle_sample(W, h_pool, k, budget_s, batch, storage="bf16"):
@@ -438,6 +507,9 @@ def main(argv=None):
                        "sample_kernel_us_back_to_back": round(sa.elapsed_time(sb) * 1e3 / 200, 3),
                        "step": "head (top-k and sparse tensor) then the draw, one call, PDL-chained"}
 
+    recall_info = recall_leg(args, vie, shape, W, head if args.storage == "bf16" else None, dev) \
+        if args.recall > 0 else None
+
     line = {
         "metric": METRIC, "value": round(value, 3), "unit": UNIT, "n_gpus": world,
         "steps": K, "warmup": args.warmup, "ms_per_step": round(step_us / 1e3, 6),
@@ -461,6 +533,7 @@ def main(argv=None):
                 "top-k out, synchronised)", "clock": "host wall clock over the steps"},
         "gpu_launches": K * launches_per_step,
         **({"sampling": sample_info} if sample_info else {}),
+        **({"recall": recall_info} if recall_info else {}),
         "clocks": ClockSampler.summarize(clocks, t_wall0, t_wall1),
     }
     if plan.path == 1:

@@ -55,6 +55,9 @@ typedef enum { VIE_DTYPE_BF16 = 0 } vie_dtype;
 #define VIE_K_MAX 1024     /* largest k of vie_head_topk                    */
 #define VIE_BATCH_MAX 1024 /* largest batch of vie_head_topk                */
 #define VIE_D_MAX 16384    /* largest hidden size d                         */
+#define VIE_MANY_MAX (1 << 24)     /* largest n of vie_head_topk_many       */
+#define VIE_RECALL_N_MAX (1 << 28) /* largest n of vie_recall_hits          */
+#define VIE_RECALL_M_MAX (1 << 20) /* largest candidate count m             */
 
 /* Read-only facts about a handle (for callers that size buffers or report). */
 typedef struct {
@@ -239,6 +242,46 @@ vie_status vie_head_topk_sample(vie_head *head, const float *h, int32_t batch, i
                                 uint64_t step, int32_t *out_idx, float *out_logits,
                                 float *out_sparse, int32_t *out_token, float *out_prob,
                                 vie_stream stream);
+
+/*
+ * vie_head_topk_many - the exact top-k of many hidden states, e.g. as the
+ * ground truth against which an approximate head's Recall@k is measured
+ * (Section 4.3 measures it over 20k hidden states).  The same results as
+ * vie_head_topk on each block of up to VIE_BATCH_MAX consecutive states,
+ * enqueued one block after the other on `stream`.
+ *
+ *   h          device, fp32 [n, d], row-major (4-byte aligned).
+ *   n          1 <= n <= VIE_MANY_MAX;   k as for vie_head_topk.
+ *   out_idx, out_logits  device, int32 / fp32 [n, k].
+ *
+ * Errors as for vie_head_topk; a block that fails to launch stops the call
+ * (earlier blocks stay enqueued).
+ */
+vie_status vie_head_topk_many(vie_head *head, const float *h, int64_t n, int32_t k,
+                              int32_t *out_idx, float *out_logits, vie_stream stream);
+
+/*
+ * vie_recall_hits - Recall@k bookkeeping (Section 4.3: recall is the share
+ * of the exact head's top-k tokens that an approximate search also
+ * retrieves).  For each query q:
+ *   out_hits[q] = #{ j < k : exact[q, j] >= 0 and exact[q, j] is among
+ *                            approx[q, 0], ..., approx[q, m - 1] },
+ * the candidates taken as a set (a repeated candidate counts once) and
+ * negative candidates as empty slots.  Recall@k over the n queries is
+ * sum(out_hits) / (n k).  Integer work: the counts are exact.
+ *
+ *   exact     device, int32 [n, k]: the exact top-k indices (vie_head_topk,
+ *             vie_head_topk_many).
+ *   approx    device, int32 [n, m]: the approximate method's candidates.
+ *   1 <= n <= VIE_RECALL_N_MAX;  1 <= k <= VIE_K_MAX;  1 <= m <= VIE_RECALL_M_MAX.
+ *   out_hits  device, int32 [n].  All buffers 4-byte aligned.
+ *
+ * Asynchronous on `stream`, launched as a programmatic dependent of the
+ * kernel before it (it reads its inputs only after that kernel completed).
+ * Errors: VIE_ERR_INVALID_ARG (NULL, sizes, alignment), VIE_ERR_CUDA.
+ */
+vie_status vie_recall_hits(const int32_t *exact, int32_t k, const int32_t *approx, int32_t m,
+                           int64_t n, int32_t *out_hits, vie_stream stream);
 
 /*
  * vie_scatter_sparse_logits - the sparse full-vocabulary logit tensor of

@@ -30,6 +30,9 @@ VIE_DTYPE_BF16 = 0
 VIE_K_MAX = 1024
 VIE_BATCH_MAX = 1024
 VIE_D_MAX = 16384
+VIE_MANY_MAX = 1 << 24
+VIE_RECALL_N_MAX = 1 << 28
+VIE_RECALL_M_MAX = 1 << 20
 
 STATUS_NAMES = {0: "VIE_OK", 1: "VIE_ERR_INVALID_ARG", 2: "VIE_ERR_UNSUPPORTED",
                 3: "VIE_ERR_CUDA", 4: "VIE_ERR_OOM", 5: "VIE_ERR_DEVICE"}
@@ -37,7 +40,7 @@ STATUS_NAMES = {0: "VIE_OK", 1: "VIE_ERR_INVALID_ARG", 2: "VIE_ERR_UNSUPPORTED",
 # Every entry point of include/vie_head.h.
 EXPORTS = ("vie_head_create", "vie_head_destroy", "vie_head_get_props", "vie_head_plan", "vie_head_topk",
            "vie_head_topk_sparse", "vie_head_topk_host", "vie_sample_topk", "vie_head_topk_sample",
-           "vie_head_create_e4m3", "vie_head_export_e4m3",
+           "vie_head_create_e4m3", "vie_head_export_e4m3", "vie_head_topk_many", "vie_recall_hits",
            "vie_head_topk_noalloc", "vie_scatter_sparse_logits", "vie_device_status",
            "vie_head_device_status", "vie_last_error")
 
@@ -95,6 +98,8 @@ def load(path: str | None = None, build_if_missing: bool = True):
             "vie_head_topk_sample": ([P, P, I32, I32, F32, F32, F32, U64, U64, P, P, P, P, P, P],
                                      ctypes.c_int),
             "vie_head_topk_noalloc": ([P, I64, I32, P, I32, I32, P, P, P], ctypes.c_int),
+            "vie_head_topk_many": ([P, P, I64, I32, P, P, P], ctypes.c_int),
+            "vie_recall_hits": ([P, I32, P, I32, I64, P, P], ctypes.c_int),
             "vie_scatter_sparse_logits": ([P, P, I32, I32, I64, P, P], ctypes.c_int),
             "vie_device_status": ([P], ctypes.c_int),
             "vie_head_device_status": ([P, P], ctypes.c_int),
@@ -197,6 +202,34 @@ def sample_topk(idx, logits, temperature: float = 1.0, top_p: float = 1.0, min_p
     return out_token, out_prob
 
 
+def vie_head_topk_many(head: int, h: int, n: int, k: int, out_idx: int, out_logits: int,
+                       stream: int = 0) -> int:
+    return load().vie_head_topk_many(head, h, n, k, out_idx, out_logits, stream)
+
+
+def vie_recall_hits(exact: int, k: int, approx: int, m: int, n: int, out_hits: int,
+                    stream: int = 0) -> int:
+    return load().vie_recall_hits(exact, k, approx, m, n, out_hits, stream)
+
+
+def recall_hits(exact, approx, out_hits=None, stream=None):
+    """Recall@k bookkeeping on CUDA index lists: exact int32 [n, k] and
+    approx int32 [n, m] -> hits int32 [n] (how many exact indices each
+    query's candidates contain; Recall@k = hits.sum() / (n k))."""
+    import torch
+    if exact.dim() != 2 or approx.dim() != 2 or exact.shape[0] != approx.shape[0]:
+        raise ValueError("exact [n, k] and approx [n, m] must have one row per query")
+    if exact.dtype != torch.int32 or approx.dtype != torch.int32 or not (exact.is_cuda and approx.is_cuda):
+        raise ValueError("exact and approx must be CUDA int32 tensors")
+    exact, approx = exact.contiguous(), approx.contiguous()
+    n, k, m = int(exact.shape[0]), int(exact.shape[1]), int(approx.shape[1])
+    if out_hits is None:
+        out_hits = torch.empty((n,), dtype=torch.int32, device=exact.device)
+    check(vie_recall_hits(exact.data_ptr(), k, approx.data_ptr(), m, n, out_hits.data_ptr(),
+                          _stream_ptr(stream)))
+    return out_hits
+
+
 def vie_head_topk_noalloc(W_out: int, V: int, d: int, h: int, batch: int, k: int, out_idx: int,
                           out_logits: int, stream: int = 0) -> int:
     """Top-k straight from caller-owned weights, scratch in a fixed library
@@ -283,6 +316,22 @@ class Head:
             out_logits = torch.empty((b, k), dtype=torch.float32, device=h.device)
         check(vie_head_topk(self.handle, h.data_ptr(), b, k, out_idx.data_ptr(),
                             out_logits.data_ptr(), _stream_ptr(stream)))
+        return out_idx, out_logits
+
+    def topk_many(self, h, k: int, out_idx=None, out_logits=None, stream=None):
+        """Exact top-k of many hidden states h [n, d] (any n up to
+        VIE_MANY_MAX), e.g. the ground truth of a Recall@k evaluation."""
+        import torch
+        if h.dim() != 2 or h.dtype != torch.float32 or not h.is_cuda or h.shape[1] != self.d:
+            raise ValueError(f"h must be a CUDA float32 tensor [n, {self.d}]")
+        h = h.contiguous()
+        n = int(h.shape[0])
+        if out_idx is None:
+            out_idx = torch.empty((n, k), dtype=torch.int32, device=h.device)
+        if out_logits is None:
+            out_logits = torch.empty((n, k), dtype=torch.float32, device=h.device)
+        check(vie_head_topk_many(self.handle, h.data_ptr(), n, k, out_idx.data_ptr(),
+                                 out_logits.data_ptr(), _stream_ptr(stream)))
         return out_idx, out_logits
 
     def plan(self, batch: int, k: int):

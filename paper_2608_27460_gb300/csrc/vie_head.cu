@@ -587,6 +587,24 @@ vie_status vie_head_topk(vie_head *head, const float *h, int32_t batch, int32_t 
     return run_topk("vie_head_topk", head, h, batch, k, out_idx, out_logits, nullptr, stream);
 }
 
+vie_status vie_head_topk_many(vie_head *head, const float *h, int64_t n, int32_t k,
+                              int32_t *out_idx, float *out_logits, vie_stream stream) {
+    const char *fn = "vie_head_topk_many";
+    if (n < 1 || n > VIE_MANY_MAX)
+        return fail(VIE_ERR_INVALID_ARG, "%s: n=%lld outside [1, %d]", fn, static_cast<long long>(n),
+                    VIE_MANY_MAX);
+    if (head == nullptr) return fail(VIE_ERR_INVALID_ARG, "%s: head is NULL", fn);
+    for (int64_t q0 = 0; q0 < n; q0 += VIE_BATCH_MAX) {
+        const int32_t b = static_cast<int32_t>(n - q0 < VIE_BATCH_MAX ? n - q0 : VIE_BATCH_MAX);
+        const vie_status st =
+            run_topk(fn, head, h == nullptr ? nullptr : h + q0 * head->d, b, k,
+                     out_idx == nullptr ? nullptr : out_idx + q0 * k,
+                     out_logits == nullptr ? nullptr : out_logits + q0 * k, nullptr, stream);
+        if (st != VIE_OK) return st;
+    }
+    return VIE_OK;
+}
+
 vie_status vie_head_topk_sparse(vie_head *head, const float *h, int32_t batch, int32_t k,
                                 int32_t *out_idx, float *out_logits, float *out_sparse,
                                 vie_stream stream) {
@@ -617,6 +635,27 @@ vie_status vie_sample_topk(const int32_t *idx, const float *logits, int32_t batc
         return fail(VIE_ERR_INVALID_ARG, "%s: buffers must be 4-byte aligned", fn);
     const cudaError_t e = vie::launch_sample_topk(idx, logits, batch, k, temperature, top_p, min_p,
                                                   seed, step, out_token, out_prob,
+                                                  static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return fail_cuda(e, fn);
+    return VIE_OK;
+}
+
+vie_status vie_recall_hits(const int32_t *exact, int32_t k, const int32_t *approx, int32_t m,
+                           int64_t n, int32_t *out_hits, vie_stream stream) {
+    const char *fn = "vie_recall_hits";
+    if (exact == nullptr || approx == nullptr || out_hits == nullptr)
+        return fail(VIE_ERR_INVALID_ARG, "%s: NULL buffer", fn);
+    if (n < 1 || n > VIE_RECALL_N_MAX)
+        return fail(VIE_ERR_INVALID_ARG, "%s: n=%lld outside [1, %d]", fn, static_cast<long long>(n),
+                    VIE_RECALL_N_MAX);
+    if (k < 1 || k > VIE_K_MAX)
+        return fail(VIE_ERR_INVALID_ARG, "%s: k=%d outside [1, %d]", fn, k, VIE_K_MAX);
+    if (m < 1 || m > VIE_RECALL_M_MAX)
+        return fail(VIE_ERR_INVALID_ARG, "%s: m=%d outside [1, %d]", fn, m, VIE_RECALL_M_MAX);
+    if ((reinterpret_cast<uintptr_t>(exact) | reinterpret_cast<uintptr_t>(approx) |
+         reinterpret_cast<uintptr_t>(out_hits)) & 3u)
+        return fail(VIE_ERR_INVALID_ARG, "%s: buffers must be 4-byte aligned", fn);
+    const cudaError_t e = vie::launch_recall_hits(exact, k, approx, m, n, out_hits,
                                                   static_cast<cudaStream_t>(stream));
     if (e != cudaSuccess) return fail_cuda(e, fn);
     return VIE_OK;

@@ -40,6 +40,9 @@ struct TcParams;
 // Ring depth and dynamic shared memory of the tensor-core kernel for query
 // groups of nq_tmpl (8, 16 or 32) and kps K-blocks per stage; false if
 // unsupported.
+// Recall@k: per query, how many exact top-k indices the candidates contain.
+cudaError_t launch_recall_hits(const int32_t *exact, int k, const int32_t *approx, int m, int64_t n,
+                               int32_t *hits, cudaStream_t stream);
 // Top-k sampling: one draw per query from its k sorted candidates.
 cudaError_t launch_sample_topk(const int32_t *idx, const float *logits, int batch, int k, float T,
                                float top_p, float min_p, uint64_t seed, uint64_t step,

@@ -97,6 +97,35 @@ def test_sampling_rejects_bad_arguments_on_host(lib):
     assert vie.vie_head_topk_sample(0, p, 1, 50, 1.0, 1.0, 0.0, 0, 0, p, p, 0, p, p) == vie.VIE_ERR_INVALID_ARG
 
 
+def test_limits_match_the_header():
+    text = open(HEADER).read()
+    for name in ("VIE_K_MAX", "VIE_BATCH_MAX", "VIE_D_MAX", "VIE_MANY_MAX", "VIE_RECALL_N_MAX",
+                 "VIE_RECALL_M_MAX"):
+        m = re.search(r"#define\s+" + name + r"\s+(\S+(?:\s*<<\s*\d+\))?)", text)
+        assert m, name
+        assert eval(m.group(1)) == getattr(vie, name), name
+
+
+def test_recall_rejects_bad_arguments_on_host(lib):
+    p = 0x10000
+    def call(exact=p, k=2, approx=p, m=2, n=4, out=p):
+        return vie.vie_recall_hits(exact, k, approx, m, n, out)
+    assert call(exact=0) == vie.VIE_ERR_INVALID_ARG
+    assert call(approx=0) == vie.VIE_ERR_INVALID_ARG
+    assert call(out=0) == vie.VIE_ERR_INVALID_ARG
+    assert call(n=0) == vie.VIE_ERR_INVALID_ARG
+    assert call(n=vie.VIE_RECALL_N_MAX + 1) == vie.VIE_ERR_INVALID_ARG
+    assert call(k=0) == vie.VIE_ERR_INVALID_ARG
+    assert call(k=vie.VIE_K_MAX + 1) == vie.VIE_ERR_INVALID_ARG
+    assert call(m=0) == vie.VIE_ERR_INVALID_ARG
+    assert call(m=vie.VIE_RECALL_M_MAX + 1) == vie.VIE_ERR_INVALID_ARG
+    assert call(approx=p + 2) == vie.VIE_ERR_INVALID_ARG
+    assert "vie_recall_hits" in vie.vie_last_error()
+    assert vie.vie_head_topk_many(0, p, 10, 2, p, p) == vie.VIE_ERR_INVALID_ARG
+    assert vie.vie_head_topk_many(0, p, 0, 2, p, p) == vie.VIE_ERR_INVALID_ARG
+    assert vie.vie_head_topk_many(0, p, vie.VIE_MANY_MAX + 1, 2, p, p) == vie.VIE_ERR_INVALID_ARG
+
+
 def test_product_path_does_not_import_the_oracle():
     pkg = os.path.join(ROOT, "paper_2608_27460_gb300")
     for dirpath, _, files in os.walk(pkg):
