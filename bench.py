@@ -40,8 +40,10 @@ PROFILE_DIR = os.path.join(ROOT, "profiles")
 KERNEL_SOURCES = {
     "stream_topk": ["vie_stream_topk.cuh", "vie_device.cuh", "vie_stream_topk_inst.cuh"],
     "stream_topk_e4m3": ["vie_stream_topk.cuh", "vie_device.cuh", "vie_stream_topk_inst.cuh"],
-    "tc_topk": ["vie_tc_topk.cuh", "vie_tc_topk.cu", "vie_tcgen05.cuh", "vie_device.cuh",
+    "tc_topk": ["vie_tc_topk.cuh", "vie_tc_topk.cu", "vie_tc_launch.cuh", "vie_tcgen05.cuh", "vie_device.cuh",
                 "vie_stream_topk.cuh"],
+    "tc_topk_e4m3": ["vie_tc_topk.cuh", "vie_tc_topk_e4m3.cu", "vie_tc_launch.cuh", "vie_tcgen05.cuh",
+                     "vie_device.cuh", "vie_stream_topk.cuh"],
 }
 
 
@@ -484,8 +486,9 @@ def main(argv=None):
     alg_bytes = w_bytes + b * shape.d * 4 + b * k * 8
     achieved = alg_bytes / (kern_us * 1e-6) / 1e9
     plan = head.plan(b, k)
-    kernel = ("stream_topk_e4m3" if args.storage == "e4m3" else "stream_topk") if plan.path == 0 \
-        else "tc_topk"
+    e4m3 = args.storage == "e4m3"
+    kernel = ("stream_topk_e4m3" if e4m3 else "stream_topk") if plan.path == 0 \
+        else ("tc_topk_e4m3" if e4m3 else "tc_topk")
     traffic, prof_path = profiled_traffic(kernel, args.workload, b, k)
     value = whole_job_us_per_step(step_us, world)
     launches_per_step = plan.launches + (1 if args.sample else 0)
@@ -537,19 +540,24 @@ def main(argv=None):
         "clocks": ClockSampler.summarize(clocks, t_wall0, t_wall1),
     }
     if plan.path == 1:
-        # the batched path against the bf16 tensor-core roofline as well:
-        # algorithmic flops 2*V*d*b; the MMAs issue 2*V*d_pad*(2 rows per
-        # query: hi and lo halves of h) over the padded query group
+        # the tensor-core path against its tensor roofline as well: algorithmic
+        # flops 2*V*d*b; the MMAs issue 2*V*d_pad*(columns per query: hi and lo
+        # bf16 halves of h, or four e4m3 pieces) over the padded query group.
+        # The e4m3 peak is the measured bf16 peak times the nominal fp8 / bf16
+        # ratio of 2.
+        cols = 4 if e4m3 else 2
         alg_flops = 2.0 * shape.V * shape.d * b
         per_group = -(-b // plan.groups)
-        nq_tile = max(8, 1 << (per_group - 1).bit_length())  # the tile the library picked
-        issued = 2.0 * shape.V * props.d_pad * 2 * nq_tile * plan.groups
+        nq_tile = max(4 if e4m3 else 8, 1 << (per_group - 1).bit_length())  # the tile the library picked
+        issued = 2.0 * shape.V * props.d_pad * cols * nq_tile * plan.groups
         tf = alg_flops / (kern_us * 1e-6) / 1e12
+        tpeak = peaks["bf16_tflops"] * (2.0 if e4m3 else 1.0)
         line["roofline_tensor"] = {
-            "bound": "tensor", "achieved": round(tf, 2), "peak": peaks["bf16_tflops"],
-            "unit": "TFLOP/s", "frac": round(tf / peaks["bf16_tflops"], 5),
+            "bound": "tensor", "achieved": round(tf, 2), "peak": round(tpeak, 1),
+            "unit": "TFLOP/s", "frac": round(tf / tpeak, 5),
             "issued_mma_tflops": round(issued / (kern_us * 1e-6) / 1e12, 2),
-            "peak_source": peak_src}
+            "peak_source": peak_src + (" (bf16 x 2 for e4m3)" if e4m3 else ""),
+            "operands": "e4m3 x e4m3 (kind::f8f6f4)" if e4m3 else "bf16 x bf16 (kind::f16)"}
     if not args.no_cpu_baseline and world == 1:
         us, n, threads, results = cpu_oracle_sample(W, h, k, args.cpu_seconds, b, args.storage)
         line["cpu_baseline"] = {"value": round(us, 1), "unit": UNIT, "cores": threads, "kind": "oracle",

@@ -109,8 +109,11 @@ vie_status vie_head_create(const void *W_out, int64_t V, int32_t d, vie_dtype dt
  *          to even, saturated at +-448);
  * and every top-k call on the handle (vie_head_topk, _sparse, _host,
  * _sample) computes z_i = scale_i * sum_j e4m3(q_ij) * h_j with fp32
- * accumulation, then the same exact top-k.  Such a handle always uses the
- * streaming CUDA-core kernel (vie_head_plan reports path 0).  Same errors as
+ * accumulation, then the same exact top-k.  Calls with k <= 128 on rows of
+ * at least 128 codes run on the tensor cores (tcgen05 kind::f8f6f4; each
+ * query enters as four e4m3 pieces with power-of-two scales, which keep it to
+ * within 2^-16 |h_j| per entry), from batch 1 (vie_head_plan reports path
+ * 1); other calls use the streaming CUDA-core kernel.  Same errors as
  * vie_head_create.
  */
 vie_status vie_head_create_e4m3(const void *W_out, int64_t V, int32_t d, vie_head **out);

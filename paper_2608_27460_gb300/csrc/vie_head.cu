@@ -62,10 +62,11 @@ struct vie_head {
                         // [3] merging CTAs done (tensor-core path)
     int64_t scratch_bytes;
     // tensor-core path (batches): hi/lo bf16 query matrix and TMA descriptors
-    void *hB;             // [kTcHRows][d_pad] bf16
+    void *hB;             // [kTcHRows][d_pad] bf16, or e4m3 query pieces [4 NQ][d_pad]
+    float *qscale;        // e4m3 heads: [32][kQ8Pieces] piece scales of the query group
     bool tc_ready;
-    CUtensorMap mapW;     // W as [V][d_pad], box 128 rows x 64 columns, 128-byte swizzle
-    CUtensorMap mapH[4];  // hB, box 16 / 32 / 64 / 128 rows x 64 columns
+    CUtensorMap mapW;     // W as [V][d_pad], box 128 rows x 128 bytes, 128-byte swizzle
+    CUtensorMap mapH[4];  // hB, box 16 / 32 / 64 / 128 rows x 128 bytes
     // vie_head_topk_host: device staging of queries and top-k (grown on demand)
     float *stage_h;
     int32_t *stage_idx;
@@ -188,14 +189,15 @@ int env_int(const char *name, int dflt) {
 //   VIE_STATIC_PCT       share of the chunks assigned statically, in % (85)
 //   VIE_POOL_DIV         pool pieces are chunks / this (1)
 //   VIE_TC_MIN_BATCH     smallest batch sent to the tensor-core path (2)
-//   VIE_TC_KPS           K-blocks of 64 columns per tensor-core ring stage (4)
+//   VIE_TC_KPS           128-byte K-blocks per tensor-core ring stage (4)
+//   VIE_TC_MIN_BATCH_E4M3  the same threshold for e4m3 heads (1)
 struct Knobs {
-    int stage_min_bytes, static_pct, tc_min_batch, tc_kps, pool_div;
+    int stage_min_bytes, static_pct, tc_min_batch, tc_kps, pool_div, tc_min_batch_e4m3;
 };
 const Knobs &knobs() {
     static const Knobs k = {env_int("VIE_STAGE_MIN_KB", 48) * 1024, env_int("VIE_STATIC_PCT", 85),
                             env_int("VIE_TC_MIN_BATCH", 2), env_int("VIE_TC_KPS", 4),
-                            env_int("VIE_POOL_DIV", 1)};
+                            env_int("VIE_POOL_DIV", 1), env_int("VIE_TC_MIN_BATCH_E4M3", 1)};
     return k;
 }
 
@@ -258,6 +260,21 @@ EncodeTiledFn encode_tiled() {
         return reinterpret_cast<EncodeTiledFn>(p);
     }();
     return fn;
+}
+
+// 2-D uint8 tensor map [rows][cols] (cols contiguous, pitch bytes), box
+// box_rows x 128 columns, 128-byte swizzle, out-of-range elements read as 0.
+bool make_map_u8(CUtensorMap *m, void *base, uint64_t rows, uint64_t cols, uint64_t pitch,
+                 uint32_t box_rows) {
+    EncodeTiledFn fn = encode_tiled();
+    if (fn == nullptr) return false;
+    const cuuint64_t dims[2] = {cols, rows};
+    const cuuint64_t strides[1] = {pitch};
+    const cuuint32_t box[2] = {128u, box_rows};
+    const cuuint32_t estr[2] = {1, 1};
+    return fn(m, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, base, dims, strides, box, estr,
+              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
 // 2-D bf16 tensor map [rows][cols] (cols contiguous, pitch bytes), box
@@ -338,6 +355,7 @@ static vie_status create_head(const void *W_out, int64_t V, int32_t d, vie_dtype
     if (e == cudaSuccess)
         e = cudaMalloc(&hd->hB, static_cast<size_t>(vie::kTcHRows) * hd->d_pad * 2);
     if (e == cudaSuccess) e = cudaMemset(hd->hB, 0, static_cast<size_t>(vie::kTcHRows) * hd->d_pad * 2);
+    if (e == cudaSuccess && e4m3) e = cudaMalloc(&hd->qscale, 32 * vie::kQ8Pieces * sizeof(float));
     if (e == cudaSuccess) e = cudaMemset(hd->words, 0, 4 * sizeof(uint32_t));
     if (e == cudaSuccess && e4m3) {
         int64_t blocks = (V + 7) / 8;  // 8 rows (warps) per block
@@ -362,11 +380,16 @@ static vie_status create_head(const void *W_out, int64_t V, int32_t d, vie_dtype
         cudaFree(hd->cand);
         cudaFree(hd->words);
         cudaFree(hd->hB);
+        cudaFree(hd->qscale);
         delete hd;
         return st;
     }
-    if (e4m3) {  // e4m3 heads stream through the CUDA-core kernel at every batch size
-        hd->tc_ready = false;
+    if (e4m3) {  // kind::f8f6f4 maps: codes [V][d_pad] and the query pieces, 128-byte rows
+        const uint64_t pitch8 = static_cast<uint64_t>(hd->d_pad);
+        hd->tc_ready = hd->d_pad >= 128 &&
+                       make_map_u8(&hd->mapW, hd->W, static_cast<uint64_t>(V), hd->d_pad, pitch8, vie::kTcTile);
+        for (int i = 0; i < 4 && hd->tc_ready; ++i)
+            hd->tc_ready = make_map_u8(&hd->mapH[i], hd->hB, vie::kTcHRows, hd->d_pad, pitch8, 16u << i);
         *out = hd;
         return VIE_OK;
     }
@@ -414,6 +437,7 @@ vie_status vie_head_destroy(vie_head *head) {
     cudaFree(head->cand);
     cudaFree(head->words);
     cudaFree(head->hB);
+    cudaFree(head->qscale);
     cudaFree(head->stage_h);
     cudaFree(head->stage_idx);
     cudaFree(head->stage_logits);
@@ -438,22 +462,25 @@ vie_status vie_head_get_props(const vie_head *head, vie_head_props *props) {
 // The launch plan of a top-k call (path, query groups, launches).
 // Query slots per tensor-core launch: the smallest tile that holds the batch;
 // 64 (one pass over W for up to 64 queries) only where k fits its lists.
-static int tc_group(int32_t batch, int32_t k) {
+// e4m3 heads: up to 32 (four accumulator columns per query).
+static int tc_group(int32_t batch, int32_t k, bool q8) {
+    if (q8 && batch <= 4) return 4;
     if (batch <= 8) return 8;
     if (batch <= 16) return 16;
-    if (batch <= 32 || k > vie::tc_max_k(64)) return 32;
+    if (q8 || batch <= 32 || k > vie::tc_max_k(64)) return 32;
     return 64;
 }
 
 static bool use_tc(const vie_head *head, int32_t batch, int32_t k) {
-    return head->tc_ready && batch >= knobs().tc_min_batch && k <= vie::tc_max_k(32) &&
-           head->d_pad >= 64;
+    const bool q8 = head->scale != nullptr;
+    return head->tc_ready && batch >= (q8 ? knobs().tc_min_batch_e4m3 : knobs().tc_min_batch) &&
+           k <= vie::tc_max_k(32, q8) && head->d_pad >= (q8 ? 128 : 64);
 }
 
 static vie_topk_plan make_plan(const vie_head *head, int32_t batch, int32_t k) {
     vie_topk_plan pl;
     if (use_tc(head, batch, k)) {
-        const int nqt = tc_group(batch, k);
+        const int nqt = tc_group(batch, k, head->scale != nullptr);
         pl.path = 1;
         pl.groups = (batch + nqt - 1) / nqt;
         pl.launches = 2 * pl.groups;  // hi/lo prep; projection, per-CTA top-k and merge
@@ -471,22 +498,33 @@ static vie_topk_plan make_plan(const vie_head *head, int32_t batch, int32_t k) {
 static vie_status run_topk_tc(const char *fn, vie_head *head, const float *h, int32_t batch,
                               int32_t k, int32_t *out_idx, float *out_logits, float *sparse,
                               cudaStream_t s) {
-    const int nqt = tc_group(batch, k);
-    int stages = 0;
+    const bool q8 = head->scale != nullptr;
+    const int nqt = tc_group(batch, k, q8);
+    // K-blocks per stage: the most that still leave a ring of two stages
+    // (larger stages beat deeper rings of small ones); the query boxes stay
+    // resident in shared memory when they are small (e4m3 rows)
+    int stages = 0, kps = 0;
     uint32_t smem = 0;
-    int kps = knobs().tc_kps;
-    kps = kps < 1 ? 1 : (kps > vie::kTcMaxKPS ? vie::kTcMaxKPS : kps);
-    while (kps > 1 && !vie::tc_shape(nqt, kps, &stages, &smem)) --kps;
-    if (!vie::tc_shape(nqt, kps, &stages, &smem))
-        return fail(VIE_ERR_UNSUPPORTED, "%s: no tensor-core layout", fn);
+    int kps_max = knobs().tc_kps;
+    kps_max = kps_max < 1 ? 1 : (kps_max > vie::kTcMaxKPS ? vie::kTcMaxKPS : kps_max);
+    const int n_kb = (head->d_pad + (q8 ? 127 : 63)) / (q8 ? 128 : 64);
+    const int hres_bytes = q8 ? vie::tc_hres_bytes(nqt, q8, n_kb) : 0;
+    for (int c = kps_max; c >= 1 && kps == 0; --c) {
+        if (vie::tc_shape(nqt, q8, c, hres_bytes, &stages, &smem)) kps = c;
+    }
+    if (kps == 0) return fail(VIE_ERR_UNSUPPORTED, "%s: no tensor-core layout", fn);
     const int n_tiles = static_cast<int>((head->V + vie::kTcTile - 1) / vie::kTcTile);
     int pct = knobs().static_pct;
     pct = pct < 0 ? 0 : (pct > 100 ? 100 : pct);
-    const CUtensorMap &mapH = head->mapH[nqt == 8 ? 0 : (nqt == 16 ? 1 : (nqt == 32 ? 2 : 3))];
+    const int n_h = (q8 ? vie::kQ8Pieces : 2) * nqt;  // query rows: boxes of 16 / 32 / 64 / 128
+    const CUtensorMap &mapH = head->mapH[n_h == 16 ? 0 : (n_h == 32 ? 1 : (n_h == 64 ? 2 : 3))];
     for (int q0 = 0; q0 < batch; q0 += nqt) {
         const int nq = batch - q0 < nqt ? batch - q0 : nqt;
-        cudaError_t e = vie::launch_prep_queries(h + static_cast<int64_t>(q0) * head->d, nq, head->d,
-                                                 head->d_pad, 2 * nqt, head->hB, head->num_sms, s);
+        const float *hq = h + static_cast<int64_t>(q0) * head->d;
+        cudaError_t e = q8 ? vie::launch_prep_queries_e4m3(hq, nq, nqt, head->d, head->d_pad, head->hB,
+                                                           head->qscale, s)
+                           : vie::launch_prep_queries(hq, nq, head->d, head->d_pad, 2 * nqt, head->hB,
+                                                      head->num_sms, s);
         if (e != cudaSuccess) return fail_cuda(e, fn);
         vie::TcParams p;
         p.V = head->V;
@@ -505,7 +543,10 @@ static vie_status run_topk_tc(const char *fn, vie_head *head, const float *h, in
         p.out_idx = out_idx + static_cast<int64_t>(q0) * k;
         p.out_logits = out_logits + static_cast<int64_t>(q0) * k;
         p.sparse = sparse != nullptr ? sparse + static_cast<int64_t>(q0) * head->V : nullptr;
-        e = vie::launch_tc_topk(nqt, head->mapW, mapH, p, head->G, smem, s);
+        p.row_scale = head->scale;
+        p.qscale = head->qscale;
+        p.h_resident = hres_bytes > 0 ? 1 : 0;
+        e = vie::launch_tc_topk(nqt, q8, head->mapW, mapH, p, head->G, smem, s);
         if (e != cudaSuccess) return fail_cuda(e, fn);
     }
     return VIE_OK;

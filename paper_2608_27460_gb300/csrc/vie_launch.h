@@ -37,9 +37,6 @@ cudaError_t launch_stream_topk_e4m3_nb8(int mm, int r, const StreamTopkParams &p
 // ---- tensor-core head (vie_tc_topk.cu) ----
 struct TcParams;
 
-// Ring depth and dynamic shared memory of the tensor-core kernel for query
-// groups of nq_tmpl (8, 16 or 32) and kps K-blocks per stage; false if
-// unsupported.
 // Recall@k: per query, how many exact top-k indices the candidates contain.
 cudaError_t launch_recall_hits(const int32_t *exact, int k, const int32_t *approx, int m, int64_t n,
                                int32_t *hits, cudaStream_t stream);
@@ -48,13 +45,27 @@ cudaError_t launch_sample_topk(const int32_t *idx, const float *logits, int batc
                                float top_p, float min_p, uint64_t seed, uint64_t step,
                                int32_t *out_token, float *out_prob, cudaStream_t stream);
 
-// Largest k the tensor-core kernel with nq_tmpl query slots handles.
-int tc_max_k(int nq_tmpl);
-bool tc_shape(int nq_tmpl, int kps, int *stages, uint32_t *smem);
+// Largest k the tensor-core kernel with nq_tmpl query slots handles (q8: on
+// e4m3 rows).
+int tc_max_k(int nq_tmpl, bool q8 = false);
+// Ring depth and dynamic shared memory for query groups of nq_tmpl (8, 16,
+// 32 or 64; 4, 8, 16 or 32 on e4m3 rows), kps K-blocks per stage and
+// hres_bytes of resident query boxes; false if unsupported.
+bool tc_shape(int nq_tmpl, bool q8, int kps, int hres_bytes, int *stages, uint32_t *smem);
+// Bytes of query boxes kept resident in shared memory for this group shape
+// and n_kb K-blocks (0: the boxes travel with every ring stage).
+int tc_hres_bytes(int nq_tmpl, bool q8, int n_kb);
 
-// Launches tc_topk_kernel<nq_tmpl>.
-cudaError_t launch_tc_topk(int nq_tmpl, const CUtensorMap &mapW, const CUtensorMap &mapH,
+// Launches tc_topk_kernel<nq_tmpl, q8>.
+cudaError_t launch_tc_topk(int nq_tmpl, bool q8, const CUtensorMap &mapW, const CUtensorMap &mapH,
                            const TcParams &p, int grid, uint32_t smem, cudaStream_t stream);
+cudaError_t launch_tc_topk_e4m3(int nq_tmpl, const CUtensorMap &mapW, const CUtensorMap &mapH,
+                                const TcParams &p, int grid, uint32_t smem, cudaStream_t stream);
+
+// e4m3 query pieces hQ [4 nq_tmpl][d_pad] and their scales [4 nq_tmpl] for
+// the tensor-core kernel on e4m3 rows (d_pad <= 24576).
+cudaError_t launch_prep_queries_e4m3(const float *h, int nq, int nq_tmpl, int d, int d_pad, void *hQ,
+                                     float *qscale, cudaStream_t stream);
 
 // hi/lo bf16 query matrix [n_rows][d_pad] for the tensor-core kernel.
 cudaError_t launch_prep_queries(const float *h, int nq, int d, int d_pad, int n_rows, void *hB,

@@ -2,10 +2,8 @@
 // the tcgen05 projection with per-CTA top-k and the merge in its last CTA.
 #include <cuda_bf16.h>
 
-#include <utility>
-
 #include "vie_launch.h"
-#include "vie_tc_topk.cuh"
+#include "vie_tc_launch.cuh"
 
 namespace vie {
 
@@ -25,66 +23,42 @@ __global__ void prep_queries_kernel(const float *__restrict__ h, int nq, int d, 
     }
 }
 
-namespace {
-
-// Launch with programmatic stream serialisation (the kernel calls
-// griddep_wait before it touches what the previous kernel wrote).
-template <typename... KArgs, typename... Args>
-cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, uint32_t smem,
-                       cudaStream_t stream, Args &&...args) {
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = grid;
-    cfg.blockDim = block;
-    cfg.dynamicSmemBytes = smem;
-    cfg.stream = stream;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[0].val.programmaticStreamSerializationAllowed = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, kern, std::forward<Args>(args)...);
+template <int NQ, bool Q8>
+void tc_sizes(int *score_bytes, int *buf_bytes, int *kb_w_bytes, int *kb_h_bytes) {
+    *score_bytes = TcShape<NQ, Q8>::kScoreBytes;
+    *buf_bytes = TcShape<NQ, Q8>::kBufBytes;
+    *kb_w_bytes = TcShape<NQ, Q8>::kStageA;
+    *kb_h_bytes = TcShape<NQ, Q8>::kStageB;
 }
 
-template <int NQ>
-cudaError_t launch_tc_one(const CUtensorMap &mapW, const CUtensorMap &mapH, const TcParams &p,
-                          int grid, uint32_t smem, cudaStream_t stream) {
-    static bool configured[64] = {};
-    int dev = 0;
-    cudaError_t e = cudaGetDevice(&dev);
-    if (e != cudaSuccess) return e;
-    if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
-    if (!configured[dev]) {
-        e = cudaFuncSetAttribute(tc_topk_kernel<NQ>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 232448);
-        if (e != cudaSuccess) return e;
-        configured[dev] = true;
-    }
-    return launch_pdl(tc_topk_kernel<NQ>, dim3(grid), dim3(TcShape<NQ>::kThreads), smem, stream, mapW,
-                      mapH, p);
-}
-
-template <int NQ>
-int tc_stage_bytes() {
-    return TcShape<NQ>::kStageBytes;
-}
-
-}  // namespace
-
-bool tc_shape(int nq_tmpl, int kps, int *stages, uint32_t *smem) {
-    int score_bytes = 0, buf_bytes = 0, stage_bytes = 0;
-    switch (nq_tmpl) {
-        case 8: score_bytes = TcShape<8>::kScoreBytes; buf_bytes = TcShape<8>::kBufBytes;
-                stage_bytes = TcShape<8>::kStageBytes; break;
-        case 16: score_bytes = TcShape<16>::kScoreBytes; buf_bytes = TcShape<16>::kBufBytes;
-                 stage_bytes = TcShape<16>::kStageBytes; break;
-        case 32: score_bytes = TcShape<32>::kScoreBytes; buf_bytes = TcShape<32>::kBufBytes;
-                 stage_bytes = TcShape<32>::kStageBytes; break;
-        case 64: score_bytes = TcShape<64>::kScoreBytes; buf_bytes = TcShape<64>::kBufBytes;
-                 stage_bytes = TcShape<64>::kStageBytes; break;
+bool tc_sizes_of(int nq_tmpl, bool q8, int *score_bytes, int *buf_bytes, int *kb_w, int *kb_h) {
+    switch (q8 ? -nq_tmpl : nq_tmpl) {
+        case 8: tc_sizes<8, false>(score_bytes, buf_bytes, kb_w, kb_h); return true;
+        case 16: tc_sizes<16, false>(score_bytes, buf_bytes, kb_w, kb_h); return true;
+        case 32: tc_sizes<32, false>(score_bytes, buf_bytes, kb_w, kb_h); return true;
+        case 64: tc_sizes<64, false>(score_bytes, buf_bytes, kb_w, kb_h); return true;
+        case -4: tc_sizes<4, true>(score_bytes, buf_bytes, kb_w, kb_h); return true;
+        case -8: tc_sizes<8, true>(score_bytes, buf_bytes, kb_w, kb_h); return true;
+        case -16: tc_sizes<16, true>(score_bytes, buf_bytes, kb_w, kb_h); return true;
+        case -32: tc_sizes<32, true>(score_bytes, buf_bytes, kb_w, kb_h); return true;
         default: return false;
     }
+}
+
+// The 4-query e4m3 tile keeps all of its query boxes in shared memory when
+// they take at most 48 KB (d_pad <= 3072): the ring then holds weights only.
+int tc_hres_bytes(int nq_tmpl, bool q8, int n_kb) {
+    if (!q8 || nq_tmpl != 4) return 0;
+    const int b = n_kb * TcShape<4, true>::kStageB;
+    return b <= 48 * 1024 ? b : 0;
+}
+
+bool tc_shape(int nq_tmpl, bool q8, int kps, int hres_bytes, int *stages, uint32_t *smem) {
+    int score_bytes = 0, buf_bytes = 0, kb_w = 0, kb_h = 0;
+    if (!tc_sizes_of(nq_tmpl, q8, &score_bytes, &buf_bytes, &kb_w, &kb_h)) return false;
+    const int stage_bytes = kps * (hres_bytes > 0 ? kb_w : kb_w + kb_h);
     for (int s = kTcMaxStages; s >= 2; --s) {
-        const TcSmemLayout L(score_bytes, buf_bytes, s, kps * stage_bytes);
+        const TcSmemLayout L(score_bytes, buf_bytes, s, stage_bytes, hres_bytes);
         if (L.total <= 232448u) {
             *stages = s;
             *smem = L.total;
@@ -94,23 +68,28 @@ bool tc_shape(int nq_tmpl, int kps, int *stages, uint32_t *smem) {
     return false;
 }
 
-int tc_max_k(int nq_tmpl) {
-    switch (nq_tmpl) {
+int tc_max_k(int nq_tmpl, bool q8) {
+    switch (q8 ? -nq_tmpl : nq_tmpl) {
         case 8: return TcShape<8>::kMaxK;
         case 16: return TcShape<16>::kMaxK;
         case 32: return TcShape<32>::kMaxK;
         case 64: return TcShape<64>::kMaxK;
+        case -4: return TcShape<4, true>::kMaxK;
+        case -8: return TcShape<8, true>::kMaxK;
+        case -16: return TcShape<16, true>::kMaxK;
+        case -32: return TcShape<32, true>::kMaxK;
         default: return 0;
     }
 }
 
-cudaError_t launch_tc_topk(int nq_tmpl, const CUtensorMap &mapW, const CUtensorMap &mapH,
+cudaError_t launch_tc_topk(int nq_tmpl, bool q8, const CUtensorMap &mapW, const CUtensorMap &mapH,
                            const TcParams &p, int grid, uint32_t smem, cudaStream_t stream) {
+    if (q8) return launch_tc_topk_e4m3(nq_tmpl, mapW, mapH, p, grid, smem, stream);
     switch (nq_tmpl) {
-        case 8: return launch_tc_one<8>(mapW, mapH, p, grid, smem, stream);
-        case 16: return launch_tc_one<16>(mapW, mapH, p, grid, smem, stream);
-        case 32: return launch_tc_one<32>(mapW, mapH, p, grid, smem, stream);
-        case 64: return launch_tc_one<64>(mapW, mapH, p, grid, smem, stream);
+        case 8: return launch_tc_one<8, false>(mapW, mapH, p, grid, smem, stream);
+        case 16: return launch_tc_one<16, false>(mapW, mapH, p, grid, smem, stream);
+        case 32: return launch_tc_one<32, false>(mapW, mapH, p, grid, smem, stream);
+        case 64: return launch_tc_one<64, false>(mapW, mapH, p, grid, smem, stream);
         default: return cudaErrorInvalidValue;
     }
 }

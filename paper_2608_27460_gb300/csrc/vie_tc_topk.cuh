@@ -25,6 +25,13 @@
 //                tau; one bitonic sort of the final k per query.
 // Each CTA writes its per-query lists and takes a completion ticket; the
 // last CTAs to finish merge them, one query each.  All waits are bounded.
+//
+// Q8 (e4m3 rows with one fp32 scale each, tcgen05 kind::f8f6f4): a K-block
+// is 128 codes (the same 128-byte swizzle row), and each query enters as four
+// e4m3 columns c_0..c_3 with power-of-two scales s_0..s_3 such that
+// h ~ sum_p s_p c_p (each piece takes 4 more significand bits of what the
+// previous left, so the residual is below 2^-16 |h| per term, as with the bf16
+// hi/lo split); the logit of row i is scale_i * sum_p s_p acc_p.
 #pragma once
 
 #include <cuda.h>
@@ -44,6 +51,7 @@ constexpr int kTcMaxK = 128;       // largest k of this path
 constexpr int kTcListKeys = 4096;  // keys of the per-CTA lists per CTA: NQ * k <= this
 constexpr int kTcMaxKPS = 4;       // K-blocks per stage, at most
 constexpr int kTcMergeE = 4;       // merge: keys per list in the heads area
+constexpr int kQ8Pieces = 4;       // e4m3 columns per query on the Q8 path
 constexpr int kTcMaxMergers = 64;  // CTAs that merge, at most (one per query)
 
 struct TcParams {
@@ -63,27 +71,34 @@ struct TcParams {
     int32_t *out_idx;        // [nq, k]
     float *out_logits;       // [nq, k]
     float *sparse;           // [nq, V] fp32 or nullptr: slices filled with -inf here
+    const float *row_scale;  // Q8: fp32 scale per row [V]
+    const float *qscale;     // Q8: [NQ][kQ8Pieces] power-of-two piece scales (from the prep kernel)
+    int32_t h_resident;      // 1: every K-block of the query matrix is loaded once, up front
 };
 
-template <int NQ>
+template <int NQ, bool Q8 = false>
 struct TcShape {
-    static constexpr int N = 2 * NQ;
+    static constexpr int kCols = Q8 ? kQ8Pieces : 2;  // accumulator columns per query
+    static constexpr int N = kCols * NQ;
+    static constexpr int kKB = Q8 ? 2 * kTcKBlock : kTcKBlock;  // elements per 128-byte K-block
     static constexpr int kQPW = NQ >= 64 ? 4 : (NQ >= 32 ? 2 : 1);  // queries per selector warp
     static constexpr int kSelWarps = NQ / kQPW;
     static constexpr int kWarps = 6 + kSelWarps;
     static constexpr int kThreads = 32 * kWarps;
-    static constexpr int kStageA = kTcTile * kTcKBlock * 2;  // 16 KB per K-block of W
-    static constexpr int kStageB = N * kTcKBlock * 2;        // N x 128 B per K-block of H
+    static constexpr int kStageA = kTcTile * 128;  // 16 KB per K-block of W (128 B per row)
+    static constexpr int kStageB = N * 128;        // N x 128 B per K-block of H
     static constexpr int kStageBytes = kStageA + kStageB;    // per K-block; a multiple of 1024
     static constexpr int kTmemCols = (2 * N <= 32) ? 32 : (2 * N <= 64 ? 64 : (2 * N <= 128 ? 128 : 256));
-    static constexpr int kSlots = NQ >= 64 ? 1 : (NQ >= 32 ? 2 : kTcScoreSlots);  // score ring depth
+    // score ring depth (e4m3 tiles: 2, leaving shared memory to the weight ring)
+    static constexpr int kSlots = NQ >= 64 ? 1 : ((NQ >= 32 || Q8) ? 2 : kTcScoreSlots);
     static constexpr int kScoreBytes = kSlots * NQ * kTcTile * 4;
     // candidate buffer per query: compacted to k whenever fewer than 32 slots
     // (one row block) are left, so k <= kCap - 32
     static constexpr int kCap = NQ >= 64 ? 128 : 256;
     static constexpr int kMaxK0 = kCap - 32 < kTcMaxK ? kCap - 32 : kTcMaxK;
     static constexpr int kMaxK = kMaxK0 < kTcListKeys / NQ ? kMaxK0 : kTcListKeys / NQ;  // largest k
-    static constexpr int kBufBytes = NQ * kCap * 8 + NQ * 12;  // buffers, counts, thresholds
+    // buffers, counts, thresholds (and the Q8 piece scales)
+    static constexpr int kBufBytes = NQ * kCap * 8 + NQ * 12 + (Q8 ? NQ * kQ8Pieces * 4 : 0);
 };
 
 struct TcMisc {
@@ -95,15 +110,18 @@ struct TcMisc {
     int merger;                    // m >= 0: this CTA merges queries m, m + X, ...
 };
 
+// The ring (1024-byte aligned at run time) starts with the resident query
+// boxes when there are any (hres_bytes, a multiple of 1024), then the stages.
 struct TcSmemLayout {
     uint32_t bars, misc, scores, bufs, ring, total;
-    __host__ __device__ TcSmemLayout(int score_bytes, int buf_bytes, int stages, int stage_bytes) {
+    __host__ __device__ TcSmemLayout(int score_bytes, int buf_bytes, int stages, int stage_bytes,
+                                     int hres_bytes = 0) {
         bars = 0;
         misc = 512;
         scores = 1024;
         bufs = scores + score_bytes;
         ring = (bufs + buf_bytes + 1023u) & ~1023u;
-        total = ring + stages * stage_bytes + 1024;  // +1024: room to align the ring
+        total = ring + hres_bytes + stages * stage_bytes + 1024;  // +1024: room to align the ring
     }
 };
 
@@ -215,12 +233,13 @@ static __device__ __noinline__ int keep_best(uint64_t *buf, int cnt, int k, uint
 
 // The final list of one query: the best min(k, cnt) keys of buf (cnt <=
 // 32 * CAP_PER), sorted descending, written to dst[0..k) (zeros after them),
-// and its first kTcMergeE keys also to head[0..kTcMergeE).
-template <int CAP_PER>
+// and its first kTcMergeE keys also to head[0..kTcMergeE).  The sort network
+// spans 32 * PER keys, the least that holds k (k <= 32 * PER): its dependent
+// shuffles are the tail of the launch.
+template <int CAP_PER, int PER>
 static __device__ __noinline__ void write_sorted_list(uint64_t *buf, int cnt, int k, uint64_t *tau,
                                                       uint64_t *dst, uint64_t *head, int lane) {
     if (cnt > k) cnt = keep_best<CAP_PER>(buf, cnt, k, tau, lane);
-    constexpr int PER = kTcMaxK / 32;  // cnt <= k <= kTcMaxK
     uint64_t v[PER];
 #pragma unroll
     for (int j = 0; j < PER; ++j) {
@@ -236,18 +255,24 @@ static __device__ __noinline__ void write_sorted_list(uint64_t *buf, int cnt, in
     }
 }
 
-template <int NQ>
-__global__ void __launch_bounds__(TcShape<NQ>::kThreads, 1)
+template <int NQ, bool Q8>
+__global__ void __launch_bounds__(TcShape<NQ, Q8>::kThreads, 1)
     tc_topk_kernel(const __grid_constant__ CUtensorMap mapW, const __grid_constant__ CUtensorMap mapH,
                    const TcParams p) {
-    using Sh = TcShape<NQ>;
+    using Sh = TcShape<NQ, Q8>;
     constexpr int N = Sh::N;
+    constexpr int KB = Sh::kKB;
     extern __shared__ __align__(1024) unsigned char tc_smem[];
     unsigned char *smem = tc_smem;
     const int S = p.stages;
     const int KPS = p.kb_per_stage;
-    const int stage_bytes = KPS * Sh::kStageBytes;  // [KPS boxes of W][KPS boxes of H]
-    const TcSmemLayout L(Sh::kScoreBytes, Sh::kBufBytes, S, stage_bytes);
+    const bool hres = p.h_resident != 0;
+    const int n_kb = (p.d_pad + KB - 1) / KB;
+    // a stage: [KPS boxes of W][KPS boxes of H], or W only when H is resident
+    const int kb_bytes = hres ? Sh::kStageA : Sh::kStageBytes;
+    const int stage_bytes = KPS * kb_bytes;
+    const int hres_bytes = hres ? n_kb * Sh::kStageB : 0;
+    const TcSmemLayout L(Sh::kScoreBytes, Sh::kBufBytes, S, stage_bytes, hres_bytes);
     uint64_t *full = reinterpret_cast<uint64_t *>(smem + L.bars);
     uint64_t *empty = full + kTcMaxStages;
     uint64_t *tfull = empty + kTcMaxStages;
@@ -255,17 +280,19 @@ __global__ void __launch_bounds__(TcShape<NQ>::kThreads, 1)
     uint64_t *sfull = tempty + 2;
     uint64_t *sempty = sfull + kTcScoreSlots;
     uint64_t *final_bar = sempty + kTcScoreSlots;
+    uint64_t *hbar = final_bar + 1;  // the resident query boxes have landed
     TcMisc *mc = reinterpret_cast<TcMisc *>(smem + L.misc);
     float *scores = reinterpret_cast<float *>(smem + L.scores);
     uint64_t *bufs = reinterpret_cast<uint64_t *>(smem + L.bufs);
     // the 128-byte swizzle needs 1024-byte aligned tiles in the shared window
     unsigned char *ring = smem + L.ring;
     ring += (1024u - (smem_addr(ring) & 1023u)) & 1023u;
+    unsigned char *hq_res = ring;  // [n_kb][N rows x 128 B] when H is resident
+    ring += hres_bytes;
     volatile int *abort_flag = &mc->abort;
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int G = gridDim.x, cta = blockIdx.x;
-    const int n_kb = (p.d_pad + kTcKBlock - 1) / kTcKBlock;
     const int n_st = (n_kb + KPS - 1) / KPS;  // stages per tile
     const int n_tiles = static_cast<int>((p.V + kTcTile - 1) / kTcTile);
 
@@ -283,6 +310,7 @@ __global__ void __launch_bounds__(TcShape<NQ>::kThreads, 1)
             mbar_init(&sempty[s], Sh::kSelWarps);
         }
         mbar_init(final_bar, 1);
+        mbar_init(hbar, 1);
         mc->abort = 0;
         fence_mbar_init();
     }
@@ -329,15 +357,23 @@ __global__ void __launch_bounds__(TcShape<NQ>::kThreads, 1)
                         break;
                     }
                     const int kb0 = st_i * KPS, nin = min(KPS, n_kb - kb0);
-                    mbar_arrive_expect_tx(&full[s], nin * Sh::kStageBytes);
+                    mbar_arrive_expect_tx(&full[s], nin * kb_bytes);
                     unsigned char *st = ring + s * stage_bytes;
                     for (int i = 0; i < nin; ++i)
-                        tma_load_2d(st + i * Sh::kStageA, &mapW, (kb0 + i) * kTcKBlock, tile * kTcTile,
+                        tma_load_2d(st + i * Sh::kStageA, &mapW, (kb0 + i) * KB, tile * kTcTile,
                                     &full[s], pol);
-                    if (it == 0) griddep_wait();  // the hi/lo query matrix comes from the prep kernel
-                    for (int i = 0; i < nin; ++i)
-                        tma_load_2d(st + KPS * Sh::kStageA + i * Sh::kStageB, &mapH,
-                                    (kb0 + i) * kTcKBlock, 0, &full[s], pol);
+                    if (it == 0) {
+                        griddep_wait();  // the query matrix comes from the prep kernel
+                        if (hres) {
+                            mbar_arrive_expect_tx(hbar, hres_bytes);
+                            for (int kb = 0; kb < n_kb; ++kb)
+                                tma_load_2d(hq_res + kb * Sh::kStageB, &mapH, kb * KB, 0, hbar, pol);
+                        }
+                    }
+                    if (!hres)
+                        for (int i = 0; i < nin; ++i)
+                            tma_load_2d(st + KPS * Sh::kStageA + i * Sh::kStageB, &mapH,
+                                        (kb0 + i) * KB, 0, &full[s], pol);
                     issued = it + 1;
                 }
                 if (tile < 0) break;
@@ -348,14 +384,16 @@ __global__ void __launch_bounds__(TcShape<NQ>::kThreads, 1)
                 const int never = 0;
                 for (int t2 = max(0, issued - S); t2 < issued; ++t2)
                     mbar_wait(&full[t2 % S], (t2 / S) & 1, const_cast<volatile int *>(&never));
+                if (hres && issued > 0) mbar_wait(hbar, 0, const_cast<volatile int *>(&never));
             }
         }
     } else if (warp == 1) {
         // ---------------- MMA issuer ----------------
         if (lane == 0) {
-            constexpr uint32_t idesc = umma_idesc_bf16_f32(kTcTile, N);
+            constexpr uint32_t idesc = Q8 ? umma_idesc_e4m3_f32(kTcTile, N) : umma_idesc_bf16_f32(kTcTile, N);
             int it = 0;
             bool ok = true;
+            bool h_ready = !hres;
             for (int ti = 0; ok; ++ti) {
                 const int b = ti & 1, ub = ti >> 1;
                 const int s0 = it % S, u0 = it / S;
@@ -383,16 +421,27 @@ __global__ void __launch_bounds__(TcShape<NQ>::kThreads, 1)
                         ok = false;
                         break;
                     }
+                    if (!h_ready) {
+                        if (!mbar_wait(hbar, 0, abort_flag)) {
+                            ok = false;
+                            break;
+                        }
+                        h_ready = true;
+                    }
                     tc_fence_after_sync();
                     unsigned char *st = ring + s * stage_bytes;
                     const int kb0 = st_i * KPS, nin = min(KPS, n_kb - kb0);
                     for (int i = 0; i < nin; ++i) {
                         const uint64_t ad = umma_desc_k_sw128(st + i * Sh::kStageA);
-                        const uint64_t bd = umma_desc_k_sw128(st + KPS * Sh::kStageA + i * Sh::kStageB);
+                        const uint64_t bd = umma_desc_k_sw128(
+                            hres ? hq_res + (kb0 + i) * Sh::kStageB : st + KPS * Sh::kStageA + i * Sh::kStageB);
 #pragma unroll
-                        for (int k4 = 0; k4 < kTcKBlock / 16; ++k4)  // +32 bytes per K step of 16
-                            umma_bf16(d, ad + 2 * k4, bd + 2 * k4, idesc,
-                                      ((kb0 + i) | k4) != 0 ? 1u : 0u);
+                        for (int k4 = 0; k4 < 4; ++k4) {  // +32 bytes per MMA (K = 16 bf16 or 32 e4m3)
+                            if constexpr (Q8)
+                                umma_e4m3(d, ad + 2 * k4, bd + 2 * k4, idesc, ((kb0 + i) | k4) != 0 ? 1u : 0u);
+                            else
+                                umma_bf16(d, ad + 2 * k4, bd + 2 * k4, idesc, ((kb0 + i) | k4) != 0 ? 1u : 0u);
+                        }
                     }
                     umma_commit(&empty[s]);
                 }
@@ -413,6 +462,14 @@ __global__ void __launch_bounds__(TcShape<NQ>::kThreads, 1)
         // ---------------- epilogue: TMEM -> logits ----------------
         const int qw = warp & 3;  // TMEM lane quarter this warp may access
         const int row = 32 * qw + lane;
+        // Q8: the piece scales of the queries, next to the selectors' counts
+        float *qs = reinterpret_cast<float *>(bufs + NQ * Sh::kCap) + 3 * NQ;
+        if constexpr (Q8) {
+            griddep_wait();  // the prep kernel wrote them
+            const int e = (warp - 2) * 32 + lane;
+            if (e < NQ * kQ8Pieces) qs[e] = p.qscale[e];
+            named_barrier_sync(2, 128);  // the four epilogue warps
+        }
         for (int ti = 0;; ++ti) {
             const int b = ti & 1, ub = ti >> 1;
             if (!mbar_wait(&tfull[b], ub & 1, abort_flag)) {
@@ -425,6 +482,12 @@ __global__ void __launch_bounds__(TcShape<NQ>::kThreads, 1)
             tc_fence_after_sync();
             const int tile = mc->buf_tile[b];
             const int ss = ti % Sh::kSlots, su = ti / Sh::kSlots;
+            // Q8: this row's scale, loaded under the accumulator reads
+            float rsc = 1.0f;
+            if constexpr (Q8) {
+                const int64_t gr = static_cast<int64_t>(tile) * kTcTile + row;
+                if (tile >= 0 && gr < p.V) rsc = __ldg(p.row_scale + gr);
+            }
             if constexpr (N > 64) {
                 // wide tiles: wait for the score slot first, then drain the
                 // accumulator 32 columns (16 queries) at a time
@@ -438,6 +501,7 @@ __global__ void __launch_bounds__(TcShape<NQ>::kThreads, 1)
                 if (tile >= 0) {
                     const uint32_t tb = tmem + (static_cast<uint32_t>(32 * qw) << 16) + b * N;
                     float *sc = scores + ss * NQ * kTcTile;
+                    constexpr int QC = 32 / Sh::kCols;  // queries per 32 accumulator columns
 #pragma unroll
                     for (int c = 0; c < N / 16; c += 2) {
                         uint32_t r[2][16];
@@ -445,9 +509,21 @@ __global__ void __launch_bounds__(TcShape<NQ>::kThreads, 1)
                         tmem_ld_32x32b_x16(tb + 16 * (c + 1), r[1]);
                         tmem_wait_ld();
 #pragma unroll
-                        for (int qq = 0; qq < 16; ++qq)
-                            sc[(8 * c + qq) * kTcTile + row] = __uint_as_float(r[qq / 8][(2 * qq) % 16]) +
-                                                               __uint_as_float(r[qq / 8][(2 * qq) % 16 + 1]);
+                        for (int qq = 0; qq < QC; ++qq) {
+                            const int q = QC * (c / 2) + qq, c0 = Sh::kCols * qq;
+                            float z;
+                            if constexpr (Q8) {
+                                z = 0.0f;
+#pragma unroll
+                                for (int pc = 0; pc < kQ8Pieces; ++pc)
+                                    z = fmaf(qs[kQ8Pieces * q + pc],
+                                             __uint_as_float(r[(c0 + pc) / 16][(c0 + pc) % 16]), z);
+                                z *= rsc;
+                            } else {
+                                z = __uint_as_float(r[c0 / 16][c0 % 16]) + __uint_as_float(r[c0 / 16][c0 % 16 + 1]);
+                            }
+                            sc[q * kTcTile + row] = z;
+                        }
                     }
                 }
                 tc_fence_before_sync();
@@ -467,9 +543,18 @@ __global__ void __launch_bounds__(TcShape<NQ>::kThreads, 1)
                 for (int c = 0; c < N / 16; ++c) tmem_ld_32x32b_x16(tb + 16 * c, r[c]);
                 tmem_wait_ld();
 #pragma unroll
-                for (int q = 0; q < NQ; ++q)
-                    lg[q] = __uint_as_float(r[q / 8][(2 * q) % 16]) +
-                            __uint_as_float(r[q / 8][(2 * q) % 16 + 1]);
+                for (int q = 0; q < NQ; ++q) {
+                    const int c0 = Sh::kCols * q;
+                    if constexpr (Q8) {
+                        float z = 0.0f;
+#pragma unroll
+                        for (int pc = 0; pc < kQ8Pieces; ++pc)
+                            z = fmaf(qs[kQ8Pieces * q + pc], __uint_as_float(r[(c0 + pc) / 16][(c0 + pc) % 16]), z);
+                        lg[q] = z * rsc;
+                    } else {
+                        lg[q] = __uint_as_float(r[c0 / 16][c0 % 16]) + __uint_as_float(r[c0 / 16][c0 % 16 + 1]);
+                    }
+                }
             }
             tc_fence_before_sync();
             __syncwarp();
@@ -573,10 +658,17 @@ __global__ void __launch_bounds__(TcShape<NQ>::kThreads, 1)
         int *cnt_all = reinterpret_cast<int *>(bufs + NQ * CAP);
         uint64_t *tau_all = reinterpret_cast<uint64_t *>(bufs + NQ * CAP) + NQ / 2;
 #pragma unroll 1
-        for (int q = warp; q < p.nq; q += Sh::kWarps)
-            write_sorted_list<CAP_PER>(bufs + q * CAP, cnt_all[q], p.k, &tau_all[q],
-                                       p.cand + (static_cast<size_t>(q) * G + cta) * p.k,
-                                       p.heads + (static_cast<size_t>(q) * G + cta) * kTcMergeE, lane);
+        for (int q = warp; q < p.nq; q += Sh::kWarps) {
+            uint64_t *dst = p.cand + (static_cast<size_t>(q) * G + cta) * p.k;
+            uint64_t *head = p.heads + (static_cast<size_t>(q) * G + cta) * kTcMergeE;
+            if (p.k <= 32)
+                write_sorted_list<CAP_PER, 1>(bufs + q * CAP, cnt_all[q], p.k, &tau_all[q], dst, head, lane);
+            else if (p.k <= 64)
+                write_sorted_list<CAP_PER, 2>(bufs + q * CAP, cnt_all[q], p.k, &tau_all[q], dst, head, lane);
+            else
+                write_sorted_list<CAP_PER, kTcMaxK / 32>(bufs + q * CAP, cnt_all[q], p.k, &tau_all[q], dst,
+                                                         head, lane);
+        }
     }
     __syncthreads();
 

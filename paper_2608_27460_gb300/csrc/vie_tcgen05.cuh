@@ -50,6 +50,27 @@ __host__ __device__ constexpr uint32_t umma_idesc_bf16_f32(int M, int N) {
            | (static_cast<uint32_t>(M >> 4) << 24);    // M / 16
 }
 
+// Instruction descriptor of tcgen05.mma.kind::f8f6f4: fp32 accumulator,
+// e4m3 A and B (format code 0 for both), both K-major, shape M x N.
+__host__ __device__ constexpr uint32_t umma_idesc_e4m3_f32(int M, int N) {
+    return (1u << 4)                                   // D: f32
+           | (0u << 7)                                 // A: e4m3
+           | (0u << 10)                                // B: e4m3
+           | (static_cast<uint32_t>(N >> 3) << 17)     // N / 8
+           | (static_cast<uint32_t>(M >> 4) << 24);    // M / 16
+}
+
+// D[tmem] (+)= A[smem] * B[smem]^T with 8-bit float operands (K = 32 per
+// instruction: the same 32 bytes of each row as a bf16 step of K = 16).
+__device__ __forceinline__ void umma_e4m3(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc,
+                                          uint32_t idesc, uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+
 // D[tmem] (+)= A[smem] * B[smem]^T, issued by one thread.
 __device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc,
                                           uint32_t idesc, uint32_t accumulate) {

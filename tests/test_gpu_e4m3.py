@@ -1,7 +1,9 @@
 """GPU parity of the e4m3-quantised head (vie_head_create_e4m3): the
 device quantiser gives the oracle's codes and scales bit for bit, and every
 top-k call on the handle matches the oracle's head on those codes
-(z_i = scale_i * sum_j e4m3(q_ij) h_j) under the usual acceptance rule."""
+(z_i = scale_i * sum_j e4m3(q_ij) h_j) under the usual acceptance rule, on
+the tensor-core path (kind::f8f6f4, queries split into four e4m3 pieces) and
+on the streaming CUDA-core kernel."""
 import numpy as np
 import pytest
 
@@ -28,7 +30,10 @@ def test_quantiser_is_bit_exact(vie, V, d):
         np.testing.assert_array_equal(scales.cpu().numpy().view(np.uint32), osc.view(np.uint32))
         p = head.props
         assert p.d_pad == (d + 15) // 16 * 16 and p.weight_bytes == V * p.d_pad + V * 4
-        assert head.plan(16, 50).path == 0  # e4m3 heads stay on the streaming kernel
+        # the tensor-core path takes e4m3 rows of at least 128 codes, k <= 128
+        assert head.plan(16, 50).path == (1 if p.d_pad >= 128 else 0)
+        assert head.plan(1, 50).path == (1 if p.d_pad >= 128 else 0)
+        assert head.plan(4, 129).path == 0
 
 
 def _parity(vie, W, h, k, reps=1):
@@ -54,6 +59,10 @@ def _parity(vie, W, h, k, reps=1):
 
 @pytest.mark.parametrize("V,d,batch,k", [
     (20011, 640, 1, 50),
+    (20011, 640, 9, 128),    # 16-query group at the path's largest k
+    (30011, 1024, 32, 50),   # full 32-query group
+    (30011, 2048, 45, 7),    # two groups: 32 + 13
+    (10007, 200, 2, 50),     # d_pad 208: a partial last K-block of 128 codes
     (20011, 1024, 1, 50),
     (4099, 100, 3, 50),      # padded rows
     (33333, 2048, 4, 1),
@@ -134,3 +143,48 @@ def test_one_hot_queries_give_exact_products(vie, hval):
         np.testing.assert_array_equal(val[r].view(np.uint32), want.view(np.uint32))
         assert not check_topk(idx[r], val[r], z[r], k)
 
+
+@pytest.mark.parametrize("batch", [1, 16, 32])
+def test_tensor_core_error_against_the_sum_of_magnitudes(vie, batch):
+    """The four-piece split keeps each h_j to within 2^-16 |h_j|, the products
+    are exact and the accumulation is fp32, so a returned logit is within a
+    small multiple of 2^-16 of scale_i * sum_j |e4m3(q_ij)| |h_j| from the
+    oracle's value."""
+    import torch
+    V, d, k = 30011, 1024, 128
+    W, h = workload(V, d, batch, seed=57 + batch)
+    q, sc = oracle.quantize_e4m3(W)
+    z = oracle.logits_e4m3(q, sc, h)
+    mag = oracle.logits_e4m3(q & 0x7F, sc, np.abs(h))
+    with _head(vie, W) as head:
+        assert head.plan(batch, k).path == 1
+        idx, val = head.topk(torch.from_numpy(h).cuda(), k)
+        torch.cuda.synchronize()
+        assert head.device_status() == vie.VIE_OK
+    idx, val = idx.cpu().numpy(), val.cpu().numpy()
+    rel = np.array([np.abs(val[b] - z[b][idx[b]]) / mag[b][idx[b]] for b in range(batch)])
+    print(f"batch {batch}: largest error / sum of magnitudes = 2^{np.log2(rel.max()):.2f}")
+    assert rel.max() <= 2.0**-14
+
+
+def test_streaming_kernel_on_e4m3_rows():
+    """The same parity with every call forced onto the streaming CUDA-core
+    kernel (a fresh process: the path threshold is read once per process)."""
+    import os
+    import subprocess
+    import sys
+    here = os.path.dirname(os.path.abspath(__file__))
+    code = (
+        "import sys; sys.path[:0] = [%r, %r]\n"
+        "import test_gpu_e4m3 as t, paper_2608_27460_gb300 as vie\n"
+        "from gpu_cases import workload\n"
+        "vie.load()\n"
+        "for V, d, b, k in [(20011, 640, 1, 50), (30011, 1024, 8, 64), (20011, 2048, 3, 1)]:\n"
+        "    W, h = workload(V, d, b, seed=V + b)\n"
+        "    with t._head(vie, W) as head:\n"
+        "        assert head.plan(b, k).path == 0\n"
+        "    t._parity(vie, W, h, k, reps=2)\n"
+        "print('ok')\n") % (here, os.path.dirname(here))
+    env = dict(os.environ, VIE_TC_MIN_BATCH_E4M3="100000")
+    r = subprocess.run([sys.executable, "-c", code], env=env, capture_output=True, text=True, timeout=600)
+    assert r.returncode == 0 and r.stdout.strip().endswith("ok"), r.stdout + r.stderr
