@@ -477,13 +477,23 @@ static bool use_tc(const vie_head *head, int32_t batch, int32_t k) {
            k <= vie::tc_max_k(32, q8) && head->d_pad >= (q8 ? 128 : 64);
 }
 
+// Bytes of the query operand each CTA of a group of nqt slots builds itself
+// (0: a prep kernel writes it).
+static int tc_hres(const vie_head *head, int nqt) {
+    const bool q8 = head->scale != nullptr;
+    const int n_kb = (head->d_pad + (q8 ? 127 : 63)) / (q8 ? 128 : 64);
+    return vie::tc_hres_bytes(nqt, q8, n_kb);
+}
+
 static vie_topk_plan make_plan(const vie_head *head, int32_t batch, int32_t k) {
     vie_topk_plan pl;
     if (use_tc(head, batch, k)) {
         const int nqt = tc_group(batch, k, head->scale != nullptr);
         pl.path = 1;
         pl.groups = (batch + nqt - 1) / nqt;
-        pl.launches = 2 * pl.groups;  // hi/lo prep; projection, per-CTA top-k and merge
+        // per group: the query prep (unless the CTAs build the operand), then
+        // projection, per-CTA top-k and merge in one launch
+        pl.launches = (tc_hres(head, nqt) > 0 ? 1 : 2) * pl.groups;
     } else {
         const int cap = nb_cap_for(head->d_pad, pick_mm(k));
         pl.path = 0;
@@ -507,8 +517,7 @@ static vie_status run_topk_tc(const char *fn, vie_head *head, const float *h, in
     uint32_t smem = 0;
     int kps_max = knobs().tc_kps;
     kps_max = kps_max < 1 ? 1 : (kps_max > vie::kTcMaxKPS ? vie::kTcMaxKPS : kps_max);
-    const int n_kb = (head->d_pad + (q8 ? 127 : 63)) / (q8 ? 128 : 64);
-    const int hres_bytes = q8 ? vie::tc_hres_bytes(nqt, q8, n_kb) : 0;
+    const int hres_bytes = tc_hres(head, nqt);
     for (int c = kps_max; c >= 1 && kps == 0; --c) {
         if (vie::tc_shape(nqt, q8, c, hres_bytes, &stages, &smem)) kps = c;
     }
@@ -521,10 +530,10 @@ static vie_status run_topk_tc(const char *fn, vie_head *head, const float *h, in
     for (int q0 = 0; q0 < batch; q0 += nqt) {
         const int nq = batch - q0 < nqt ? batch - q0 : nqt;
         const float *hq = h + static_cast<int64_t>(q0) * head->d;
-        cudaError_t e = q8 ? vie::launch_prep_queries_e4m3(hq, nq, nqt, head->d, head->d_pad, head->hB,
-                                                           head->qscale, s)
-                           : vie::launch_prep_queries(hq, nq, head->d, head->d_pad, 2 * nqt, head->hB,
-                                                      head->num_sms, s);
+        cudaError_t e = cudaSuccess;
+        if (hres_bytes == 0)
+            e = q8 ? vie::launch_prep_queries_e4m3(hq, nq, nqt, head->d, head->d_pad, head->hB, head->qscale, s)
+                   : vie::launch_prep_queries(hq, nq, head->d, head->d_pad, 2 * nqt, head->hB, head->num_sms, s);
         if (e != cudaSuccess) return fail_cuda(e, fn);
         vie::TcParams p;
         p.V = head->V;
@@ -546,6 +555,8 @@ static vie_status run_topk_tc(const char *fn, vie_head *head, const float *h, in
         p.row_scale = head->scale;
         p.qscale = head->qscale;
         p.h_resident = hres_bytes > 0 ? 1 : 0;
+        p.h = hq;
+        p.d = head->d;
         e = vie::launch_tc_topk(nqt, q8, head->mapW, mapH, p, head->G, smem, s);
         if (e != cudaSuccess) return fail_cuda(e, fn);
     }

@@ -52,8 +52,9 @@ int tc_max_k(int nq_tmpl, bool q8 = false);
 // 32 or 64; 4, 8, 16 or 32 on e4m3 rows), kps K-blocks per stage and
 // hres_bytes of resident query boxes; false if unsupported.
 bool tc_shape(int nq_tmpl, bool q8, int kps, int hres_bytes, int *stages, uint32_t *smem);
-// Bytes of query boxes kept resident in shared memory for this group shape
-// and n_kb K-blocks (0: the boxes travel with every ring stage).
+// Bytes of the query operand each CTA builds in shared memory itself for this
+// group shape and n_kb K-blocks (0: a prep kernel writes it and its boxes
+// travel with every ring stage).
 int tc_hres_bytes(int nq_tmpl, bool q8, int n_kb);
 
 // Launches tc_topk_kernel<nq_tmpl, q8>.

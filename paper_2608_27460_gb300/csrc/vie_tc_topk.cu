@@ -45,8 +45,9 @@ bool tc_sizes_of(int nq_tmpl, bool q8, int *score_bytes, int *buf_bytes, int *kb
     }
 }
 
-// The 4-query e4m3 tile keeps all of its query boxes in shared memory when
-// they take at most 48 KB (d_pad <= 3072): the ring then holds weights only.
+// The 4-query e4m3 tile builds its whole query operand in shared memory (no
+// prep kernel; the ring holds weights only) when it takes at most 48 KB of
+// pieces (d_pad <= 3072).
 int tc_hres_bytes(int nq_tmpl, bool q8, int n_kb) {
     if (!q8 || nq_tmpl != 4) return 0;
     const int b = n_kb * TcShape<4, true>::kStageB;

@@ -32,9 +32,18 @@
 // h ~ sum_p s_p c_p (each piece takes 4 more significand bits of what the
 // previous left, so the residual is below 2^-16 |h| per term, as with the bf16
 // hi/lo split); the logit of row i is scale_i * sum_p s_p acc_p.
+//
+// Small e4m3 groups (h_resident): every CTA builds the whole query operand
+// (the four e4m3 pieces of each query) itself, straight into shared memory in
+// the 128-byte-swizzled K-major layout the MMA reads, so the call needs no
+// separate query-prep kernel and the ring carries weights only.  (For the
+// 8-query bf16 tile the same build measured slower than the prep kernel.)
 #pragma once
 
 #include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+#include <cuda_fp8.h>
 #include <cstdint>
 
 #include "vie_stream_topk.cuh"
@@ -73,7 +82,9 @@ struct TcParams {
     float *sparse;           // [nq, V] fp32 or nullptr: slices filled with -inf here
     const float *row_scale;  // Q8: fp32 scale per row [V]
     const float *qscale;     // Q8: [NQ][kQ8Pieces] power-of-two piece scales (from the prep kernel)
-    int32_t h_resident;      // 1: every K-block of the query matrix is loaded once, up front
+    int32_t h_resident;      // 1: each CTA builds the whole query operand in shared memory itself
+    const float *h;          // h_resident: the queries [nq, d] fp32
+    int32_t d;               // h_resident: their length
 };
 
 template <int NQ, bool Q8 = false>
@@ -124,6 +135,25 @@ struct TcSmemLayout {
         total = ring + hres_bytes + stages * stage_bytes + 1024;  // +1024: room to align the ring
     }
 };
+
+// The least power of two >= v for v >= 0, at least 2^-100 (so that the
+// piece scales s_0 2^-4p and their reciprocals stay normal fp32 numbers):
+// exact bit arithmetic on the fp32 encoding.
+__device__ __forceinline__ float pow2_at_least(float v) {
+    const uint32_t b = __float_as_uint(v);
+    if (b <= 0x0D800000u) return 0x1p-100f;  // zero, or at most 2^-100
+    if ((b & 0x007FFFFFu) == 0) return v;   // already a power of two
+    return __uint_as_float((b & 0x7F800000u) + 0x00800000u);
+}
+
+// x rounded to the nearest e4m3 value (ties to even, saturated at +-448),
+// and an e4m3 code's exact value.
+__device__ __forceinline__ uint8_t e4m3_code(float x) {
+    return static_cast<uint8_t>(__nv_cvt_float_to_fp8(x, __NV_SATFINITE, __NV_E4M3));
+}
+__device__ __forceinline__ float e4m3_value(uint8_t c) {
+    return __half2float(__half(__nv_cvt_fp8_to_halfraw(static_cast<__nv_fp8_storage_t>(c), __NV_E4M3)));
+}
 
 __device__ __forceinline__ uint64_t shfl_xor_u64(uint64_t v, int m) {
     const uint32_t lo = __shfl_xor_sync(0xFFFFFFFFu, static_cast<uint32_t>(v), m);
@@ -280,7 +310,6 @@ __global__ void __launch_bounds__(TcShape<NQ, Q8>::kThreads, 1)
     uint64_t *sfull = tempty + 2;
     uint64_t *sempty = sfull + kTcScoreSlots;
     uint64_t *final_bar = sempty + kTcScoreSlots;
-    uint64_t *hbar = final_bar + 1;  // the resident query boxes have landed
     TcMisc *mc = reinterpret_cast<TcMisc *>(smem + L.misc);
     float *scores = reinterpret_cast<float *>(smem + L.scores);
     uint64_t *bufs = reinterpret_cast<uint64_t *>(smem + L.bufs);
@@ -310,7 +339,6 @@ __global__ void __launch_bounds__(TcShape<NQ, Q8>::kThreads, 1)
             mbar_init(&sempty[s], Sh::kSelWarps);
         }
         mbar_init(final_bar, 1);
-        mbar_init(hbar, 1);
         mc->abort = 0;
         fence_mbar_init();
     }
@@ -322,7 +350,81 @@ __global__ void __launch_bounds__(TcShape<NQ, Q8>::kThreads, 1)
     __syncthreads();
     tc_fence_after_sync();
     const uint32_t tmem = mc->tmem_base;
-    if (tid == 0) griddep_launch_dependents();  // the merge kernel may be scheduled
+    if (tid == 0) griddep_launch_dependents();  // a kernel launched after this one may be scheduled
+    // Q8: the piece scales of the queries, next to the selectors' counts
+    float *qs = reinterpret_cast<float *>(bufs + NQ * Sh::kCap) + 3 * NQ;
+
+    if (Q8 && hres && warp > 0) {
+        // ---------------- the query operand, built in shared memory ----------------
+        // Row r of a K-block is 128 bytes; 8-row groups are 1024 bytes apart;
+        // the 16-byte chunk c of row r sits at chunk c ^ (r % 8) (the 128-byte
+        // swizzle TMA would apply).  Columns past d are zero.
+        griddep_wait();  // h comes from the kernel before this one
+        const int T = Sh::kThreads - 32, t = tid - 32;
+        const int width = n_kb * KB;  // columns of the operand, K-block padded
+        auto at = [&](int r, int byte_in_row, int kb) -> unsigned char * {
+            const int c = byte_in_row >> 4;
+            return hq_res + kb * Sh::kStageB + (r >> 3) * 1024 + (r & 7) * 128 +
+                   (((c ^ (r & 7)) << 4) | (byte_in_row & 15));
+        };
+        // rows of absent queries: zero, 16 bytes at a time (a row is 128 B in
+        // every K-block; the swizzle only permutes chunks within a row)
+        const int r_real = Sh::kCols * p.nq;
+        for (int e = t; e < n_kb * (N - r_real) * 8; e += T) {
+            const int kb = e / ((N - r_real) * 8), rem = e - kb * (N - r_real) * 8;
+            const int r = r_real + (rem >> 3);
+            *reinterpret_cast<uint4 *>(hq_res + kb * Sh::kStageB + (r >> 3) * 1024 + (r & 7) * 128 +
+                                       ((rem & 7) << 4)) = make_uint4(0u, 0u, 0u, 0u);
+        }
+        constexpr int U = 8;  // independent loads of h in flight per thread
+        {
+            // s_0 = the least power of two >= max_j |h_qj| / 448, s_p = s_0 2^-4p:
+            // every residual then stays within the pieces' range (448, 256, 128,
+            // 64) and each piece takes 4 more significand bits
+            const int q = warp - 1;
+            if (q < p.nq) {
+                float m = 0.0f;
+                for (int j = lane; j < p.d; j += 32) m = fmaxf(m, fabsf(p.h[static_cast<int64_t>(q) * p.d + j]));
+#pragma unroll
+                for (int o = 16; o >= 1; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xFFFFFFFFu, m, o));
+                const float s0 = pow2_at_least(m / 448.0f);
+                if (lane < kQ8Pieces) qs[kQ8Pieces * q + lane] = s0 * __uint_as_float((127u - 4u * lane) << 23);
+            } else if (q < NQ && lane < kQ8Pieces) {
+                qs[kQ8Pieces * q + lane] = 0.0f;
+            }
+            named_barrier_sync(3, T);
+            for (int q = 0; q < p.nq; ++q) {
+                const float *hq = p.h + static_cast<int64_t>(q) * p.d;
+                // 1 / s_p is exact: s_p is a power of two within fp32's normal range
+                const float inv0 = 1.0f / qs[kQ8Pieces * q], s0 = qs[kQ8Pieces * q];
+                for (int j0 = t; j0 < width; j0 += U * T) {
+                    float x[U];
+#pragma unroll
+                    for (int u = 0; u < U; ++u) {
+                        const int j = j0 + u * T;
+                        x[u] = j < p.d ? hq[j] : 0.0f;
+                    }
+#pragma unroll
+                    for (int u = 0; u < U; ++u) {
+                        const int j = j0 + u * T;
+                        if (j < width) {
+                            float r = x[u], sp = s0, inv = inv0;
+#pragma unroll
+                            for (int pc = 0; pc < kQ8Pieces; ++pc) {
+                                const uint8_t c = e4m3_code(r * inv);
+                                *at(kQ8Pieces * q + pc, j & (KB - 1), j / KB) = c;
+                                r -= sp * e4m3_value(c);
+                                sp *= 0x1p-4f;
+                                inv *= 16.0f;
+                            }
+                        }
+                    }
+                }
+            }
+        }
+        fence_proxy_async_smem();  // the MMAs read these bytes through the async proxy
+        named_barrier_sync(3, T);
+    }
 
     if (warp == 0) {
         // ---------------- TMA producer ----------------
@@ -362,18 +464,12 @@ __global__ void __launch_bounds__(TcShape<NQ, Q8>::kThreads, 1)
                     for (int i = 0; i < nin; ++i)
                         tma_load_2d(st + i * Sh::kStageA, &mapW, (kb0 + i) * KB, tile * kTcTile,
                                     &full[s], pol);
-                    if (it == 0) {
-                        griddep_wait();  // the query matrix comes from the prep kernel
-                        if (hres) {
-                            mbar_arrive_expect_tx(hbar, hres_bytes);
-                            for (int kb = 0; kb < n_kb; ++kb)
-                                tma_load_2d(hq_res + kb * Sh::kStageB, &mapH, kb * KB, 0, hbar, pol);
-                        }
-                    }
-                    if (!hres)
+                    if (!hres) {
+                        if (it == 0) griddep_wait();  // the query matrix comes from the prep kernel
                         for (int i = 0; i < nin; ++i)
                             tma_load_2d(st + KPS * Sh::kStageA + i * Sh::kStageB, &mapH,
                                         (kb0 + i) * KB, 0, &full[s], pol);
+                    }
                     issued = it + 1;
                 }
                 if (tile < 0) break;
@@ -384,7 +480,6 @@ __global__ void __launch_bounds__(TcShape<NQ, Q8>::kThreads, 1)
                 const int never = 0;
                 for (int t2 = max(0, issued - S); t2 < issued; ++t2)
                     mbar_wait(&full[t2 % S], (t2 / S) & 1, const_cast<volatile int *>(&never));
-                if (hres && issued > 0) mbar_wait(hbar, 0, const_cast<volatile int *>(&never));
             }
         }
     } else if (warp == 1) {
@@ -393,7 +488,6 @@ __global__ void __launch_bounds__(TcShape<NQ, Q8>::kThreads, 1)
             constexpr uint32_t idesc = Q8 ? umma_idesc_e4m3_f32(kTcTile, N) : umma_idesc_bf16_f32(kTcTile, N);
             int it = 0;
             bool ok = true;
-            bool h_ready = !hres;
             for (int ti = 0; ok; ++ti) {
                 const int b = ti & 1, ub = ti >> 1;
                 const int s0 = it % S, u0 = it / S;
@@ -420,13 +514,6 @@ __global__ void __launch_bounds__(TcShape<NQ, Q8>::kThreads, 1)
                     if (st_i > 0 && !mbar_wait(&full[s], u & 1, abort_flag)) {
                         ok = false;
                         break;
-                    }
-                    if (!h_ready) {
-                        if (!mbar_wait(hbar, 0, abort_flag)) {
-                            ok = false;
-                            break;
-                        }
-                        h_ready = true;
                     }
                     tc_fence_after_sync();
                     unsigned char *st = ring + s * stage_bytes;
@@ -462,9 +549,7 @@ __global__ void __launch_bounds__(TcShape<NQ, Q8>::kThreads, 1)
         // ---------------- epilogue: TMEM -> logits ----------------
         const int qw = warp & 3;  // TMEM lane quarter this warp may access
         const int row = 32 * qw + lane;
-        // Q8: the piece scales of the queries, next to the selectors' counts
-        float *qs = reinterpret_cast<float *>(bufs + NQ * Sh::kCap) + 3 * NQ;
-        if constexpr (Q8) {
+        if (Q8 && !hres) {
             griddep_wait();  // the prep kernel wrote them
             const int e = (warp - 2) * 32 + lane;
             if (e < NQ * kQ8Pieces) qs[e] = p.qscale[e];

@@ -11,19 +11,6 @@ namespace vie {
 
 namespace {
 
-// The least power of two >= v for v > 0, at least 2^-126 (the smallest
-// normal fp32): exact bit arithmetic on the fp32 encoding.
-__device__ __forceinline__ float pow2_at_least(float v) {
-    const uint32_t b = __float_as_uint(v);
-    if (b < 0x00800000u) return 0x1p-126f;     // zero or subnormal
-    if ((b & 0x007FFFFFu) == 0) return v;      // already a power of two
-    return __uint_as_float((b & 0x7F800000u) + 0x00800000u);
-}
-
-__device__ __forceinline__ float e4m3_value(uint8_t c) {
-    return __half2float(__half(__nv_cvt_fp8_to_halfraw(static_cast<__nv_fp8_storage_t>(c), __NV_E4M3)));
-}
-
 __device__ float block_max(float v, float *red) {
 #pragma unroll
     for (int o = 16; o >= 1; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xFFFFFFFFu, v, o));
@@ -70,7 +57,7 @@ __global__ void __launch_bounds__(256) prep_queries_e4m3_kernel(const float *__r
         float s = s0;
 #pragma unroll
         for (int pc = 0; pc < kQ8Pieces; ++pc) {
-            const uint8_t c = static_cast<uint8_t>(__nv_cvt_float_to_fp8(r / s, __NV_SATFINITE, __NV_E4M3));
+            const uint8_t c = e4m3_code(r / s);
             hQ[static_cast<int64_t>(kQ8Pieces * q + pc) * d_pad + j] = c;
             r -= s * e4m3_value(c);
             s *= 0x1p-4f;

@@ -34,6 +34,8 @@ def test_quantiser_is_bit_exact(vie, V, d):
         assert head.plan(16, 50).path == (1 if p.d_pad >= 128 else 0)
         assert head.plan(1, 50).path == (1 if p.d_pad >= 128 else 0)
         assert head.plan(4, 129).path == 0
+        if p.d_pad >= 128:  # up to 4 queries: the CTAs build the pieces themselves, one launch
+            assert head.plan(4, 50).launches == 1 and head.plan(5, 50).launches == 2
 
 
 def _parity(vie, W, h, k, reps=1):
@@ -188,3 +190,18 @@ def test_streaming_kernel_on_e4m3_rows():
     env = dict(os.environ, VIE_TC_MIN_BATCH_E4M3="100000")
     r = subprocess.run([sys.executable, "-c", code], env=env, capture_output=True, text=True, timeout=600)
     assert r.returncode == 0 and r.stdout.strip().endswith("ok"), r.stdout + r.stderr
+
+
+@pytest.mark.parametrize("batch", [1, 3, 12])
+def test_zero_and_tiny_queries(vie, batch):
+    """An all-zero query (every logit 0: the first k indices) and queries of
+    very small or very large magnitude next to ordinary ones."""
+    W, h = workload(20011, 1024, batch, seed=71 + batch)
+    h[0] = 0.0
+    if batch > 1:
+        h[1] *= 1e-30
+    if batch > 2:
+        h[2] *= 1e30
+    (idx, val), _ = _parity(vie, W, h, 50)
+    np.testing.assert_array_equal(idx[0], np.arange(50))
+    assert not np.any(val[0])

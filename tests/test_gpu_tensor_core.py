@@ -16,7 +16,7 @@ def test_plan_selects_paths(vie):
     with vie.Head(to_device_bits(W)) as head:
         p = head.plan(1, 50)
         assert (p.path, p.groups, p.launches) == (0, 1, 1)
-        p = head.plan(2, 50)
+        p = head.plan(2, 50)  # query prep, then the projection
         assert (p.path, p.groups, p.launches) == (1, 1, 2)
         p = head.plan(40, 50)  # one 64-query group: one pass over W
         assert (p.path, p.groups, p.launches) == (1, 1, 2)
