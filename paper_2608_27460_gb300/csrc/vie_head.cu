@@ -513,13 +513,13 @@ static vie_status run_topk_tc(const char *fn, vie_head *head, const float *h, in
     // K-blocks per stage: the most that still leave a ring of two stages
     // (larger stages beat deeper rings of small ones); the query boxes stay
     // resident in shared memory when they are small (e4m3 rows)
-    int stages = 0, kps = 0;
+    int stages = 0, kps = 0, slots = 0;
     uint32_t smem = 0;
     int kps_max = knobs().tc_kps;
     kps_max = kps_max < 1 ? 1 : (kps_max > vie::kTcMaxKPS ? vie::kTcMaxKPS : kps_max);
     const int hres_bytes = tc_hres(head, nqt);
     for (int c = kps_max; c >= 1 && kps == 0; --c) {
-        if (vie::tc_shape(nqt, q8, c, hres_bytes, &stages, &smem)) kps = c;
+        if (vie::tc_shape(nqt, q8, c, hres_bytes, &stages, &slots, &smem)) kps = c;
     }
     if (kps == 0) return fail(VIE_ERR_UNSUPPORTED, "%s: no tensor-core layout", fn);
     const int n_tiles = static_cast<int>((head->V + vie::kTcTile - 1) / vie::kTcTile);
@@ -542,6 +542,7 @@ static vie_status run_topk_tc(const char *fn, vie_head *head, const float *h, in
         p.nq = nq;
         p.stages = stages;
         p.kb_per_stage = kps;
+        p.score_slots = slots;
         p.static_tiles = static_cast<int32_t>(static_cast<int64_t>(n_tiles) * pct / 100 / head->G);
         p.cand = head->cand;  // [NQ][G][k] keys (NQ * k <= kTcListKeys), then the heads
         p.heads = head->cand + static_cast<size_t>(vie::kTcListKeys) * head->G;

@@ -48,10 +48,11 @@ cudaError_t launch_sample_topk(const int32_t *idx, const float *logits, int batc
 // Largest k the tensor-core kernel with nq_tmpl query slots handles (q8: on
 // e4m3 rows).
 int tc_max_k(int nq_tmpl, bool q8 = false);
-// Ring depth and dynamic shared memory for query groups of nq_tmpl (8, 16,
-// 32 or 64; 4, 8, 16 or 32 on e4m3 rows), kps K-blocks per stage and
-// hres_bytes of resident query boxes; false if unsupported.
-bool tc_shape(int nq_tmpl, bool q8, int kps, int hres_bytes, int *stages, uint32_t *smem);
+// Ring depth, score-ring depth and dynamic shared memory for query groups of
+// nq_tmpl (8, 16, 32 or 64; 4, 8, 16 or 32 on e4m3 rows), kps K-blocks per
+// stage and hres_bytes of query operand built in shared memory; false if
+// unsupported.
+bool tc_shape(int nq_tmpl, bool q8, int kps, int hres_bytes, int *stages, int *slots, uint32_t *smem);
 // Bytes of the query operand each CTA builds in shared memory itself for this
 // group shape and n_kb K-blocks (0: a prep kernel writes it and its boxes
 // travel with every ring stage).

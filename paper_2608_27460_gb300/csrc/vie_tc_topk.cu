@@ -24,23 +24,24 @@ __global__ void prep_queries_kernel(const float *__restrict__ h, int nq, int d, 
 }
 
 template <int NQ, bool Q8>
-void tc_sizes(int *score_bytes, int *buf_bytes, int *kb_w_bytes, int *kb_h_bytes) {
-    *score_bytes = TcShape<NQ, Q8>::kScoreBytes;
+void tc_sizes(int *slot_bytes, int *min_slots, int *buf_bytes, int *kb_w_bytes, int *kb_h_bytes) {
+    *slot_bytes = TcShape<NQ, Q8>::kSlotBytes;
+    *min_slots = TcShape<NQ, Q8>::kMinSlots;
     *buf_bytes = TcShape<NQ, Q8>::kBufBytes;
     *kb_w_bytes = TcShape<NQ, Q8>::kStageA;
     *kb_h_bytes = TcShape<NQ, Q8>::kStageB;
 }
 
-bool tc_sizes_of(int nq_tmpl, bool q8, int *score_bytes, int *buf_bytes, int *kb_w, int *kb_h) {
+bool tc_sizes_of(int nq_tmpl, bool q8, int *slot_bytes, int *min_slots, int *buf_bytes, int *kb_w, int *kb_h) {
     switch (q8 ? -nq_tmpl : nq_tmpl) {
-        case 8: tc_sizes<8, false>(score_bytes, buf_bytes, kb_w, kb_h); return true;
-        case 16: tc_sizes<16, false>(score_bytes, buf_bytes, kb_w, kb_h); return true;
-        case 32: tc_sizes<32, false>(score_bytes, buf_bytes, kb_w, kb_h); return true;
-        case 64: tc_sizes<64, false>(score_bytes, buf_bytes, kb_w, kb_h); return true;
-        case -4: tc_sizes<4, true>(score_bytes, buf_bytes, kb_w, kb_h); return true;
-        case -8: tc_sizes<8, true>(score_bytes, buf_bytes, kb_w, kb_h); return true;
-        case -16: tc_sizes<16, true>(score_bytes, buf_bytes, kb_w, kb_h); return true;
-        case -32: tc_sizes<32, true>(score_bytes, buf_bytes, kb_w, kb_h); return true;
+        case 8: tc_sizes<8, false>(slot_bytes, min_slots, buf_bytes, kb_w, kb_h); return true;
+        case 16: tc_sizes<16, false>(slot_bytes, min_slots, buf_bytes, kb_w, kb_h); return true;
+        case 32: tc_sizes<32, false>(slot_bytes, min_slots, buf_bytes, kb_w, kb_h); return true;
+        case 64: tc_sizes<64, false>(slot_bytes, min_slots, buf_bytes, kb_w, kb_h); return true;
+        case -4: tc_sizes<4, true>(slot_bytes, min_slots, buf_bytes, kb_w, kb_h); return true;
+        case -8: tc_sizes<8, true>(slot_bytes, min_slots, buf_bytes, kb_w, kb_h); return true;
+        case -16: tc_sizes<16, true>(slot_bytes, min_slots, buf_bytes, kb_w, kb_h); return true;
+        case -32: tc_sizes<32, true>(slot_bytes, min_slots, buf_bytes, kb_w, kb_h); return true;
         default: return false;
     }
 }
@@ -54,15 +55,22 @@ int tc_hres_bytes(int nq_tmpl, bool q8, int n_kb) {
     return b <= 48 * 1024 ? b : 0;
 }
 
-bool tc_shape(int nq_tmpl, bool q8, int kps, int hres_bytes, int *stages, uint32_t *smem) {
-    int score_bytes = 0, buf_bytes = 0, kb_w = 0, kb_h = 0;
-    if (!tc_sizes_of(nq_tmpl, q8, &score_bytes, &buf_bytes, &kb_w, &kb_h)) return false;
+// The ring first (as many stages as fit beside the fewest score slots), then
+// as many score slots as the shared memory left over holds.
+bool tc_shape(int nq_tmpl, bool q8, int kps, int hres_bytes, int *stages, int *slots, uint32_t *smem) {
+    int slot_bytes = 0, min_slots = 0, buf_bytes = 0, kb_w = 0, kb_h = 0;
+    if (!tc_sizes_of(nq_tmpl, q8, &slot_bytes, &min_slots, &buf_bytes, &kb_w, &kb_h)) return false;
     const int stage_bytes = kps * (hres_bytes > 0 ? kb_w : kb_w + kb_h);
     for (int s = kTcMaxStages; s >= 2; --s) {
-        const TcSmemLayout L(score_bytes, buf_bytes, s, stage_bytes, hres_bytes);
+        const TcSmemLayout L(min_slots * slot_bytes, buf_bytes, s, stage_bytes, hres_bytes);
         if (L.total <= 232448u) {
+            int sl = min_slots;
+            while (sl < kTcScoreSlots &&
+                   TcSmemLayout((sl + 1) * slot_bytes, buf_bytes, s, stage_bytes, hres_bytes).total <= 232448u)
+                ++sl;
             *stages = s;
-            *smem = L.total;
+            *slots = sl;
+            *smem = TcSmemLayout(sl * slot_bytes, buf_bytes, s, stage_bytes, hres_bytes).total;
             return true;
         }
     }

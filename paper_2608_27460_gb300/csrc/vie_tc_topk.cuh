@@ -19,10 +19,10 @@
 //                owns TMEM lanes 32*(w%4)..), hi + lo per query, logits into
 //                a score ring laid out [query][row];
 //   warps 6..    selectors, one query each (two when NQ = 32, four when
-//                NQ = 64): per query a shared buffer of candidates above a
-//                threshold tau; when fewer than 32 slots are left, a
-//                warp-wide bisection keeps the best k (unsorted) and raises
-//                tau; one bitonic sort of the final k per query.
+//                NQ = 64): per query a sorted list of the best keys so far,
+//                spread over the warp's registers (the streaming kernel's
+//                WarpList); a row enters only when its key beats the list's
+//                k-th, so the lists are final when the stream ends.
 // Each CTA writes its per-query lists and takes a completion ticket; the
 // last CTAs to finish merge them, one query each.  All waits are bounded.
 //
@@ -53,7 +53,7 @@ namespace vie {
 
 constexpr int kTcTile = 128;       // rows per tile (MMA M)
 constexpr int kTcKBlock = 64;      // bf16 columns per K-block (one 128-byte swizzle row)
-constexpr int kTcScoreSlots = 4;   // score ring depth
+constexpr int kTcScoreSlots = 8;   // score ring depth, at most (chosen per launch)
 constexpr int kTcMaxStages = 16;
 constexpr int kTcHRows = 128;      // rows of the hi/lo query matrix (N <= 128)
 constexpr int kTcMaxK = 128;       // largest k of this path
@@ -71,6 +71,7 @@ struct TcParams {
     int32_t stages;          // ring depth
     int32_t static_tiles;    // tiles each CTA owns before drawing from the pool
     int32_t kb_per_stage;    // K-blocks per ring stage (1..kTcMaxKPS)
+    int32_t score_slots;     // score ring depth (TcShape::kMinSlots..kTcScoreSlots)
     uint64_t *cand;          // [NQ][G][k] keys
     uint64_t *heads;         // [NQ][G][kTcMergeE]: the first keys of each list
     uint32_t *ticket;        // CTA completion counter (self-resetting)
@@ -101,15 +102,25 @@ struct TcShape {
     static constexpr int kStageBytes = kStageA + kStageB;    // per K-block; a multiple of 1024
     static constexpr int kTmemCols = (2 * N <= 32) ? 32 : (2 * N <= 64 ? 64 : (2 * N <= 128 ? 128 : 256));
     // score ring depth (e4m3 tiles: 2, leaving shared memory to the weight ring)
-    static constexpr int kSlots = NQ >= 64 ? 1 : ((NQ >= 32 || Q8) ? 2 : kTcScoreSlots);
-    static constexpr int kScoreBytes = kSlots * NQ * kTcTile * 4;
-    // candidate buffer per query: compacted to k whenever fewer than 32 slots
-    // (one row block) are left, so k <= kCap - 32
-    static constexpr int kCap = NQ >= 64 ? 128 : 256;
-    static constexpr int kMaxK0 = kCap - 32 < kTcMaxK ? kCap - 32 : kTcMaxK;
+    static constexpr int kMinSlots = NQ >= 64 ? 1 : 2;     // score ring depth, at least
+    static constexpr int kSlotBytes = NQ * kTcTile * 4;    // one tile's logits, [query][row]
+    // A selector keeps each query's best keys either in a register list of
+    // 32 * kMM positions (2 at 64 queries, where k <= 64; else 4), one
+    // insertion per key above the list's k-th, or - for the 4-query e4m3
+    // tile, whose weight stream is short beside a burst of insertions - in a
+    // shared buffer of kCap candidates above a bound, compacted to the best k
+    // by bisection when it fills and sorted once at the end.
+    static constexpr bool kBufSel = Q8 && NQ == 4;
+    static constexpr int kMM = NQ >= 64 ? 2 : 4;
+    static constexpr int kCap = 256;
+    static constexpr int kMaxK0 = kBufSel ? kTcMaxK : (32 * kMM < kTcMaxK ? 32 * kMM : kTcMaxK);
     static constexpr int kMaxK = kMaxK0 < kTcListKeys / NQ ? kMaxK0 : kTcListKeys / NQ;  // largest k
-    // buffers, counts, thresholds (and the Q8 piece scales)
-    static constexpr int kBufBytes = NQ * kCap * 8 + NQ * 12 + (Q8 ? NQ * kQ8Pieces * 4 : 0);
+    // shared memory next to the scores: the Q8 piece scales [NQ][4] fp32, then
+    // (buffer selectors) the counts [NQ], bounds [NQ] and buffers [NQ][kCap]
+    static constexpr int kQsBytes = Q8 ? NQ * kQ8Pieces * 4 : 0;
+    static constexpr int kCntOff = kQsBytes, kTauOff = (kCntOff + NQ * 4 + 7) & ~7;
+    static constexpr int kBufOff = (kTauOff + NQ * 8 + 15) & ~15;
+    static constexpr int kBufBytes = 16 + (kBufSel ? kBufOff + NQ * kCap * 8 : kQsBytes);
 };
 
 struct TcMisc {
@@ -302,7 +313,8 @@ __global__ void __launch_bounds__(TcShape<NQ, Q8>::kThreads, 1)
     const int kb_bytes = hres ? Sh::kStageA : Sh::kStageBytes;
     const int stage_bytes = KPS * kb_bytes;
     const int hres_bytes = hres ? n_kb * Sh::kStageB : 0;
-    const TcSmemLayout L(Sh::kScoreBytes, Sh::kBufBytes, S, stage_bytes, hres_bytes);
+    const int SL = p.score_slots;
+    const TcSmemLayout L(SL * Sh::kSlotBytes, Sh::kBufBytes, S, stage_bytes, hres_bytes);
     uint64_t *full = reinterpret_cast<uint64_t *>(smem + L.bars);
     uint64_t *empty = full + kTcMaxStages;
     uint64_t *tfull = empty + kTcMaxStages;
@@ -334,7 +346,7 @@ __global__ void __launch_bounds__(TcShape<NQ, Q8>::kThreads, 1)
             mbar_init(&tfull[b], 2);
             mbar_init(&tempty[b], 4);
         }
-        for (int s = 0; s < Sh::kSlots; ++s) {
+        for (int s = 0; s < SL; ++s) {
             mbar_init(&sfull[s], 4);
             mbar_init(&sempty[s], Sh::kSelWarps);
         }
@@ -352,7 +364,7 @@ __global__ void __launch_bounds__(TcShape<NQ, Q8>::kThreads, 1)
     const uint32_t tmem = mc->tmem_base;
     if (tid == 0) griddep_launch_dependents();  // a kernel launched after this one may be scheduled
     // Q8: the piece scales of the queries, next to the selectors' counts
-    float *qs = reinterpret_cast<float *>(bufs + NQ * Sh::kCap) + 3 * NQ;
+    float *qs = reinterpret_cast<float *>(bufs);
 
     if (Q8 && hres && warp > 0) {
         // ---------------- the query operand, built in shared memory ----------------
@@ -566,7 +578,7 @@ __global__ void __launch_bounds__(TcShape<NQ, Q8>::kThreads, 1)
             }
             tc_fence_after_sync();
             const int tile = mc->buf_tile[b];
-            const int ss = ti % Sh::kSlots, su = ti / Sh::kSlots;
+            const int ss = ti % SL, su = ti / SL;
             // Q8: this row's scale, loaded under the accumulator reads
             float rsc = 1.0f;
             if constexpr (Q8) {
@@ -576,7 +588,7 @@ __global__ void __launch_bounds__(TcShape<NQ, Q8>::kThreads, 1)
             if constexpr (N > 64) {
                 // wide tiles: wait for the score slot first, then drain the
                 // accumulator 32 columns (16 queries) at a time
-                if (ti >= Sh::kSlots && !mbar_wait(&sempty[ss], (su - 1) & 1, abort_flag)) {
+                if (ti >= SL && !mbar_wait(&sempty[ss], (su - 1) & 1, abort_flag)) {
                     if (lane == 0) {
                         atomicOr(p.err, kErrWaitTimeout);
                         mc->abort = 1;
@@ -644,7 +656,7 @@ __global__ void __launch_bounds__(TcShape<NQ, Q8>::kThreads, 1)
             tc_fence_before_sync();
             __syncwarp();
             if (lane == 0) mbar_arrive(&tempty[b]);
-            if (ti >= Sh::kSlots && !mbar_wait(&sempty[ss], (su - 1) & 1, abort_flag)) {
+            if (ti >= SL && !mbar_wait(&sempty[ss], (su - 1) & 1, abort_flag)) {
                 if (lane == 0) {
                     atomicOr(p.err, kErrWaitTimeout);
                     mc->abort = 1;
@@ -676,86 +688,153 @@ __global__ void __launch_bounds__(TcShape<NQ, Q8>::kThreads, 1)
                 for (int64_t i = sel * 32 + lane; i < fn; i += Sh::kSelWarps * 32) rw[i] = ninf;
             }
         }
-        // per query of this warp: candidate count and threshold, in shared
-        // memory next to its buffer (only this warp touches them)
         constexpr int QPW = Sh::kQPW;
-        constexpr int CAP = Sh::kCap, CAP_PER = CAP / 32;
-        int *cnt_s = reinterpret_cast<int *>(bufs + NQ * CAP) + QPW * sel;
-        uint64_t *tau_s = reinterpret_cast<uint64_t *>(bufs + NQ * CAP) + NQ / 2 + QPW * sel;
-        if (lane < QPW) {
-            cnt_s[lane] = 0;
-            tau_s[lane] = 0;
-        }
-        __syncwarp();
-        const unsigned lt_mask = (1u << lane) - 1u;
-        for (int ti = 0;; ++ti) {
-            const int ss = ti % Sh::kSlots, su = ti / Sh::kSlots;
-            if (!mbar_wait(&sfull[ss], su & 1, abort_flag)) {
-                if (lane == 0) {
-                    atomicOr(p.err, kErrWaitTimeout);
-                    mc->abort = 1;
-                }
-                break;
+        if constexpr (Sh::kBufSel) {
+            // per query of this warp: candidates above the bound tau in a shared
+            // buffer, their count and tau next to it (only this warp touches them)
+            constexpr int CAP = Sh::kCap, CAP_PER = CAP / 32;
+            unsigned char *bb = reinterpret_cast<unsigned char *>(bufs);
+            int *cnt_s = reinterpret_cast<int *>(bb + Sh::kCntOff) + QPW * sel;
+            uint64_t *tau_s = reinterpret_cast<uint64_t *>(bb + Sh::kTauOff) + QPW * sel;
+            uint64_t *buf0 = reinterpret_cast<uint64_t *>(bb + Sh::kBufOff);
+            if (lane < QPW) {
+                cnt_s[lane] = 0;
+                tau_s[lane] = 0;
             }
-            const int tile = mc->slot_tile[ss];
-            if (tile < 0) break;
-            const int64_t row0 = static_cast<int64_t>(tile) * kTcTile;
-            const int rows = static_cast<int>(min(static_cast<int64_t>(kTcTile), p.V - row0));
-            const float *sc = scores + ss * NQ * kTcTile;
+            __syncwarp();
+            const unsigned lt_mask = (1u << lane) - 1u;
+            for (int ti = 0;; ++ti) {
+                const int ss = ti % SL, su = ti / SL;
+                if (!mbar_wait(&sfull[ss], su & 1, abort_flag)) {
+                    if (lane == 0) {
+                        atomicOr(p.err, kErrWaitTimeout);
+                        mc->abort = 1;
+                    }
+                    break;
+                }
+                const int tile = mc->slot_tile[ss];
+                if (tile < 0) break;
+                const int64_t row0 = static_cast<int64_t>(tile) * kTcTile;
+                const int rows = static_cast<int>(min(static_cast<int64_t>(kTcTile), p.V - row0));
+                const float *sc = scores + ss * NQ * kTcTile;
+#pragma unroll 1
+                for (int j = 0; j < QPW; ++j) {
+                    const int q = QPW * sel + j;
+                    if (q >= p.nq) break;
+                    uint64_t *buf = buf0 + q * CAP;
+                    int cnt = cnt_s[j];
+                    uint64_t tau = tau_s[j];
+                    for (int rb = 0; rb < rows; rb += 32) {
+                        if (cnt > CAP - 32) {  // room for one more row block
+                            cnt = keep_best<CAP_PER>(buf, cnt, p.k, &tau_s[j], lane);
+                            tau = tau_s[j];
+                        }
+                        const int r = rb + lane;
+                        const uint64_t key =
+                            (r < rows) ? make_key(sc[q * kTcTile + r], static_cast<uint32_t>(row0 + r)) : 0;
+                        const bool in = key > tau;
+                        const unsigned m = __ballot_sync(0xFFFFFFFFu, in);
+                        if (in) buf[cnt + __popc(m & lt_mask)] = key;
+                        cnt += __popc(m);
+                    }
+                    __syncwarp();
+                    if (lane == 0) cnt_s[j] = cnt;
+                    __syncwarp();
+                }
+                if (lane == 0) mbar_arrive(&sempty[ss]);
+            }
+            // this CTA's sorted top-k per query and its first keys -> scratch
+            // (written even after a wait gave up: the merge then stays in bounds)
 #pragma unroll 1
             for (int j = 0; j < QPW; ++j) {
                 const int q = QPW * sel + j;
                 if (q >= p.nq) break;
-                uint64_t *buf = bufs + q * CAP;
-                int cnt = cnt_s[j];
-                uint64_t tau = tau_s[j];
-                for (int rb = 0; rb < rows; rb += 32) {
-                    if (cnt > CAP - 32) {  // room for one more row block
-                        cnt = keep_best<CAP_PER>(buf, cnt, p.k, &tau_s[j], lane);
-                        tau = tau_s[j];
+                uint64_t *dst = p.cand + (static_cast<size_t>(q) * G + cta) * p.k;
+                uint64_t *head = p.heads + (static_cast<size_t>(q) * G + cta) * kTcMergeE;
+                uint64_t *buf = buf0 + q * CAP;
+                if (p.k <= 32)
+                    write_sorted_list<CAP_PER, 1>(buf, cnt_s[j], p.k, &tau_s[j], dst, head, lane);
+                else if (p.k <= 64)
+                    write_sorted_list<CAP_PER, 2>(buf, cnt_s[j], p.k, &tau_s[j], dst, head, lane);
+                else
+                    write_sorted_list<CAP_PER, kTcMaxK / 32>(buf, cnt_s[j], p.k, &tau_s[j], dst, head, lane);
+            }
+        } else {
+            // per query of this warp: its best keys so far as a sorted list spread
+            // over the warp's registers, and the k-th of them as the entry bound
+            constexpr int MM = Sh::kMM;
+            WarpList<MM> list[QPW];
+            uint64_t tau[QPW];
+#pragma unroll
+            for (int j = 0; j < QPW; ++j) {
+                list[j].clear();
+                tau[j] = 0;
+            }
+            for (int ti = 0;; ++ti) {
+                const int ss = ti % SL, su = ti / SL;
+                if (!mbar_wait(&sfull[ss], su & 1, abort_flag)) {
+                    if (lane == 0) {
+                        atomicOr(p.err, kErrWaitTimeout);
+                        mc->abort = 1;
                     }
-                    const int r = rb + lane;
-                    const uint64_t key =
-                        (r < rows) ? make_key(sc[q * kTcTile + r], static_cast<uint32_t>(row0 + r)) : 0;
-                    const bool in = key > tau;
-                    const unsigned m = __ballot_sync(0xFFFFFFFFu, in);
-                    if (in) buf[cnt + __popc(m & lt_mask)] = key;
-                    cnt += __popc(m);
+                    break;
+                }
+                const int tile = mc->slot_tile[ss];
+                if (tile < 0) break;
+                const int64_t row0 = static_cast<int64_t>(tile) * kTcTile;
+                const int rows = static_cast<int>(min(static_cast<int64_t>(kTcTile), p.V - row0));
+                const float *sc = scores + ss * NQ * kTcTile;
+#pragma unroll
+                for (int j = 0; j < QPW; ++j) {
+                    const int q = QPW * sel + j;
+                    if (q < p.nq) {
+                        for (int rb = 0; rb < rows; rb += 32) {
+                            const int r = rb + lane;
+                            const uint64_t key =
+                                (r < rows) ? make_key(sc[q * kTcTile + r], static_cast<uint32_t>(row0 + r)) : 0;
+                            // every key above the block's entry bound goes in (one that
+                            // an earlier key of the block pushed below the k-th lands
+                            // past position k, harmlessly); the bound is refreshed once
+                            // per block
+                            unsigned m = __ballot_sync(0xFFFFFFFFu, key > tau[j]);
+                            if (m) {
+                                do {
+                                    const int src = __ffs(m) - 1;
+                                    m &= m - 1;
+                                    list[j].insert(shfl_u64(key, src), lane);
+                                } while (m);
+                                tau[j] = list[j].at(p.k - 1);
+                            }
+                        }
+                    }
                 }
                 __syncwarp();
-                if (lane == 0) cnt_s[j] = cnt;
-                __syncwarp();
+                if (lane == 0) mbar_arrive(&sempty[ss]);
             }
-            if (lane == 0) mbar_arrive(&sempty[ss]);
+            // this CTA's sorted top-k per query and its first keys -> scratch
+            // (written even after a wait gave up: the merge then stays in bounds)
+#pragma unroll
+            for (int j = 0; j < QPW; ++j) {
+                const int q = QPW * sel + j;
+                if (q < p.nq) {
+                    uint64_t *dst = p.cand + (static_cast<size_t>(q) * G + cta) * p.k;
+                    uint64_t *head = p.heads + (static_cast<size_t>(q) * G + cta) * kTcMergeE;
+#pragma unroll
+                    for (int s2 = 0; s2 < MM; ++s2) {
+                        const int pos = lane * MM + s2;
+                        if (pos < p.k) dst[pos] = list[j].v[s2];
+                        if (pos < kTcMergeE) head[pos] = list[j].v[s2];
+                    }
+                }
+            }
         }
     }
 
-    // Every warp is free now: warp w sorts and writes the lists of queries
-    // w, w + kWarps, ... (each query's buffer, count and bound are in shared
-    // memory, next to one another).
     __syncthreads();
     if (warp == 1) {
         tc_fence_after_sync();
         tmem_dealloc(tmem, Sh::kTmemCols);
     }
-    {
-        constexpr int CAP = Sh::kCap, CAP_PER = CAP / 32;
-        int *cnt_all = reinterpret_cast<int *>(bufs + NQ * CAP);
-        uint64_t *tau_all = reinterpret_cast<uint64_t *>(bufs + NQ * CAP) + NQ / 2;
-#pragma unroll 1
-        for (int q = warp; q < p.nq; q += Sh::kWarps) {
-            uint64_t *dst = p.cand + (static_cast<size_t>(q) * G + cta) * p.k;
-            uint64_t *head = p.heads + (static_cast<size_t>(q) * G + cta) * kTcMergeE;
-            if (p.k <= 32)
-                write_sorted_list<CAP_PER, 1>(bufs + q * CAP, cnt_all[q], p.k, &tau_all[q], dst, head, lane);
-            else if (p.k <= 64)
-                write_sorted_list<CAP_PER, 2>(bufs + q * CAP, cnt_all[q], p.k, &tau_all[q], dst, head, lane);
-            else
-                write_sorted_list<CAP_PER, kTcMaxK / 32>(bufs + q * CAP, cnt_all[q], p.k, &tau_all[q], dst,
-                                                         head, lane);
-        }
-    }
-    __syncthreads();
 
     // ---------------- completion ticket ----------------
     // bar.sync orders every thread's writes (lists, heads, sparse fill)
