@@ -532,8 +532,9 @@ def main(argv=None):
                      "kernel_us_p10_p50_p90": [round(float(np.percentile(kern_ms, q)) * 1e3, 2)
                                                for q in (10, 50, 90)]},
         "e2e": {"value": round(whole_job_us_per_step(e2e_us, world), 3), "unit": UNIT, "h2d_bytes_per_step": b * shape.d * 4,
-                "d2h_bytes_per_step": b * k * 8, "api": "vie_head_topk_host (pinned host h in, "
-                "top-k out, synchronised)", "clock": "host wall clock over the steps"},
+                "d2h_bytes_per_step": b * k * 8, "api": "vie_head_topk_host (pinned host h read and "
+                "top-k written in place by the kernels over NVLink-C2C, synchronised)",
+                "clock": "host wall clock over the steps"},
         "gpu_launches": K * launches_per_step,
         **({"sampling": sample_info} if sample_info else {}),
         **({"recall": recall_info} if recall_info else {}),

@@ -190,7 +190,11 @@ vie_status vie_head_topk_sparse(vie_head *head, const float *h, int32_t batch, i
  *   out_sparse   device, fp32 [batch, V] (4-byte aligned), or NULL.
  *   batch, k, stream: as for vie_head_topk.
  *
- * The queries and the top-k pass through device buffers owned by the handle:
+ * Page-locked buffers (mapped into the device's address space) are used in
+ * place: the kernels read page-locked queries straight from host memory, and
+ * when idx_host and logits_host are both page-locked the kernel that merges
+ * the top-k writes it there, with no copies.  Other buffers pass through
+ * device buffers owned by the handle:
  * allocated by the first call that needs them (larger ones by a later call
  * that needs more, VIE_ERR_OOM if that fails), freed by vie_head_destroy.  The
  * call synchronises `stream` before it returns, so the host outputs are

@@ -733,6 +733,17 @@ vie_status vie_head_topk_sample(vie_head *head, const float *h, int32_t batch, i
                            out_token, out_prob, stream);
 }
 
+// The device address of pinned (page-locked, mapped) host memory, or nullptr
+// for memory the device cannot address directly.
+static void *mapped_view(const void *host_ptr) {
+    cudaPointerAttributes a;
+    if (cudaPointerGetAttributes(&a, host_ptr) != cudaSuccess) {
+        cudaGetLastError();
+        return nullptr;
+    }
+    return a.type == cudaMemoryTypeHost ? a.devicePointer : nullptr;
+}
+
 vie_status vie_head_topk_host(vie_head *head, const float *h_host, int32_t batch, int32_t k,
                               int32_t *idx_host, float *logits_host, float *out_sparse,
                               vie_stream stream) {
@@ -748,7 +759,16 @@ vie_status vie_head_topk_host(vie_head *head, const float *h_host, int32_t batch
     vie_status st = check_device(head);
     if (st != VIE_OK) return st;
     const size_t nh = static_cast<size_t>(batch) * head->d, no = static_cast<size_t>(batch) * k;
-    if (head->stage_h_elems < nh) {
+    // pinned buffers are used in place: the kernels read the queries from
+    // host memory (measured faster than a copy in first) and the merging CTA
+    // writes the top-k there (no copies back); VIE_HOST_H_DIRECT=0 copies
+    // pinned queries in all the same
+    int32_t *idx_dev = static_cast<int32_t *>(mapped_view(idx_host));
+    float *logits_dev = static_cast<float *>(mapped_view(logits_host));
+    const bool out_direct = idx_dev != nullptr && logits_dev != nullptr;
+    static const bool h_direct_knob = env_int("VIE_HOST_H_DIRECT", 1) != 0;
+    const float *h_dev = h_direct_knob ? static_cast<const float *>(mapped_view(h_host)) : nullptr;
+    if (h_dev == nullptr && head->stage_h_elems < nh) {
         cudaFree(head->stage_h);
         head->stage_h = nullptr;
         head->stage_h_elems = 0;
@@ -759,7 +779,7 @@ vie_status vie_head_topk_host(vie_head *head, const float *h_host, int32_t batch
         }
         head->stage_h_elems = nh;
     }
-    if (head->stage_out_elems < no) {
+    if (!out_direct && head->stage_out_elems < no) {
         cudaFree(head->stage_idx);
         cudaFree(head->stage_logits);
         head->stage_idx = nullptr;
@@ -774,14 +794,20 @@ vie_status vie_head_topk_host(vie_head *head, const float *h_host, int32_t batch
         head->stage_out_elems = no;
     }
     cudaStream_t s = static_cast<cudaStream_t>(stream);
-    cudaError_t e = cudaMemcpyAsync(head->stage_h, h_host, nh * sizeof(float), cudaMemcpyHostToDevice, s);
-    if (e != cudaSuccess) return fail_cuda(e, "vie_head_topk_host: copy of h");
-    st = run_topk(fn, head, head->stage_h, batch, k, head->stage_idx, head->stage_logits, out_sparse,
-                  stream);
+    cudaError_t e = cudaSuccess;
+    if (h_dev == nullptr) {
+        e = cudaMemcpyAsync(head->stage_h, h_host, nh * sizeof(float), cudaMemcpyHostToDevice, s);
+        if (e != cudaSuccess) return fail_cuda(e, "vie_head_topk_host: copy of h");
+    }
+    st = run_topk(fn, head, h_dev != nullptr ? h_dev : head->stage_h, batch, k,
+                  out_direct ? idx_dev : head->stage_idx, out_direct ? logits_dev : head->stage_logits,
+                  out_sparse, stream);
     if (st != VIE_OK) return st;
-    e = cudaMemcpyAsync(idx_host, head->stage_idx, no * sizeof(int32_t), cudaMemcpyDeviceToHost, s);
-    if (e == cudaSuccess)
-        e = cudaMemcpyAsync(logits_host, head->stage_logits, no * sizeof(float), cudaMemcpyDeviceToHost, s);
+    if (!out_direct) {
+        e = cudaMemcpyAsync(idx_host, head->stage_idx, no * sizeof(int32_t), cudaMemcpyDeviceToHost, s);
+        if (e == cudaSuccess)
+            e = cudaMemcpyAsync(logits_host, head->stage_logits, no * sizeof(float), cudaMemcpyDeviceToHost, s);
+    }
     if (e == cudaSuccess) e = cudaStreamSynchronize(s);
     if (e != cudaSuccess) return fail_cuda(e, "vie_head_topk_host: copy of the top-k");
     return VIE_OK;
