@@ -446,6 +446,11 @@ __global__ void __launch_bounds__(TcShape<NQ, Q8>::kThreads, 1)
             const uint64_t pol = l2_evict_first_policy();
             const int Ns = p.static_tiles;
             const int pool0 = G * Ns;
+            // The pool counter is re-armed by the previous launch's last
+            // merging CTA, and this launch may start before that one ends
+            // (programmatic dependent launch): the first draw waits for it.
+            // With static tiles to issue first, the wait has long been over.
+            if (Ns == 0) griddep_wait();
             uint32_t draw = (Ns == 0) ? atomic_add_relaxed_gpu(p.next_tile, 1u) : 0u;
             int it = 0, issued = 0;
             bool ok = true;
@@ -457,7 +462,10 @@ __global__ void __launch_bounds__(TcShape<NQ, Q8>::kThreads, 1)
                     tile = pool0 + static_cast<int>(draw);
                     if (tile >= n_tiles) tile = -1;
                 }
-                if (tile >= 0 && ti + 1 >= Ns) draw = atomic_add_relaxed_gpu(p.next_tile, 1u);
+                if (tile >= 0 && ti + 1 >= Ns) {
+                    if (ti + 1 == Ns) griddep_wait();
+                    draw = atomic_add_relaxed_gpu(p.next_tile, 1u);
+                }
                 const int nst = tile < 0 ? 1 : n_st;
                 for (int st_i = 0; st_i < nst; ++st_i, ++it) {
                     const int s = it % S, u = it / S;
