@@ -8,7 +8,8 @@ top-k, and the sparse -inf logit tensor.  Default workload: the Qwen3-0.6B-shape
 k = 50, seeded synthetic weights and queries (no real checkpoint here).
 
 Prints one JSON line (rank 0).  ``--impl reference`` times the CPU oracle on
-the same workload instead (the reference arm of this build).
+the same workload instead: there is no other implementation of this head to
+run, so the oracle is the reference arm.
 """
 from __future__ import annotations
 

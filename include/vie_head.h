@@ -43,7 +43,7 @@ typedef void *vie_stream;         /* a cudaStream_t */
 typedef enum {
     VIE_OK = 0,
     VIE_ERR_INVALID_ARG = 1, /* a pointer, size or enum value is out of range */
-    VIE_ERR_UNSUPPORTED = 2, /* valid request beyond what this build serves  */
+    VIE_ERR_UNSUPPORTED = 2, /* valid request beyond what this library serves */
     VIE_ERR_CUDA = 3,        /* a CUDA runtime call or a launch failed        */
     VIE_ERR_OOM = 4,         /* device memory could not be allocated          */
     VIE_ERR_DEVICE = 5       /* a kernel recorded a device-side problem       */
@@ -51,7 +51,7 @@ typedef enum {
 
 typedef enum { VIE_DTYPE_BF16 = 0 } vie_dtype;
 
-/* Limits of this build. */
+/* Limits of this library. */
 #define VIE_K_MAX 1024     /* largest k of vie_head_topk                    */
 #define VIE_BATCH_MAX 1024 /* largest batch of vie_head_topk                */
 #define VIE_D_MAX 16384    /* largest hidden size d                         */
@@ -79,7 +79,7 @@ typedef struct {
  *          of 2 bytes.  Only read during the call; the caller may free it
  *          afterwards.
  *   V      1 <= V <= 2^31 - 2;   d   1 <= d <= VIE_D_MAX;
- *   dtype  VIE_DTYPE_BF16 (the only dtype of this build).
+ *   dtype  VIE_DTYPE_BF16 (the only dtype of this library).
  *   out    host; receives the new handle.
  *
  * The handle owns a padded copy [V, d_pad] (d_pad = d rounded up to a

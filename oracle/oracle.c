@@ -18,7 +18,7 @@
  * element is widened exactly to fp64 and each z_i is one sequential fp64
  * sum over j = 0..d-1 in index order.  No blocking, no reordering.
  *
- * Readings of points the paper leaves open (each is listed in the design doc):
+ * Readings of points the paper leaves open:
  *   - ties between equal logits are broken by ascending vocabulary index;
  *   - the sparse tensor is fp32 with -inf = 0xFF800000;
  *   - within a row of the sparse tensor, indices are expected to be distinct;
@@ -31,7 +31,7 @@
  * probable tokens; Section 3: the retrieved logits feed standard logit
  * processors such as top-p and min-p as a second stage; Section 4 samples
  * with k = 50).  The paper names no random generator and no processor order;
- * the readings taken (also listed in the design doc) are:
+ * the readings taken are:
  *   - probabilities are the softmax of z / T over the k candidates;
  *   - top-p and min-p are both defined on that softmax, so each keeps a
  *     prefix of the candidates (they are sorted by logit) and the kept set is
