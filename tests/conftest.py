@@ -24,7 +24,7 @@ def cuda_available():
 
 @pytest.fixture(scope="session")
 def vie(cuda_available):
-    """The CUDA binding, loaded on a GPU machine; GPU tests fail loudly without it."""
+    """The CUDA binding, loaded where a CUDA device is present; GPU tests fail loudly without it."""
     if not cuda_available:
         pytest.skip("no CUDA device")
     import paper_2608_27460_gb300 as vie_mod

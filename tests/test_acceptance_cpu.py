@@ -1,4 +1,4 @@
-"""The acceptance checker accepts the oracle's own answer and rejects the
+"""The acceptance rule accepts the oracle's own answer and rejects the
 mistakes a GPU path could make (CPU only)."""
 import numpy as np
 
