@@ -65,6 +65,9 @@ def _parity(vie, W, h, k, reps=1):
     (30011, 1024, 32, 50),   # full 32-query group
     (30011, 2048, 45, 7),    # two groups: 32 + 13
     (10007, 200, 2, 50),     # d_pad 208: a partial last K-block of 128 codes
+    (130, 128, 1, 50),       # one and a bit tiles: most CTAs write empty lists
+    (300, 512, 12, 100),     # 16-query group over three tiles
+    (64, 256, 3, 64),        # k = V
     (20011, 1024, 1, 50),
     (4099, 100, 3, 50),      # padded rows
     (33333, 2048, 4, 1),

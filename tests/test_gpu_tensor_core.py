@@ -37,6 +37,10 @@ def test_plan_selects_paths(vie):
     (20011, 1152, 100, 50),  # 64 + 36 queries
     (30011, 256, 32, 1),     # greedy, full group of 32
     (50021, 1024, 17, 77),
+    (100, 64, 4, 50),        # one tile: most CTAs draw nothing and write empty lists
+    (64, 128, 2, 64),        # k = V on one CTA
+    (200, 256, 40, 64),      # 64-query tile over two tiles
+    (129, 128, 8, 128),      # largest k, a one-row last tile
 ])
 def test_tensor_core_parity(vie, V, d, batch, k):
     W, h = workload(V, d, batch, seed=V + batch + k)
