@@ -341,6 +341,24 @@ def cpu_oracle_sample(W, h_pool, k, budget_s, batch, storage="bf16"):
     return dt / n * 1e6, n, threads, results
 
 
+def cpu_oracle_single_thread(W, h_pool, k, batch, storage="bf16", steps=2, budget_s=5.0):
+    """The same decode step on one host core: up to `steps` steps, fewer once
+    `budget_s` is spent (at least one)."""
+    import oracle
+    topk, _ = oracle_head(W, storage)
+    V = W.shape[0]
+    t0 = time.perf_counter()
+    n = 0
+    while n < steps:
+        hb = h_pool[(n * batch) % len(h_pool):][:batch]
+        idx, val = topk(hb, k, 1)
+        oracle.scatter(idx, val.astype(np.float32), V)
+        n += 1
+        if time.perf_counter() - t0 >= budget_s:
+            break
+    return (time.perf_counter() - t0) / n * 1e6, n
+
+
 def run_reference(args, rank, world):
     """Reference arm: the CPU oracle timed on this host on the same workload."""
     if rank != 0:
@@ -603,10 +621,12 @@ def main(argv=None):
             "operands": "e4m3 x e4m3 (kind::f8f6f4)" if e4m3 else "bf16 x bf16 (kind::f16)"}
     if not args.no_cpu_baseline and world == 1:
         us, n, threads, results = cpu_oracle_sample(W, h, k, args.cpu_seconds, b, args.storage)
+        us1, n1 = cpu_oracle_single_thread(W, h, k, b, args.storage)
         line["cpu_baseline"] = {"value": round(us, 1), "unit": UNIT, "cores": threads, "kind": "oracle",
                                 "sample": f"{n} decode steps (batch {b}) of the same workload in "
                                           f"{args.cpu_seconds:.0f} s: fp64 projection, full sort, "
-                                          "sparse tensor"}
+                                          "sparse tensor",
+                                "single_core": {"value": round(us1, 1), "unit": UNIT, "steps": n1}}
         # two of the sampled steps double as a parity check of the device path
         sys.path.insert(0, os.path.join(ROOT, "tests"))
         import oracle
