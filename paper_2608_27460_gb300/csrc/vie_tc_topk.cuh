@@ -224,14 +224,24 @@ static __device__ __noinline__ int keep_best(uint64_t *buf, int cnt, int k, uint
         const int e = j * 32 + lane;
         v[j] = e < cnt ? buf[e] : 0ull;  // 0 is below every key
     }
+    // two bits per step: the counts at the three candidate digits are
+    // independent reductions, so the chain of dependent ones halves
     uint32_t th = 0;
 #pragma unroll 1
-    for (int bit = 31; bit >= 0; --bit) {
-        const uint32_t c = th | (1u << bit);
-        int n = 0;
+    for (int bit = 30; bit >= 0; bit -= 2) {
+        const uint32_t c1 = th | (1u << bit), c2 = th | (2u << bit), c3 = th | (3u << bit);
+        int n1 = 0, n2 = 0, n3 = 0;
 #pragma unroll
-        for (int j = 0; j < PER; ++j) n += static_cast<uint32_t>(v[j] >> 32) >= c ? 1 : 0;
-        if (static_cast<int>(__reduce_add_sync(0xFFFFFFFFu, n)) >= k) th = c;
+        for (int j = 0; j < PER; ++j) {
+            const uint32_t hi = static_cast<uint32_t>(v[j] >> 32);
+            n1 += hi >= c1 ? 1 : 0;
+            n2 += hi >= c2 ? 1 : 0;
+            n3 += hi >= c3 ? 1 : 0;
+        }
+        n1 = static_cast<int>(__reduce_add_sync(0xFFFFFFFFu, n1));
+        n2 = static_cast<int>(__reduce_add_sync(0xFFFFFFFFu, n2));
+        n3 = static_cast<int>(__reduce_add_sync(0xFFFFFFFFu, n3));
+        th = n3 >= k ? c3 : (n2 >= k ? c2 : (n1 >= k ? c1 : th));
     }
     int n_gt = 0, n_ge = 0;
 #pragma unroll
@@ -280,7 +290,8 @@ static __device__ __noinline__ int keep_best(uint64_t *buf, int cnt, int k, uint
 template <int CAP_PER, int PER>
 static __device__ __noinline__ void write_sorted_list(uint64_t *buf, int cnt, int k, uint64_t *tau,
                                                       uint64_t *dst, uint64_t *head, int lane) {
-    if (cnt > k) cnt = keep_best<CAP_PER>(buf, cnt, k, tau, lane);
+    // (up to 32 * PER keys are sorted as they are; the first k are kept)
+    if (cnt > 32 * PER) cnt = keep_best<CAP_PER>(buf, cnt, k, tau, lane);
     uint64_t v[PER];
 #pragma unroll
     for (int j = 0; j < PER; ++j) {
