@@ -191,14 +191,29 @@ int env_int(const char *name, int dflt) {
 //   VIE_TC_MIN_BATCH     smallest batch sent to the tensor-core path (2)
 //   VIE_TC_KPS           128-byte K-blocks per tensor-core ring stage (4)
 //   VIE_TC_MIN_BATCH_E4M3  the same threshold for e4m3 heads (1)
+//   VIE_HALF_ROWS        streaming projection by half-warps: 1 on, 0 off,
+//                        -1 when a row's last pass would leave half the lanes idle (-1)
 struct Knobs {
-    int stage_min_bytes, static_pct, tc_min_batch, tc_kps, pool_div, tc_min_batch_e4m3;
+    int stage_min_bytes, static_pct, tc_min_batch, tc_kps, pool_div, tc_min_batch_e4m3, half_rows;
 };
 const Knobs &knobs() {
     static const Knobs k = {env_int("VIE_STAGE_MIN_KB", 48) * 1024, env_int("VIE_STATIC_PCT", 85),
                             env_int("VIE_TC_MIN_BATCH", 2), env_int("VIE_TC_KPS", 4),
-                            env_int("VIE_POOL_DIV", 1), env_int("VIE_TC_MIN_BATCH_E4M3", 1)};
+                            env_int("VIE_POOL_DIV", 1), env_int("VIE_TC_MIN_BATCH_E4M3", 1),
+                            env_int("VIE_HALF_ROWS", -1)};
     return k;
+}
+
+// Whether the streaming projection gives each half-warp its own row: with
+// 16-byte chunks c per row, a full warp's last pass over a row runs c mod 32
+// lanes; at most 16 of them means half-warps finish the row in one fewer
+// lane slot per row pair.  Needs two rows per warp (R >= 2).
+int half_rows_for(int r, int chunks) {
+    if (r < 2) return 0;
+    const int v = knobs().half_rows;
+    if (v >= 0) return v > 0 ? 1 : 0;
+    const int tail = chunks % 32;
+    return (tail != 0 && tail <= 16) ? 1 : 0;
 }
 
 // Rows of a pool piece for stages of rs rows.
@@ -608,6 +623,7 @@ static vie_status run_topk(const char *fn, vie_head *head, const float *h, int32
         pct = pct < 0 ? 0 : (pct > 100 ? 100 : pct);
         p.static_chunks = static_cast<int32_t>(n_chunks * pct / 100 / head->G);
         p.pool_rows = pool_rows_for(shp.rs);
+        p.half_rows = half_rows_for(shp.r, head->d_pad / (head->scale != nullptr ? 16 : 8));
         p.cand = head->cand;
         p.heads = head->cand + static_cast<size_t>(kMaxNB) * head->G * VIE_K_MAX;
         p.ticket = head->words;
@@ -986,6 +1002,7 @@ extern "C" vie_status vie_head_topk_noalloc(const void *W_out, int64_t V, int32_
         pct = pct < 0 ? 0 : (pct > 100 ? 100 : pct);
         p.static_chunks = static_cast<int32_t>(n_chunks * pct / 100 / G);
         p.pool_rows = pool_rows_for(shp.rs);
+        p.half_rows = half_rows_for(shp.r, d / 8);
         p.cand = reinterpret_cast<uint64_t *>(nd.scratch + kNoAllocCounterBytes);
         p.heads = p.cand + static_cast<size_t>(nb_max) * G * k;
         p.ticket = counters;

@@ -40,6 +40,7 @@
 #include <cuda_fp8.h>
 
 #include <cstdint>
+#include <type_traits>
 
 #include "vie_device.cuh"
 
@@ -68,6 +69,7 @@ struct StreamTopkParams {
     int32_t stages;          // S, weight ring depth
     int32_t static_chunks;   // chunks each CTA owns before drawing from the pool
     int32_t pool_rows;       // rows of a pool piece (<= rows_per_stage)
+    int32_t half_rows;       // 1: each half-warp projects its own row (R >= 2)
     uint64_t *cand;          // [NB][G][k] keys
     uint64_t *heads;         // [NB][G][kFastE]: the first keys of each list
     uint32_t *ticket;        // CTA completion counter (self-resetting)
@@ -800,98 +802,115 @@ __global__ void __launch_bounds__(kThreads, 1) stream_topk_kernel(const StreamTo
                 const int64_t row0 = chunk;
                 const int rows = stage_rows(row0, pool_row0, RS, RSH, p.V);
                 const unsigned char *stage = ring + s * stage_bytes;
-                // warp w owns rows w, w + 8, ... (at most R of them) of the stage
-                int rr[R];
+                // Warp w owns rows w, w + 8, ... (at most R of them) of the
+                // stage.  SPLIT = 1: the whole warp works on each row, lane
+                // l on chunks l, l + 32, ...  SPLIT = 2: the half-warps take
+                // the two rows of a pair (w + 8(2i), w + 8(2i+1)), half-lane l
+                // on chunks l, l + 16, ..., so rows of 16 * odd chunks leave
+                // no lane idle on the last pass.  Either way every row sums
+                // its products in the same order wherever it sits.
+                auto project = [&](auto split) -> bool {
+                    constexpr int SPLIT = decltype(split)::value;
+                    constexpr int RL = R / SPLIT;   // rows per lane
+                    constexpr int LW = 32 / SPLIT;  // lanes per row
+                    const int sub = lane / LW, sl = lane % LW;
+                    int rr[RL];
 #pragma unroll
-                for (int i = 0; i < R; ++i) rr[i] = min(w + i * kDotWarps, rows - 1);
-                float acc[R][NB];
+                    for (int i = 0; i < RL; ++i) rr[i] = min(w + (i * SPLIT + sub) * kDotWarps, rows - 1);
+                    float acc[RL][NB];
 #pragma unroll
-                for (int i = 0; i < R; ++i)
+                    for (int i = 0; i < RL; ++i)
 #pragma unroll
-                    for (int nb = 0; nb < NB; ++nb) acc[i][nb] = 0.0f;
-                float rscale[R];  // e4m3 rows: their scales, loaded under the FMA loop
+                        for (int nb = 0; nb < NB; ++nb) acc[i][nb] = 0.0f;
+                    float rscale[RL];  // e4m3 rows: their scales, loaded under the FMA loop
 #pragma unroll
-                for (int i = 0; i < R; ++i) rscale[i] = Q8 ? __ldg(p.row_scale + row0 + rr[i]) : 1.0f;
-                if (w < rows) {
-                    for (int c = lane; c < C; c += 32) {
-                        uint4 wv[R];
+                    for (int i = 0; i < RL; ++i) rscale[i] = Q8 ? __ldg(p.row_scale + row0 + rr[i]) : 1.0f;
+                    if (w < rows) {
+                        for (int c = sl; c < C; c += LW) {
+                            uint4 wv[RL];
 #pragma unroll
-                        for (int i = 0; i < R; ++i)
-                            wv[i] = *reinterpret_cast<const uint4 *>(stage + rr[i] * row_bytes + c * 16);
+                            for (int i = 0; i < RL; ++i)
+                                wv[i] = *reinterpret_cast<const uint4 *>(stage + rr[i] * row_bytes + c * 16);
 #pragma unroll
-                        for (int nb = 0; nb < NB; ++nb) {
-                            if constexpr (Q8) {
-                                const float *hq = h_s + nb * 4 * (C * 4) + c * 4;
-                                const float4 h0 = *reinterpret_cast<const float4 *>(hq);
-                                const float4 h1 = *reinterpret_cast<const float4 *>(hq + 1 * (C * 4));
-                                const float4 h2 = *reinterpret_cast<const float4 *>(hq + 2 * (C * 4));
-                                const float4 h3 = *reinterpret_cast<const float4 *>(hq + 3 * (C * 4));
+                            for (int nb = 0; nb < NB; ++nb) {
+                                if constexpr (Q8) {
+                                    const float *hq = h_s + nb * 4 * (C * 4) + c * 4;
+                                    const float4 h0 = *reinterpret_cast<const float4 *>(hq);
+                                    const float4 h1 = *reinterpret_cast<const float4 *>(hq + 1 * (C * 4));
+                                    const float4 h2 = *reinterpret_cast<const float4 *>(hq + 2 * (C * 4));
+                                    const float4 h3 = *reinterpret_cast<const float4 *>(hq + 3 * (C * 4));
 #pragma unroll
-                                for (int i = 0; i < R; ++i) {
-                                    float a = acc[i][nb];
-                                    a = fma_e4m3x4(wv[i].x, h0, a);
-                                    a = fma_e4m3x4(wv[i].y, h1, a);
-                                    a = fma_e4m3x4(wv[i].z, h2, a);
-                                    a = fma_e4m3x4(wv[i].w, h3, a);
-                                    acc[i][nb] = a;
-                                }
-                            } else {
-                                const float4 ha = *reinterpret_cast<const float4 *>(
-                                    h_s + (nb * 2 + 0) * (C * 4) + c * 4);
-                                const float4 hb = *reinterpret_cast<const float4 *>(
-                                    h_s + (nb * 2 + 1) * (C * 4) + c * 4);
+                                    for (int i = 0; i < RL; ++i) {
+                                        float a = acc[i][nb];
+                                        a = fma_e4m3x4(wv[i].x, h0, a);
+                                        a = fma_e4m3x4(wv[i].y, h1, a);
+                                        a = fma_e4m3x4(wv[i].z, h2, a);
+                                        a = fma_e4m3x4(wv[i].w, h3, a);
+                                        acc[i][nb] = a;
+                                    }
+                                } else {
+                                    const float4 ha = *reinterpret_cast<const float4 *>(
+                                        h_s + (nb * 2 + 0) * (C * 4) + c * 4);
+                                    const float4 hb = *reinterpret_cast<const float4 *>(
+                                        h_s + (nb * 2 + 1) * (C * 4) + c * 4);
 #pragma unroll
-                                for (int i = 0; i < R; ++i) {
-                                    float a = acc[i][nb];
-                                    a = fmaf(bf16_lo(wv[i].x), ha.x, a);
-                                    a = fmaf(bf16_hi(wv[i].x), ha.y, a);
-                                    a = fmaf(bf16_lo(wv[i].y), ha.z, a);
-                                    a = fmaf(bf16_hi(wv[i].y), ha.w, a);
-                                    a = fmaf(bf16_lo(wv[i].z), hb.x, a);
-                                    a = fmaf(bf16_hi(wv[i].z), hb.y, a);
-                                    a = fmaf(bf16_lo(wv[i].w), hb.z, a);
-                                    a = fmaf(bf16_hi(wv[i].w), hb.w, a);
-                                    acc[i][nb] = a;
+                                    for (int i = 0; i < RL; ++i) {
+                                        float a = acc[i][nb];
+                                        a = fmaf(bf16_lo(wv[i].x), ha.x, a);
+                                        a = fmaf(bf16_hi(wv[i].x), ha.y, a);
+                                        a = fmaf(bf16_lo(wv[i].y), ha.z, a);
+                                        a = fmaf(bf16_hi(wv[i].y), ha.w, a);
+                                        a = fmaf(bf16_lo(wv[i].z), hb.x, a);
+                                        a = fmaf(bf16_hi(wv[i].z), hb.y, a);
+                                        a = fmaf(bf16_lo(wv[i].w), hb.z, a);
+                                        a = fmaf(bf16_hi(wv[i].w), hb.w, a);
+                                        acc[i][nb] = a;
+                                    }
                                 }
                             }
                         }
                     }
-                }
-                // every read of the weight stage has retired: hand it back
-                __syncwarp();
-                if (lane == 0) mbar_arrive(&empty[s]);
+                    // every read of the weight stage has retired: hand it back
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(&empty[s]);
 #pragma unroll
-                for (int i = 0; i < R; ++i)
+                    for (int i = 0; i < RL; ++i)
 #pragma unroll
-                    for (int nb = 0; nb < NB; ++nb) {
-                        float a = acc[i][nb];
+                        for (int nb = 0; nb < NB; ++nb) {
+                            float a = acc[i][nb];
 #pragma unroll
-                        for (int o = 16; o >= 1; o >>= 1) a += __shfl_xor_sync(0xFFFFFFFFu, a, o);
-                        acc[i][nb] = a;
+                            for (int o = LW / 2; o >= 1; o >>= 1) a += __shfl_xor_sync(0xFFFFFFFFu, a, o);
+                            acc[i][nb] = a;
+                        }
+                    const int ss = t % kScoreStages, su = t / kScoreStages;
+                    if (t >= kScoreStages && !mbar_wait(&sempty[ss], (su - 1) & 1, abort_flag)) {
+                        if (lane == 0) {
+                            atomicOr(p.err, kErrWaitTimeout);
+                            ms->abort = 1;
+                        }
+                        return false;
                     }
-                const int ss = t % kScoreStages, su = t / kScoreStages;
-                if (t >= kScoreStages && !mbar_wait(&sempty[ss], (su - 1) & 1, abort_flag)) {
-                    if (lane == 0) {
-                        atomicOr(p.err, kErrWaitTimeout);
-                        ms->abort = 1;
-                    }
-                    break;
-                }
-                float *sc = scores + ss * RS * NB;
-                if (lane == 0) {
-                    if (w == 0) ms->chunk_s[ss] = chunk;
+                    float *sc = scores + ss * RS * NB;
+                    if (sl == 0) {
+                        if (w == 0 && sub == 0) ms->chunk_s[ss] = chunk;
 #pragma unroll
-                    for (int i = 0; i < R; ++i) {
-                        const int r = w + i * kDotWarps;
-                        if (r < rows) {
+                        for (int i = 0; i < RL; ++i) {
+                            const int r = w + (i * SPLIT + sub) * kDotWarps;
+                            if (r < rows) {
 #pragma unroll
-                            for (int nb = 0; nb < NB; ++nb)
-                                sc[r * NB + nb] = Q8 ? acc[i][nb] * rscale[i] : acc[i][nb];
+                                for (int nb = 0; nb < NB; ++nb)
+                                    sc[r * NB + nb] = Q8 ? acc[i][nb] * rscale[i] : acc[i][nb];
+                            }
                         }
                     }
-                }
-                __syncwarp();
-                if (lane == 0) mbar_arrive(&sfull[ss]);
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(&sfull[ss]);
+                    return true;
+                };
+                const bool ok = (R >= 2 && p.half_rows)
+                                    ? project(std::integral_constant<int, (R >= 2 ? 2 : 1)>{})
+                                    : project(std::integral_constant<int, 1>{});
+                if (!ok) break;
             }
             // pass the end of the stream on to the selector
             if (!*abort_flag) {
