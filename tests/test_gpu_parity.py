@@ -3,6 +3,8 @@
 Small cases span several stages and CTAs with ragged tails; the full-size
 cases use the five workload shapes with the launch configuration the bench
 times.  Acceptance rules are in tests/acceptance.py."""
+import functools
+
 import numpy as np
 import pytest
 
@@ -240,18 +242,42 @@ def test_props(vie):
 
 
 # ---------------------------------------------------------------------------
-# Full-size workloads, sampled queries (the oracle computes each one fully).
+# Full-size workloads in the launch configuration the bench times: one fused
+# call (top-k and the sparse tensor) per decode step of `batch` queries, so
+# batch 1 runs on the streaming kernel and batches of 2 or more on the tensor
+# cores.  The sampled queries are computed in full by the oracle.
 FULL = [("gemma3-270m", 1, 50, 3), ("qwen3-0.6b", 1, 50, 3), ("llama3.2-1b", 1, 50, 2),
-        ("llama3.2-1b", 4, 1, 4), ("llama3.2-1b", 4, 50, 4), ("gemma3-1b", 8, 50, 8),
-        ("gemma3-1b-ties", 4, 50, 4), ("llama3.2-3b", 16, 50, 16)]
+        ("llama3.2-1b", 1, 1, 2), ("llama3.2-1b", 4, 1, 4), ("llama3.2-1b", 4, 50, 4),
+        ("gemma3-1b", 1, 50, 2), ("gemma3-1b", 2, 50, 2), ("gemma3-1b", 4, 50, 4),
+        ("gemma3-1b", 8, 50, 8), ("gemma3-1b-ties", 1, 50, 4), ("gemma3-1b-ties", 4, 50, 4),
+        ("llama3.2-3b", 16, 50, 16), ("llama3.2-3b", 64, 50, 64)]
+
+
+@functools.lru_cache(maxsize=1)
+def _full_head(name):
+    """Weights and 64 queries of one workload (kept while the cases of that
+    workload run; they are listed together)."""
+    W, h, _, _ = synth.make_head(synth.HEADS[name], seed=0, n_queries=64)
+    return W, h
 
 
 @pytest.mark.parametrize("name,batch,k,n", FULL, ids=[f"{a}-b{b}-k{c}" for a, b, c, _ in FULL])
 def test_parity_full_size(vie, name, batch, k, n):
-    shape = synth.HEADS[name]
-    W, h, meta, _ = synth.make_head(shape, seed=0, n_queries=n)
-    idx, val = run_head(vie, W, h[:n], k)
+    import torch
+    W, h = _full_head(name)
+    V = W.shape[0]
     z = oracle.logits(W, h[:n])
-    for q in range(n):
-        e = check_topk(idx[q], val[q], z[q], k)
-        assert not e, (q, e)
+    with vie.Head(to_device_bits(W)) as head:
+        want_path = 0 if batch == 1 else 1
+        assert head.plan(batch, k).path == want_path
+        hd = torch.from_numpy(np.ascontiguousarray(h[:n])).cuda()
+        for q0 in range(0, n, batch):
+            idx, val, sparse = head.topk_sparse(hd[q0:q0 + batch], k)
+            torch.cuda.synchronize()
+            idx, val, sparse = idx.cpu().numpy(), val.cpu().numpy(), sparse.cpu().numpy()
+            for q in range(batch):
+                e = check_topk(idx[q], val[q], z[q0 + q], k)
+                assert not e, (q0 + q, e)
+            want, ok = oracle.scatter(idx, val, V)
+            assert ok and np.array_equal(want.view(np.uint32), sparse.view(np.uint32))
+        assert head.device_status() == vie.VIE_OK, vie.vie_last_error()
