@@ -38,23 +38,28 @@ def test_quantiser_is_bit_exact(vie, V, d):
             assert head.plan(4, 50).launches == 1 and head.plan(5, 50).launches == 2
 
 
-def _parity(vie, W, h, k, reps=1):
+def _parity(vie, W, h, k, reps=1, batch=None):
+    """Top-k of every query of h on an e4m3 handle against the oracle's e4m3
+    head; `batch` queries per call (all of them in one call by default)."""
     import torch
     q, sc = oracle.quantize_e4m3(W)
     z = oracle.logits_e4m3(q, sc, h)
+    n = h.shape[0]
+    batch = batch or n
     with _head(vie, W) as head:
         hd = torch.from_numpy(h).cuda()
         prev = None
         for _ in range(reps):
-            idx, val = head.topk(hd, k)
+            parts = [head.topk(hd[q0:q0 + batch], k) for q0 in range(0, n, batch)]
             torch.cuda.synchronize()
-            cur = (idx.cpu().numpy(), val.cpu().numpy())
+            cur = (np.concatenate([i.cpu().numpy() for i, _ in parts]),
+                   np.concatenate([v.cpu().numpy() for _, v in parts]))
             if prev is not None:
                 assert np.array_equal(prev[0], cur[0]) and np.array_equal(prev[1].view(np.uint32),
                                                                            cur[1].view(np.uint32))
             prev = cur
         assert head.device_status() == vie.VIE_OK
-    fails = {q_: e for q_ in range(h.shape[0]) if (e := check_topk(prev[0][q_], prev[1][q_], z[q_], k))}
+    fails = {q_: e for q_ in range(n) if (e := check_topk(prev[0][q_], prev[1][q_], z[q_], k))}
     assert not fails, next(iter(fails.items()))
     return prev, z
 
@@ -95,7 +100,7 @@ def test_duplicate_rows_tie_by_index(vie):
 def test_e4m3_full_size(vie, name, batch, k, n):
     shape = synth.HEADS[name]
     W, h, _, _ = synth.make_head(shape, seed=0, n_queries=n)
-    _parity(vie, W, h[:n], k)
+    _parity(vie, W, h[:n], k, batch=batch)  # one call per decode step of `batch` queries
 
 
 def test_host_entry_and_sampling_on_e4m3(vie):
