@@ -143,6 +143,46 @@ typedef struct {
 vie_status vie_head_plan(const vie_head *head, int32_t batch, int32_t k, vie_topk_plan *plan);
 
 /*
+ * Launch options - a hook for tests and tuning; the paper has no counterpart.
+ *
+ * By default the path and launch shape of a call depend only on the call
+ * (batch, k), the handle (V, d, bf16 or e4m3 rows) and the device: the
+ * defaults below are the shapes that measured fastest on GB300 and that the
+ * test suite covers.  An option changes how the work is laid out (which
+ * kernel, stage sizes, work split), never the results: every setting gives
+ * the same top-k under the same ranking rule.  Options are process-wide
+ * (all handles, all threads) and are read when a call plans its launches, so
+ * a change takes effect from the next call on; change them only while no
+ * other thread is inside a call of this library.  Nothing is read from the
+ * environment.
+ */
+typedef enum {
+    VIE_OPT_STAGE_MIN_KB = 0,      /* smallest streaming weight stage, KB       (48)  */
+    VIE_OPT_STATIC_PCT = 1,        /* % of W's pieces dealt round robin, rest
+                                      drawn from a shared pool                   (85)  */
+    VIE_OPT_POOL_DIV = 2,          /* pool pieces = one stage / this, 1..64      (1)   */
+    VIE_OPT_TC_MIN_BATCH = 3,      /* smallest batch of a bf16 head sent to the
+                                      tensor cores (k <= 128)                   (2)   */
+    VIE_OPT_TC_KPS = 4,            /* most K-blocks per tensor-core stage, 1..4  (4)   */
+    VIE_OPT_TC_MIN_BATCH_E4M3 = 5, /* the same threshold for e4m3 heads          (1)   */
+    VIE_OPT_HALF_ROWS = 6,         /* streaming projection, one row per
+                                      half-warp: 1 on, 0 off, -1 automatic       (-1)  */
+    VIE_OPT_HOST_H_DIRECT = 7,     /* vie_head_topk_host reads page-locked
+                                      queries in place: 1, or copies them: 0     (1)   */
+    VIE_OPT_COUNT = 8
+} vie_launch_option;
+
+#define VIE_OPT_DEFAULT INT32_MIN /* value that restores an option's default */
+
+/* Sets one option (VIE_OPT_DEFAULT restores its default).  Errors:
+ * VIE_ERR_INVALID_ARG for an unknown option or a value outside the range
+ * given above (the option keeps its value). */
+vie_status vie_set_launch_option(vie_launch_option option, int32_t value);
+
+/* Reads one option's current value into *value (host). */
+vie_status vie_get_launch_option(vie_launch_option option, int32_t *value);
+
+/*
  * vie_head_topk - exact top-k of z = W_out h for a batch of queries
  * (Section 3: output projection followed by top-k selection, computed by
  * exhaustive MIPS over every row, Section 2).
@@ -318,16 +358,25 @@ vie_status vie_scatter_sparse_logits(const int32_t *idx, const float *logits, in
  * callers cannot make one.  This entry point takes the weights as they are
  * and keeps its scratch in a fixed array compiled into the library instead.
  *
- *   W_out       device, bf16 bit patterns, row-major [V, d], 16-byte aligned,
- *               d a multiple of 8 (rows must already be 16-byte vectors).
+ *   W_out       device memory of the current device (or managed memory),
+ *               bf16 bit patterns, row-major [V, d], 16-byte aligned, d a
+ *               multiple of 8 (rows must already be 16-byte vectors).
  *   V, d        1 <= V <= 2^31 - 2;  8 <= d <= VIE_D_MAX.
  *   h, batch, k, out_idx, out_logits, stream: as for vie_head_topk.
  *
+ * Every batch runs on the streaming CUDA-core kernel, in query groups of up
+ * to `cap` queries, one launch per group:
+ *   cap = 8 for k <= 64, 4 for k <= 256, 1 above, then halved (not below 1)
+ *         while cap * d * 4 > 65536.
  * Scratch: one 1 MiB array per device (every GPU that loads the library keeps
- * it until the process exits).  A launch needs 8 * slots * ctas * (k + 4)
- * bytes of it, where ctas = min(SM count, ceil(V / 64)) and slots = the query group
- * width (the batch rounded up to a power of two, at most 8); larger requests
- * return VIE_ERR_UNSUPPORTED with the sizes in the message.  The call clears
+ * it until the process exits), of which the first 256 bytes hold counters.
+ * A call needs
+ *   8 * (round_up_even(slots * ctas * k) + slots * ctas * 4)
+ * bytes of the rest, where ctas = min(SM count, ceil(V / 64), 1024) and
+ * slots = the batch rounded up to a power of two, at most cap; larger
+ * requests return VIE_ERR_UNSUPPORTED with the sizes in the message.  Groups
+ * of one call run one after the other on `stream` and reuse the same lists
+ * (the kernel re-arms its counters at the end of each launch).  The call clears
  * the counters at the start of the array with cudaMemsetAsync on `stream`
  * and allocates nothing (no cudaMalloc, no cudaFree, no allocating library
  * routine).

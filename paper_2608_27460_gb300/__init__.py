@@ -34,6 +34,18 @@ VIE_MANY_MAX = 1 << 24
 VIE_RECALL_N_MAX = 1 << 28
 VIE_RECALL_M_MAX = 1 << 20
 
+# Launch options (vie_launch_option): tuning and test hooks, never results.
+VIE_OPT_STAGE_MIN_KB = 0
+VIE_OPT_STATIC_PCT = 1
+VIE_OPT_POOL_DIV = 2
+VIE_OPT_TC_MIN_BATCH = 3
+VIE_OPT_TC_KPS = 4
+VIE_OPT_TC_MIN_BATCH_E4M3 = 5
+VIE_OPT_HALF_ROWS = 6
+VIE_OPT_HOST_H_DIRECT = 7
+VIE_OPT_COUNT = 8
+VIE_OPT_DEFAULT = -(2 ** 31)
+
 STATUS_NAMES = {0: "VIE_OK", 1: "VIE_ERR_INVALID_ARG", 2: "VIE_ERR_UNSUPPORTED",
                 3: "VIE_ERR_CUDA", 4: "VIE_ERR_OOM", 5: "VIE_ERR_DEVICE"}
 
@@ -42,7 +54,7 @@ EXPORTS = ("vie_head_create", "vie_head_destroy", "vie_head_get_props", "vie_hea
            "vie_head_topk_sparse", "vie_head_topk_host", "vie_sample_topk", "vie_head_topk_sample",
            "vie_head_create_e4m3", "vie_head_export_e4m3", "vie_head_topk_many", "vie_recall_hits",
            "vie_head_topk_noalloc", "vie_scatter_sparse_logits", "vie_device_status",
-           "vie_head_device_status", "vie_last_error")
+           "vie_head_device_status", "vie_last_error", "vie_set_launch_option", "vie_get_launch_option")
 
 
 class VieError(RuntimeError):
@@ -104,6 +116,8 @@ def load(path: str | None = None, build_if_missing: bool = True):
             "vie_device_status": ([P], ctypes.c_int),
             "vie_head_device_status": ([P, P], ctypes.c_int),
             "vie_last_error": ([], ctypes.c_char_p),
+            "vie_set_launch_option": ([ctypes.c_int, I32], ctypes.c_int),
+            "vie_get_launch_option": ([ctypes.c_int, ctypes.POINTER(I32)], ctypes.c_int),
         }
         for name, (args, res) in sig.items():
             fn = getattr(lib, name)
@@ -248,6 +262,40 @@ def vie_device_status(stream: int = 0) -> int:
 
 def vie_head_device_status(head: int, stream: int = 0) -> int:
     return load().vie_head_device_status(head, stream)
+
+
+def vie_set_launch_option(option: int, value: int) -> int:
+    return load().vie_set_launch_option(option, value)
+
+
+def vie_get_launch_option(option: int):
+    """Returns (status, value)."""
+    v = ctypes.c_int32(0)
+    st = load().vie_get_launch_option(option, ctypes.byref(v))
+    return st, v.value
+
+
+class launch_options:
+    """Context manager that sets launch options for its body and restores
+    the previous values afterwards, e.g.
+    ``with launch_options({VIE_OPT_TC_MIN_BATCH: 10**6}): ...`` keeps every
+    batch on the streaming kernel.  Options are process-wide."""
+
+    def __init__(self, values: dict):
+        self.values = dict(values)
+        self.saved = {}
+
+    def __enter__(self):
+        for o, v in self.values.items():
+            st, old = vie_get_launch_option(o)
+            check(st)
+            self.saved[o] = old
+            check(vie_set_launch_option(o, v))
+        return self
+
+    def __exit__(self, *exc):
+        for o, v in self.saved.items():
+            vie_set_launch_option(o, v)
 
 
 def check(status: int) -> None:

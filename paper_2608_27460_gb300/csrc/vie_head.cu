@@ -4,6 +4,7 @@
 #include <cuda_fp8.h>
 #include <cuda_runtime.h>
 
+#include <atomic>
 #include <climits>
 #include <cmath>
 #include <cstdarg>
@@ -179,30 +180,28 @@ int nb_cap_for(int d_pad, int mm) {
     return nb;
 }
 
-int env_int(const char *name, int dflt) {
-    const char *v = getenv(name);
-    return (v != nullptr && *v != 0) ? atoi(v) : dflt;
-}
-
-// Launch-shape knobs (they change speed, never results):
-//   VIE_STAGE_MIN_KB     smallest weight stage worth one bulk copy (48)
-//   VIE_STATIC_PCT       share of the chunks assigned statically, in % (85)
-//   VIE_POOL_DIV         pool pieces are chunks / this (1)
-//   VIE_TC_MIN_BATCH     smallest batch sent to the tensor-core path (2)
-//   VIE_TC_KPS           128-byte K-blocks per tensor-core ring stage (4)
-//   VIE_TC_MIN_BATCH_E4M3  the same threshold for e4m3 heads (1)
-//   VIE_HALF_ROWS        streaming projection by half-warps: 1 on, 0 off,
-//                        -1 when a row's last pass would leave half the lanes idle (-1)
-struct Knobs {
-    int stage_min_bytes, static_pct, tc_min_batch, tc_kps, pool_div, tc_min_batch_e4m3, half_rows;
+// Launch-shape options (they change speed, never results), set through
+// vie_set_launch_option.  Process-wide; each call reads them when it plans
+// its launches.  The defaults are the measured best shapes.
+struct OptionSpec {
+    int dflt, lo, hi;
 };
-const Knobs &knobs() {
-    static const Knobs k = {env_int("VIE_STAGE_MIN_KB", 48) * 1024, env_int("VIE_STATIC_PCT", 85),
-                            env_int("VIE_TC_MIN_BATCH", 2), env_int("VIE_TC_KPS", 4),
-                            env_int("VIE_POOL_DIV", 1), env_int("VIE_TC_MIN_BATCH_E4M3", 1),
-                            env_int("VIE_HALF_ROWS", -1)};
-    return k;
-}
+constexpr OptionSpec kOptionSpec[VIE_OPT_COUNT] = {
+    {48, 1, 227},      // VIE_OPT_STAGE_MIN_KB
+    {85, 0, 100},      // VIE_OPT_STATIC_PCT
+    {1, 1, 64},        // VIE_OPT_POOL_DIV
+    {2, 1, INT32_MAX}, // VIE_OPT_TC_MIN_BATCH
+    {4, 1, 4},         // VIE_OPT_TC_KPS
+    {1, 1, INT32_MAX}, // VIE_OPT_TC_MIN_BATCH_E4M3
+    {-1, -1, 1},       // VIE_OPT_HALF_ROWS
+    {1, 0, 1},         // VIE_OPT_HOST_H_DIRECT
+};
+std::atomic<int> g_options[VIE_OPT_COUNT] = {
+    {kOptionSpec[0].dflt}, {kOptionSpec[1].dflt}, {kOptionSpec[2].dflt}, {kOptionSpec[3].dflt},
+    {kOptionSpec[4].dflt}, {kOptionSpec[5].dflt}, {kOptionSpec[6].dflt}, {kOptionSpec[7].dflt}};
+static_assert(VIE_OPT_COUNT == 8, "one default per option");
+
+int opt(vie_launch_option o) { return g_options[o].load(std::memory_order_relaxed); }
 
 // Whether the streaming projection gives each half-warp its own row: with
 // 16-byte chunks c per row, a full warp's last pass over a row runs c mod 32
@@ -210,7 +209,7 @@ const Knobs &knobs() {
 // lane slot per row pair.  Needs two rows per warp (R >= 2).
 int half_rows_for(int r, int chunks) {
     if (r < 2) return 0;
-    const int v = knobs().half_rows;
+    const int v = opt(VIE_OPT_HALF_ROWS);
     if (v >= 0) return v > 0 ? 1 : 0;
     const int tail = chunks % 32;
     return (tail != 0 && tail <= 16) ? 1 : 0;
@@ -218,8 +217,8 @@ int half_rows_for(int r, int chunks) {
 
 // Rows of a pool piece for stages of rs rows.
 int pool_rows_for(int rs) {
-    int div = knobs().pool_div;
-    div = div < 1 ? 1 : (div > rs ? rs : div);
+    int div = opt(VIE_OPT_POOL_DIV);
+    div = div > rs ? rs : div;
     return (rs + div - 1) / div;
 }
 
@@ -233,7 +232,7 @@ struct LaunchShape {
 bool pick_shape(int nb, int d_pad, int row_bytes, LaunchShape *out) {
     const int r_max = nb == 1 ? 8 : 4;  // 8 rows per warp only for single-query launches
     int r = 1;
-    while (r < r_max && 8 * r * row_bytes < knobs().stage_min_bytes) r <<= 1;
+    while (r < r_max && 8 * r * row_bytes < opt(VIE_OPT_STAGE_MIN_KB) * 1024) r <<= 1;
     for (int rs = 8 * r; rs >= 1; --rs) {
         for (int s = vie::kMaxStages; s >= 2; --s) {
             const vie::SmemLayout L(nb, d_pad, rs, s, row_bytes);
@@ -312,6 +311,26 @@ bool make_map_bf16(CUtensorMap *m, void *base, uint64_t rows, uint64_t cols, uin
 extern "C" {
 
 const char *vie_last_error(void) { return g_err; }
+
+vie_status vie_set_launch_option(vie_launch_option option, int32_t value) {
+    if (static_cast<int>(option) < 0 || option >= VIE_OPT_COUNT)
+        return fail(VIE_ERR_INVALID_ARG, "vie_set_launch_option: unknown option %d", static_cast<int>(option));
+    const OptionSpec &sp = kOptionSpec[option];
+    if (value == VIE_OPT_DEFAULT) value = sp.dflt;
+    if (value < sp.lo || value > sp.hi)
+        return fail(VIE_ERR_INVALID_ARG, "vie_set_launch_option: value %d of option %d outside [%d, %d]",
+                    value, static_cast<int>(option), sp.lo, sp.hi);
+    g_options[option].store(value, std::memory_order_relaxed);
+    return VIE_OK;
+}
+
+vie_status vie_get_launch_option(vie_launch_option option, int32_t *value) {
+    if (static_cast<int>(option) < 0 || option >= VIE_OPT_COUNT || value == nullptr)
+        return fail(VIE_ERR_INVALID_ARG, "vie_get_launch_option: bad option %d or NULL value",
+                    static_cast<int>(option));
+    *value = opt(option);
+    return VIE_OK;
+}
 
 static vie_status create_head(const void *W_out, int64_t V, int32_t d, vie_dtype dtype, bool e4m3,
                               vie_head **out) {
@@ -488,7 +507,7 @@ static int tc_group(int32_t batch, int32_t k, bool q8) {
 
 static bool use_tc(const vie_head *head, int32_t batch, int32_t k) {
     const bool q8 = head->scale != nullptr;
-    return head->tc_ready && batch >= (q8 ? knobs().tc_min_batch_e4m3 : knobs().tc_min_batch) &&
+    return head->tc_ready && batch >= (q8 ? opt(VIE_OPT_TC_MIN_BATCH_E4M3) : opt(VIE_OPT_TC_MIN_BATCH)) &&
            k <= vie::tc_max_k(32, q8) && head->d_pad >= (q8 ? 128 : 64);
 }
 
@@ -530,16 +549,15 @@ static vie_status run_topk_tc(const char *fn, vie_head *head, const float *h, in
     // resident in shared memory when they are small (e4m3 rows)
     int stages = 0, kps = 0, slots = 0;
     uint32_t smem = 0;
-    int kps_max = knobs().tc_kps;
-    kps_max = kps_max < 1 ? 1 : (kps_max > vie::kTcMaxKPS ? vie::kTcMaxKPS : kps_max);
+    int kps_max = opt(VIE_OPT_TC_KPS);
+    kps_max = kps_max > vie::kTcMaxKPS ? vie::kTcMaxKPS : kps_max;
     const int hres_bytes = tc_hres(head, nqt);
     for (int c = kps_max; c >= 1 && kps == 0; --c) {
         if (vie::tc_shape(nqt, q8, c, hres_bytes, &stages, &slots, &smem)) kps = c;
     }
     if (kps == 0) return fail(VIE_ERR_UNSUPPORTED, "%s: no tensor-core layout", fn);
     const int n_tiles = static_cast<int>((head->V + vie::kTcTile - 1) / vie::kTcTile);
-    int pct = knobs().static_pct;
-    pct = pct < 0 ? 0 : (pct > 100 ? 100 : pct);
+    const int pct = opt(VIE_OPT_STATIC_PCT);
     const int n_h = (q8 ? vie::kQ8Pieces : 2) * nqt;  // query rows: boxes of 16 / 32 / 64 / 128
     const CUtensorMap &mapH = head->mapH[n_h == 16 ? 0 : (n_h == 32 ? 1 : (n_h == 64 ? 2 : 3))];
     for (int q0 = 0; q0 < batch; q0 += nqt) {
@@ -619,8 +637,7 @@ static vie_status run_topk(const char *fn, vie_head *head, const float *h, int32
         p.rows_per_stage = shp.rs;
         p.stages = shp.stages;
         const int64_t n_chunks = (head->V + shp.rs - 1) / shp.rs;
-        int pct = knobs().static_pct;
-        pct = pct < 0 ? 0 : (pct > 100 ? 100 : pct);
+        const int pct = opt(VIE_OPT_STATIC_PCT);
         p.static_chunks = static_cast<int32_t>(n_chunks * pct / 100 / head->G);
         p.pool_rows = pool_rows_for(shp.rs);
         p.half_rows = half_rows_for(shp.r, head->d_pad / (head->scale != nullptr ? 16 : 8));
@@ -777,13 +794,12 @@ vie_status vie_head_topk_host(vie_head *head, const float *h_host, int32_t batch
     const size_t nh = static_cast<size_t>(batch) * head->d, no = static_cast<size_t>(batch) * k;
     // pinned buffers are used in place: the kernels read the queries from
     // host memory (measured faster than a copy in first) and the merging CTA
-    // writes the top-k there (no copies back); VIE_HOST_H_DIRECT=0 copies
-    // pinned queries in all the same
+    // writes the top-k there (no copies back); VIE_OPT_HOST_H_DIRECT = 0
+    // copies pinned queries in all the same
     int32_t *idx_dev = static_cast<int32_t *>(mapped_view(idx_host));
     float *logits_dev = static_cast<float *>(mapped_view(logits_host));
     const bool out_direct = idx_dev != nullptr && logits_dev != nullptr;
-    static const bool h_direct_knob = env_int("VIE_HOST_H_DIRECT", 1) != 0;
-    const float *h_dev = h_direct_knob ? static_cast<const float *>(mapped_view(h_host)) : nullptr;
+    const float *h_dev = opt(VIE_OPT_HOST_H_DIRECT) != 0 ? static_cast<const float *>(mapped_view(h_host)) : nullptr;
     if (h_dev == nullptr && head->stage_h_elems < nh) {
         cudaFree(head->stage_h);
         head->stage_h = nullptr;
@@ -948,6 +964,17 @@ extern "C" vie_status vie_head_topk_noalloc(const void *W_out, int64_t V, int32_
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return fail_cuda(e, "cudaGetDevice");
     if (dev < 0 || dev >= 64) return fail(VIE_ERR_UNSUPPORTED, "%s: device %d", fn, dev);
+    // the weights are streamed by bulk copies: device (or managed) memory of
+    // this device only (the query may be page-locked host memory)
+    cudaPointerAttributes pa;
+    e = cudaPointerGetAttributes(&pa, W_out);
+    if (e != cudaSuccess) {
+        cudaGetLastError();
+        return fail(VIE_ERR_INVALID_ARG, "%s: W_out is not a CUDA pointer", fn);
+    }
+    if ((pa.type != cudaMemoryTypeDevice && pa.type != cudaMemoryTypeManaged) || pa.device != dev)
+        return fail(VIE_ERR_INVALID_ARG, "%s: W_out must be device memory of the current device %d", fn,
+                    dev);
     NoAllocDevice &nd = g_noalloc[dev];
     std::call_once(nd.once, [&nd, dev]() {
         nd.setup_error = cudaGetSymbolAddress(reinterpret_cast<void **>(&nd.scratch), g_noalloc_scratch);
@@ -966,14 +993,23 @@ extern "C" vie_status vie_head_topk_noalloc(const void *W_out, int64_t V, int32_
     const int cap = nb_cap_for(d, mm);
     int nb_max = 1;
     while (nb_max < cap && nb_max < batch) nb_max <<= 1;
+    // lists [nb_max][G][k], then the heads [nb_max][G][kFastE], which the
+    // merge reads 16 bytes at a time: the list area is rounded up to an even
+    // number of keys so the heads start on a 16-byte boundary
+    const size_t list_keys = (static_cast<size_t>(nb_max) * G * k + 1) & ~static_cast<size_t>(1);
     const size_t lists_bytes =
-        static_cast<size_t>(nb_max) * G * (k + vie::kFastE) * sizeof(uint64_t);  // lists, heads
+        (list_keys + static_cast<size_t>(nb_max) * G * vie::kFastE) * sizeof(uint64_t);
     if (lists_bytes > kNoAllocScratchBytes - kNoAllocCounterBytes)
         return fail(VIE_ERR_UNSUPPORTED,
-                    "%s: needs %zu bytes of scratch (%d query slots x %d CTAs x (k=%d + %d) x 8), "
-                    "more than the fixed %zu; use vie_head_topk or a smaller batch or k",
+                    "%s: needs %zu bytes of scratch (%d query slots x %d CTAs x (k=%d + %d) x 8, "
+                    "lists rounded to 16 bytes), more than the fixed %zu; use vie_head_topk or a "
+                    "smaller batch or k",
                     fn, lists_bytes, nb_max, G, k, vie::kFastE,
                     kNoAllocScratchBytes - kNoAllocCounterBytes);
+    uint64_t *cand = reinterpret_cast<uint64_t *>(nd.scratch + kNoAllocCounterBytes);
+    uint64_t *heads = cand + list_keys;
+    if ((reinterpret_cast<uintptr_t>(cand) | reinterpret_cast<uintptr_t>(heads)) & 15u)
+        return fail(VIE_ERR_UNSUPPORTED, "%s: scratch lists not 16-byte aligned", fn);
 
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     uint32_t *counters = reinterpret_cast<uint32_t *>(nd.scratch);
@@ -998,13 +1034,12 @@ extern "C" vie_status vie_head_topk_noalloc(const void *W_out, int64_t V, int32_
         p.rows_per_stage = shp.rs;
         p.stages = shp.stages;
         const int64_t n_chunks = (V + shp.rs - 1) / shp.rs;
-        int pct = knobs().static_pct;
-        pct = pct < 0 ? 0 : (pct > 100 ? 100 : pct);
+        const int pct = opt(VIE_OPT_STATIC_PCT);
         p.static_chunks = static_cast<int32_t>(n_chunks * pct / 100 / G);
         p.pool_rows = pool_rows_for(shp.rs);
         p.half_rows = half_rows_for(shp.r, d / 8);
-        p.cand = reinterpret_cast<uint64_t *>(nd.scratch + kNoAllocCounterBytes);
-        p.heads = p.cand + static_cast<size_t>(nb_max) * G * k;
+        p.cand = cand;
+        p.heads = heads;
         p.ticket = counters;
         p.next_chunk = counters + 2;
         p.err = nd.flag;

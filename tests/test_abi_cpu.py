@@ -134,3 +134,34 @@ def test_product_path_does_not_import_the_oracle():
                 text = open(os.path.join(dirpath, f)).read()
                 assert not re.search(r"^\s*(import|from)\s+oracle\b", text, re.M), f
                 assert "oracle.c" not in text and "liboracle" not in text, f
+
+
+def test_launch_options_hook(lib):
+    """The launch options are set only through the explicit hook: defaults
+    as documented, out-of-range values rejected (the option keeps its value),
+    VIE_OPT_DEFAULT restores, the context manager puts values back; the
+    library reads no environment variable."""
+    defaults = {vie.VIE_OPT_STAGE_MIN_KB: 48, vie.VIE_OPT_STATIC_PCT: 85, vie.VIE_OPT_POOL_DIV: 1,
+                vie.VIE_OPT_TC_MIN_BATCH: 2, vie.VIE_OPT_TC_KPS: 4, vie.VIE_OPT_TC_MIN_BATCH_E4M3: 1,
+                vie.VIE_OPT_HALF_ROWS: -1, vie.VIE_OPT_HOST_H_DIRECT: 1}
+    assert len(defaults) == vie.VIE_OPT_COUNT
+    for o, v in defaults.items():
+        assert vie.vie_get_launch_option(o) == (vie.VIE_OK, v)
+    assert vie.vie_set_launch_option(vie.VIE_OPT_STATIC_PCT, 101) == vie.VIE_ERR_INVALID_ARG
+    assert vie.vie_set_launch_option(vie.VIE_OPT_HALF_ROWS, -2) == vie.VIE_ERR_INVALID_ARG
+    assert vie.vie_set_launch_option(vie.VIE_OPT_TC_KPS, 0) == vie.VIE_ERR_INVALID_ARG
+    assert vie.vie_set_launch_option(vie.VIE_OPT_COUNT, 1) == vie.VIE_ERR_INVALID_ARG
+    assert vie.vie_set_launch_option(-1, 1) == vie.VIE_ERR_INVALID_ARG
+    assert vie.vie_get_launch_option(vie.VIE_OPT_STATIC_PCT) == (vie.VIE_OK, 85)
+    assert vie.vie_set_launch_option(vie.VIE_OPT_STATIC_PCT, 50) == vie.VIE_OK
+    assert vie.vie_get_launch_option(vie.VIE_OPT_STATIC_PCT) == (vie.VIE_OK, 50)
+    assert vie.vie_set_launch_option(vie.VIE_OPT_STATIC_PCT, vie.VIE_OPT_DEFAULT) == vie.VIE_OK
+    assert vie.vie_get_launch_option(vie.VIE_OPT_STATIC_PCT) == (vie.VIE_OK, 85)
+    with vie.launch_options({vie.VIE_OPT_HALF_ROWS: 1, vie.VIE_OPT_TC_MIN_BATCH: 1000}):
+        assert vie.vie_get_launch_option(vie.VIE_OPT_HALF_ROWS) == (vie.VIE_OK, 1)
+        assert vie.vie_get_launch_option(vie.VIE_OPT_TC_MIN_BATCH) == (vie.VIE_OK, 1000)
+    for o, v in defaults.items():
+        assert vie.vie_get_launch_option(o) == (vie.VIE_OK, v)
+    for src in ("vie_head.cu", "vie_tc_topk.cu", "vie_tc_topk_e4m3.cu", "vie_sample.cu", "vie_recall.cu"):
+        text = open(os.path.join(ROOT, "paper_2608_27460_gb300", "csrc", src)).read()
+        assert "getenv" not in text, src

@@ -177,27 +177,15 @@ def test_tensor_core_error_against_the_sum_of_magnitudes(vie, batch):
     assert rel.max() <= 2.0**-14
 
 
-def test_streaming_kernel_on_e4m3_rows():
+def test_streaming_kernel_on_e4m3_rows(vie):
     """The same parity with every call forced onto the streaming CUDA-core
-    kernel (a fresh process: the path threshold is read once per process)."""
-    import os
-    import subprocess
-    import sys
-    here = os.path.dirname(os.path.abspath(__file__))
-    code = (
-        "import sys; sys.path[:0] = [%r, %r]\n"
-        "import test_gpu_e4m3 as t, paper_2608_27460_gb300 as vie\n"
-        "from gpu_cases import workload\n"
-        "vie.load()\n"
-        "for V, d, b, k in [(20011, 640, 1, 50), (30011, 1024, 8, 64), (20011, 2048, 3, 1)]:\n"
-        "    W, h = workload(V, d, b, seed=V + b)\n"
-        "    with t._head(vie, W) as head:\n"
-        "        assert head.plan(b, k).path == 0\n"
-        "    t._parity(vie, W, h, k, reps=2)\n"
-        "print('ok')\n") % (here, os.path.dirname(here))
-    env = dict(os.environ, VIE_TC_MIN_BATCH_E4M3="100000")
-    r = subprocess.run([sys.executable, "-c", code], env=env, capture_output=True, text=True, timeout=600)
-    assert r.returncode == 0 and r.stdout.strip().endswith("ok"), r.stdout + r.stderr
+    kernel through the launch-option hook."""
+    with vie.launch_options({vie.VIE_OPT_TC_MIN_BATCH_E4M3: 100000}):
+        for V, d, b, k in [(20011, 640, 1, 50), (30011, 1024, 8, 64), (20011, 2048, 3, 1)]:
+            W, h = workload(V, d, b, seed=V + b)
+            with _head(vie, W) as head:
+                assert head.plan(b, k).path == 0
+            _parity(vie, W, h, k, reps=2)
 
 
 @pytest.mark.parametrize("batch", [1, 3, 12])

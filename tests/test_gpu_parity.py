@@ -85,35 +85,24 @@ def test_tie_stress_duplicate_rows(vie):
 
 
 @pytest.mark.parametrize("half_rows", [0, 1])
-def test_streaming_row_mappings(half_rows):
+def test_streaming_row_mappings(vie, half_rows):
     """Both ways the streaming kernel spreads a stage over a warp (whole-warp
-    rows, or one row per half-warp), forced for every shape, with every batch
-    on the streaming kernel; duplicated rows must still tie bit for bit.  A
-    fresh process: the launch knobs are read once per process."""
-    import os
-    import subprocess
-    import sys
-    here = os.path.dirname(os.path.abspath(__file__))
-    code = (
-        "import sys; sys.path[:0] = [%r, %r]\n"
-        "import paper_2608_27460_gb300 as vie\n"
-        "from gpu_cases import assert_parity, to_device_bits, workload\n"
-        "vie.load()\n"
-        "for V, d, b, k, dup in [(20011, 640, 1, 50, 0.0), (20011, 640, 3, 1, 0.0),\n"
-        "                        (33333, 1152, 4, 50, 0.05), (4099, 100, 2, 50, 0.0),\n"
-        "                        (70001, 512, 8, 50, 0.05), (20011, 2048, 1, 64, 0.0)]:\n"
-        "    W, h = workload(V, d, b, seed=V + d + b, dup_frac=dup, planted=0.5 if dup else 0.0)\n"
-        "    with vie.Head(to_device_bits(W)) as head:\n"
-        "        assert head.plan(b, k).path == 0\n"
-        "    idx, val, _ = assert_parity(vie, W, h, k, reps=2)\n"
-        "    for q in range(b):\n"
-        "        for j in range(1, k):\n"
-        "            if val[q, j] == val[q, j - 1]:\n"
-        "                assert idx[q, j] > idx[q, j - 1]\n"
-        "print('ok')\n") % (here, os.path.dirname(here))
-    env = dict(os.environ, VIE_HALF_ROWS=str(half_rows), VIE_TC_MIN_BATCH="100000")
-    r = subprocess.run([sys.executable, "-c", code], env=env, capture_output=True, text=True, timeout=600)
-    assert r.returncode == 0 and r.stdout.strip().endswith("ok"), r.stdout + r.stderr
+    rows, or one row per half-warp), forced through the launch-option hook for
+    every shape, with every batch on the streaming kernel; duplicated rows
+    must still tie bit for bit."""
+    opts = {vie.VIE_OPT_HALF_ROWS: half_rows, vie.VIE_OPT_TC_MIN_BATCH: 100000}
+    with vie.launch_options(opts):
+        for V, d, b, k, dup in [(20011, 640, 1, 50, 0.0), (20011, 640, 3, 1, 0.0),
+                                (33333, 1152, 4, 50, 0.05), (4099, 100, 2, 50, 0.0),
+                                (70001, 512, 8, 50, 0.05), (20011, 2048, 1, 64, 0.0)]:
+            W, h = workload(V, d, b, seed=V + d + b, dup_frac=dup, planted=0.5 if dup else 0.0)
+            with vie.Head(to_device_bits(W)) as head:
+                assert head.plan(b, k).path == 0
+            idx, val, _ = assert_parity(vie, W, h, k, reps=2)
+            for q in range(b):
+                for j in range(1, k):
+                    if val[q, j] == val[q, j - 1]:
+                        assert idx[q, j] > idx[q, j - 1]
 
 
 def test_negative_zero_ranks_as_zero(vie):
