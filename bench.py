@@ -1,11 +1,15 @@
 #!/usr/bin/env python3
 """Benchmark of the exact output head: microseconds per decode step.
 
-One step = the whole hot path over one batch of queries in one launch
-(vie_head_topk_sparse): the streaming projection, the per-CTA and global
-top-k, and the sparse -inf logit tensor.  Default workload: the Qwen3-0.6B-shaped head
-(W_out bf16 [151936, 1024] = 311 MB, larger than the 129 MB L2), batch 1,
-k = 50, seeded synthetic weights and queries (no real checkpoint here).
+One step = the whole hot path over one batch of queries (vie_head_topk_sparse):
+the projection z = W_out h, the per-CTA and global top-k, and the sparse -inf
+logit tensor.  Headline workload: the largest batch-1 head of the paper's
+models, the Gemma-3-1B-shaped head (W_out bf16 [262144, 1152] = 604 MB, larger
+than the 129 MB L2), batch 1, k = 50, seeded synthetic weights and queries (no
+real checkpoint here).  Every timed step's top-k is checked against the
+oracle.  The same line carries ``per_config``: every workload, batch and k of
+the five model shapes, each timed the same way and parity-checked on every
+step (1000 distinct decode steps on the Qwen3-0.6B shape).
 
 Prints one JSON line (rank 0).  ``--impl reference`` times the CPU oracle on
 the same workload instead: there is no other implementation of this head to
@@ -51,15 +55,22 @@ KERNEL_SOURCES = {
 def parse_args(argv=None):
     ap = argparse.ArgumentParser(description=__doc__)
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=2000)
-    ap.add_argument("--warmup", type=int, default=200)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--workload", default="qwen3-0.6b", choices=sorted(synth.HEADS))
+    ap.add_argument("--workload", default="gemma3-1b", choices=sorted(synth.HEADS))
     ap.add_argument("--batch", type=int, default=1)
     ap.add_argument("--k", type=int, default=50)
     ap.add_argument("--queries", type=int, default=64, help="distinct resident queries cycled")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--cpu-seconds", type=float, default=15.0, help="oracle sample budget")
+    ap.add_argument("--cpu-seconds", type=float, default=10.0, help="oracle sample budget")
+    ap.add_argument("--no-per-config", action="store_true",
+                    help="skip the per_config sweep over every workload, batch and k")
+    ap.add_argument("--config-steps", type=int, default=50,
+                    help="timed steps of each per_config entry (each parity-checked)")
+    ap.add_argument("--long-parity-steps", type=int, default=1000,
+                    help="distinct decode steps of the Qwen3-0.6B-shaped b = 1 entry, every one "
+                         "timed and checked against the oracle")
     ap.add_argument("--e2e-steps", type=int, default=200)
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--storage", choices=["bf16", "e4m3"], default="bf16",
@@ -414,8 +425,190 @@ def workload_config(args, shape):
 
 
 # ---------------------------------------------------------------------------
+class Flush:
+    """A 256 MB read between timed steps: W_out (and everything else) leaves
+    the 129 MB L2 with clean lines, as the other layers of a decode step
+    would leave it."""
+
+    def __init__(self, torch, dev, enabled=True):
+        self.torch = torch
+        self.buf = torch.ones(256 * 1024 * 1024 // 4, dtype=torch.float32, device=dev) if enabled else None
+        self.sink = torch.empty((), dtype=torch.float32, device=dev)
+
+    def __call__(self):
+        if self.buf is not None:
+            self.torch.sum(self.buf, dim=0, out=self.sink)
+
+
+def timed_steps(torch, launch, K, W, flush, stream):
+    """Per-step device time (µs) of K steps launch(0..K-1), each bracketed by
+    CUDA events on the launching stream after the L2 flush.  The W warm-up
+    steps run the identical sequence (flush, event, launch, event) so the
+    first timed steps pay nothing the others do not."""
+    for i in range(W):
+        flush()
+        a, c = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        launch(i, warm=True)
+        c.record(stream)
+    torch.cuda.synchronize()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
+    for i in range(K):
+        flush()
+        ev[i][0].record(stream)
+        launch(i, warm=False)
+        ev[i][1].record(stream)
+    torch.cuda.synchronize()
+    return [a.elapsed_time(c) * 1e3 for a, c in ev]
+
+
+def us_stats(us):
+    return {"us_mean": round(statistics.mean(us), 3), "us_p50": round(float(np.percentile(us, 50)), 3),
+            "us_p10_p90": [round(float(np.percentile(us, q)), 2) for q in (10, 90)]}
+
+
+def kernel_name(plan_path, storage):
+    e4m3 = storage == "e4m3"
+    if plan_path == 0:
+        return "stream_topk_e4m3" if e4m3 else "stream_topk"
+    return "tc_topk_e4m3" if e4m3 else "tc_topk"
+
+
+def check_steps(W, h, starts, b, k, idx_steps, val_steps, storage="bf16", chunk=64):
+    """Every timed step's top-k against the oracle: the oracle's fp64 logits
+    of each distinct query (in chunks), then the acceptance rule per query of
+    every step that used it.  Returns (all ok, steps checked, first failure)."""
+    sys.path.insert(0, os.path.join(ROOT, "tests"))
+    from acceptance import check_topk, oracle_order_top
+    logits = oracle_head(W, storage)[1]
+    need = sorted({starts[i % len(starts)] + q for i in range(idx_steps.shape[0]) for q in range(b)})
+    by_query = {}
+    for i in range(idx_steps.shape[0]):
+        q0 = starts[i % len(starts)]
+        for q in range(b):
+            by_query.setdefault(q0 + q, []).append((i, q))
+    ok, first = True, None
+    for c0 in range(0, len(need), chunk):
+        rows = need[c0:c0 + chunk]
+        z = logits(h[rows])
+        for r, row in enumerate(rows):
+            order = oracle_order_top(z[r], k)
+            for i, q in by_query[row]:
+                errs = check_topk(idx_steps[i, q], val_steps[i, q], z[r], k, order=order)
+                if errs and ok:
+                    ok, first = False, f"step {i} query {q}: {errs[0]}"
+    return ok, int(idx_steps.shape[0]), first
+
+
+def roofline_of(alg_bytes, us, peaks):
+    ach = alg_bytes / (us * 1e-6) / 1e9
+    return ach, ach / peaks["hbm_gbs"]
+
+
+def tensor_roofline(shape, props, b, plan, us, peaks, peak_src, e4m3):
+    """The tensor-core path against its tensor roofline as well: algorithmic
+    flops 2*V*d*b; the MMAs issue 2*V*d_pad*(columns per query: hi and lo
+    bf16 halves of h, or four e4m3 pieces) over the padded query group.  The
+    e4m3 peak is the measured bf16 peak times the nominal fp8 / bf16 ratio 2."""
+    cols = 4 if e4m3 else 2
+    alg_flops = 2.0 * shape.V * shape.d * b
+    per_group = -(-b // plan.groups)
+    nq_tile = max(4 if e4m3 else 8, 1 << (per_group - 1).bit_length())  # the tile the library picked
+    issued = 2.0 * shape.V * props.d_pad * cols * nq_tile * plan.groups
+    tf = alg_flops / (us * 1e-6) / 1e12
+    tpeak = peaks["bf16_tflops"] * (2.0 if e4m3 else 1.0)
+    return {"bound": "tensor", "achieved": round(tf, 2), "peak": round(tpeak, 1),
+            "unit": "TFLOP/s", "frac": round(tf / tpeak, 5),
+            "issued_mma_tflops": round(issued / (us * 1e-6) / 1e12, 2),
+            "peak_source": peak_src + (" (bf16 x 2 for e4m3)" if e4m3 else ""),
+            "operands": "e4m3 x e4m3 (kind::f8f6f4)" if e4m3 else "bf16 x bf16 (kind::f16)"}
+
+
+def config_entry(torch, vie, dev, stream, flush, name, b, k, steps, warmup, n_batches, peaks,
+                 peak_src, cache, seed):
+    """One per_config entry: the workload's head (weights drawn once per
+    workload and kept in `cache` for its other batches), `steps` timed decode
+    steps cycling n_batches distinct query batches, every step's top-k
+    checked against the oracle."""
+    shape = synth.HEADS[name]
+    if cache.get("name") != name:
+        if cache.get("head") is not None:
+            cache["head"].close()
+        cache.clear()
+        W, _, meta, _ = synth.make_head(shape, seed=seed, n_queries=1)
+        Wd = torch.from_numpy(W.view(np.int16)).to(dev)
+        cache.update(name=name, W=W, meta=meta, head=vie.Head(Wd))
+        del Wd
+    W, head = cache["W"], cache["head"]
+    nq = n_batches * b
+    offset = synth.HEAD_ORDER.index(shape.name) if shape.name in synth.HEAD_ORDER else len(synth.HEAD_ORDER)
+    h, _ = synth.make_queries(W, nq, seed + 2000 + 97 * b + k + offset,
+                              planted_frac=0.25 if shape.dup_frac > 0 else 0.0,
+                              dup_src=cache["meta"]["dup_src"])
+    hd = torch.from_numpy(h).to(dev)
+    starts = [j * b for j in range(n_batches)]
+    idx_steps = torch.empty((steps, b, k), dtype=torch.int32, device=dev)
+    val_steps = torch.empty((steps, b, k), dtype=torch.float32, device=dev)
+    sparse = torch.empty((b, shape.V), dtype=torch.float32, device=dev)
+    sptr = int(stream.cuda_stream)
+
+    def launch(i, warm):
+        q0 = starts[i % n_batches]
+        j = i % steps
+        vie.check(vie.vie_head_topk_sparse(head.handle, hd[q0].data_ptr(), b, k, idx_steps[j].data_ptr(),
+                                           val_steps[j].data_ptr(), sparse.data_ptr(), sptr))
+
+    us = timed_steps(torch, launch, steps, warmup, flush, stream)
+    vie.check(head.device_status())
+    plan = head.plan(b, k)
+    props = head.props
+    alg = props.weight_bytes + b * shape.d * 4 + b * k * 8
+    mean = statistics.mean(us)
+    ach, frac = roofline_of(alg, mean, peaks)
+    kern = kernel_name(plan.path, "bf16")
+    traffic, prof = profiled_traffic(kern, name, b, k)
+    ok, n_checked, first = check_steps(W, h, starts, b, k, idx_steps.cpu().numpy(), val_steps.cpu().numpy())
+    e = {"workload": name, "V": shape.V, "d": shape.d, "batch": b, "k": k,
+         "path": "streaming" if plan.path == 0 else "tensor-core", "launches_per_step": plan.launches,
+         "steps": steps, **us_stats(us),
+         "roofline": {"bound": "hbm", "achieved": round(ach, 1), "frac": round(frac, 4),
+                      "frac_of_nominal_8tbs": round(ach / NOMINAL_HBM_GBS, 4),
+                      "frac_at_p50": round(roofline_of(alg, float(np.percentile(us, 50)), peaks)[1], 4),
+                      "algorithmic_bytes_per_launch": alg, "traffic": traffic,
+                      "profile": os.path.relpath(prof, ROOT) if prof else None},
+         "bar_80pct_of_8tbs_us": round(props.weight_bytes / (0.8 * NOMINAL_HBM_GBS * 1e9) * 1e6, 2),
+         "parity": {"ok": bool(ok), "steps_checked": n_checked, "distinct_batches": n_batches,
+                    **({"first_failure": first} if first else {})}}
+    if plan.path == 1:
+        e["roofline_tensor"] = tensor_roofline(shape, props, b, plan, mean, peaks, peak_src, False)
+    del hd, idx_steps, val_steps, sparse
+    return e
+
+
+# every workload, batch and k of the five model shapes (Section 4's models)
+PER_CONFIG = [("gemma3-270m", 1, 50), ("qwen3-0.6b", 1, 50),
+              ("llama3.2-1b", 1, 50), ("llama3.2-1b", 1, 1), ("llama3.2-1b", 4, 50), ("llama3.2-1b", 4, 1),
+              ("gemma3-1b", 1, 50), ("gemma3-1b", 2, 50), ("gemma3-1b", 4, 50), ("gemma3-1b", 8, 50),
+              ("gemma3-1b-ties", 1, 50), ("gemma3-1b-ties", 2, 50), ("gemma3-1b-ties", 4, 50),
+              ("gemma3-1b-ties", 8, 50), ("llama3.2-3b", 16, 50), ("llama3.2-3b", 64, 50)]
+
+
+def per_config_sweep(args, torch, vie, dev, stream, flush, peaks, peak_src, cache):
+    out = []
+    for name, b, k in PER_CONFIG:
+        steps, nb = args.config_steps, (8 if b < 4 else (4 if b < 16 else 2))
+        if name == "qwen3-0.6b" and b == 1 and args.long_parity_steps > 0:
+            steps = nb = args.long_parity_steps  # the 1000-step config: every step a new query
+        out.append(config_entry(torch, vie, dev, stream, flush, name, b, k, steps, 10, nb, peaks,
+                                peak_src, cache, args.seed))
+    if cache.get("head") is not None:
+        cache["head"].close()
+    return out
+
+
 def main(argv=None):
     args = parse_args(argv)
+    args.warmup = max(args.warmup, 3)
     rank, world, local = dist_env()
     if args.impl == "reference":
         return run_reference(args, rank, world)
@@ -432,14 +625,15 @@ def main(argv=None):
 
     shape = synth.HEADS[args.workload]
     nq = max(args.queries, args.batch)
-    W, h, _, _ = synth.make_head(shape, seed=args.seed + rank * 7919, n_queries=nq)
+    W, h, meta, _ = synth.make_head(shape, seed=args.seed + rank * 7919, n_queries=nq)
     Wd = torch.from_numpy(W.view(np.int16)).to(dev)
     head = vie.Head(Wd, storage=args.storage)
     del Wd
     hd = torch.from_numpy(h).to(dev)
     b, k, V = args.batch, args.k, shape.V
-    idx = torch.empty((b, k), dtype=torch.int32, device=dev)
-    val = torch.empty((b, k), dtype=torch.float32, device=dev)
+    K = args.steps
+    idx_steps = torch.empty((K, b, k), dtype=torch.int32, device=dev)  # each timed step's own top-k
+    val_steps = torch.empty((K, b, k), dtype=torch.float32, device=dev)
     sparse = torch.empty((b, V), dtype=torch.float32, device=dev)
     stream = torch.cuda.current_stream(dev)
     sptr = int(stream.cuda_stream)
@@ -448,68 +642,53 @@ def main(argv=None):
     prob = torch.empty((b,), dtype=torch.float32, device=dev)
     SAMPLING = (0.8, 0.9, 0.05)  # temperature, top-p, min-p
 
-    def head_call(i, stream_ptr=None):
+    def head_call(i, stream_ptr=None, slot=None):
         q0 = starts[i % nq]
         sp = sptr if stream_ptr is None else stream_ptr
+        j = (i % K) if slot is None else slot
         if args.sample:
             vie.check(vie.vie_head_topk_sample(head.handle, hd[q0].data_ptr(), b, k, *SAMPLING,
-                                               args.seed, i, idx.data_ptr(), val.data_ptr(),
+                                               args.seed, i, idx_steps[j].data_ptr(), val_steps[j].data_ptr(),
                                                sparse.data_ptr(), tok.data_ptr(), prob.data_ptr(), sp))
         else:
-            vie.check(vie.vie_head_topk_sparse(head.handle, hd[q0].data_ptr(), b, k, idx.data_ptr(),
-                                               val.data_ptr(), sparse.data_ptr(), sp))
+            vie.check(vie.vie_head_topk_sparse(head.handle, hd[q0].data_ptr(), b, k, idx_steps[j].data_ptr(),
+                                               val_steps[j].data_ptr(), sparse.data_ptr(), sp))
 
-    def step(i):
-        head_call(i)
-
+    flush = Flush(torch, dev, enabled=args.l2 == "flush")
     sampler = ClockSampler(gpu_id_for_smi(local)) if rank == 0 else None
     if sampler:
         sampler.start()
-    for i in range(args.warmup):
-        step(i)
-    torch.cuda.synchronize()
-    vie.check(head.device_status())
-
-    K = args.steps
-    flush = torch.ones(256 * 1024 * 1024 // 4, dtype=torch.float32, device=dev) \
-        if args.l2 == "flush" else None
-    flush_sink = torch.empty((), dtype=torch.float32, device=dev)
-    ev_a = [torch.cuda.Event(enable_timing=True) for _ in range(K)]
-    ev_b = [torch.cuda.Event(enable_timing=True) for _ in range(K)]
-    start = torch.cuda.Event(enable_timing=True)
-    end = torch.cuda.Event(enable_timing=True)
     if world > 1:
         torch.distributed.barrier()
     torch.cuda.synchronize()
     t_wall0 = time.time()
-    start.record(stream)
-    for i in range(K):
-        q0 = starts[i % nq]
-        if flush is not None:
-            torch.sum(flush, dim=0, out=flush_sink)  # reads 256 MB: W_out leaves L2
-        ev_a[i].record(stream)
-        head_call(i)
-        ev_b[i].record(stream)
-    end.record(stream)
-    torch.cuda.synchronize()
+    if args.l2 == "flush":
+        kern_us = timed_steps(torch, lambda i, warm: head_call(i), K, args.warmup, flush, stream)
+        step_us = statistics.mean(kern_us)  # the flush between steps is not head time
+    else:
+        for i in range(args.warmup):
+            head_call(i)
+        torch.cuda.synchronize()
+        a, c = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for i in range(K):
+            head_call(i)
+        c.record(stream)
+        torch.cuda.synchronize()
+        step_us = a.elapsed_time(c) * 1e3 / K
+        kern_us = [step_us]
     t_wall1 = time.time()
     if world > 1:
         torch.distributed.barrier()
-    total_ms = start.elapsed_time(end)
-    kern_ms = [a.elapsed_time(c) for a, c in zip(ev_a, ev_b)]
     clocks = sampler.stop() if sampler else []
     vie.check(head.device_status())
-
-    if flush is not None:
-        step_us = statistics.mean(kern_ms) * 1e3  # the flush between steps is not head time
-    else:
-        step_us = total_ms * 1e3 / K
+    idx_h, val_h = idx_steps.cpu().numpy(), val_steps.cpu().numpy()
     step_us = rank_max(step_us, world, dev)  # the slowest rank
 
     # end-to-end through the public API with host buffers: each step is one
-    # vie_head_topk_host call, which copies that step's h in from pinned host
-    # memory, runs the head (sparse tensor included) and copies the top-k
-    # (indices + logits) back to pinned host memory before it returns
+    # vie_head_topk_host call, which reads that step's h from pinned host
+    # memory, runs the head (sparse tensor included) and leaves the top-k
+    # (indices + logits) in pinned host memory before it returns
     h_host = torch.from_numpy(h).pin_memory()
     idx_host = torch.empty((b, k), dtype=torch.int32).pin_memory()
     val_host = torch.empty((b, k), dtype=torch.float32).pin_memory()
@@ -538,29 +717,29 @@ def main(argv=None):
 
     props = head.props
     peaks, peak_src = measured_peaks()
-    kern_us = statistics.mean(kern_ms) * 1e3
+    mean_us = statistics.mean(kern_us)
     w_bytes = props.weight_bytes  # bf16: V*d_pad*2; e4m3: V*d_pad + V*4 (codes and scales)
     alg_bytes = w_bytes + b * shape.d * 4 + b * k * 8
-    achieved = alg_bytes / (kern_us * 1e-6) / 1e9
+    achieved = alg_bytes / (mean_us * 1e-6) / 1e9
     plan = head.plan(b, k)
     e4m3 = args.storage == "e4m3"
-    kernel = ("stream_topk_e4m3" if e4m3 else "stream_topk") if plan.path == 0 \
-        else ("tc_topk_e4m3" if e4m3 else "tc_topk")
+    kernel = kernel_name(plan.path, args.storage)
     traffic, prof_path = profiled_traffic(kernel, args.workload, b, k)
     value = whole_job_us_per_step(step_us, world)
     launches_per_step = plan.launches + (1 if args.sample else 0)
-    graph_info = None if args.no_graph else graph_leg(torch, head_call, flush, flush_sink, stream, head, vie,
-                                                      min(K, 500))
+    graph_info = None if args.no_graph else graph_leg(
+        torch, lambda i, sp: head_call(i, sp, slot=0), flush.buf, flush.sink, stream, head, vie, min(K, 500))
     sample_info = None
     if args.sample:
         # the sampling kernel alone, on this step's candidates, back to back
+        i0, v0 = idx_steps[0], val_steps[0]
         sa, sb = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         for i in range(20):
-            vie.check(vie.vie_sample_topk(idx.data_ptr(), val.data_ptr(), b, k, *SAMPLING, args.seed, i,
+            vie.check(vie.vie_sample_topk(i0.data_ptr(), v0.data_ptr(), b, k, *SAMPLING, args.seed, i,
                                           tok.data_ptr(), prob.data_ptr(), sptr))
         sa.record(stream)
         for i in range(200):
-            vie.check(vie.vie_sample_topk(idx.data_ptr(), val.data_ptr(), b, k, *SAMPLING, args.seed, i,
+            vie.check(vie.vie_sample_topk(i0.data_ptr(), v0.data_ptr(), b, k, *SAMPLING, args.seed, i,
                                           tok.data_ptr(), prob.data_ptr(), sptr))
         sb.record(stream)
         torch.cuda.synchronize()
@@ -581,18 +760,20 @@ def main(argv=None):
         "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": peaks["hbm_gbs"],
                      "unit": "GB/s", "frac": round(achieved / peaks["hbm_gbs"], 4),
                      "traffic": traffic, "peak_source": peak_src,
-                     "kernel": ("stream_topk_kernel" + (" (e4m3 rows)" if args.storage == "e4m3" else ""))
+                     "kernel": ("stream_topk_kernel" + (" (e4m3 rows)" if e4m3 else ""))
                                if plan.path == 0 else "tc_topk_kernel (step: prep + projection + merge)",
                      "profile": os.path.relpath(prof_path, ROOT) if prof_path else None,
-                     "kernel_us": round(kern_us, 3),
+                     "kernel_us": round(mean_us, 3),
+                     "kernel_us_p50": round(float(np.percentile(kern_us, 50)), 3),
                      "algorithmic_bytes_per_launch": alg_bytes,
                      "frac_of_nominal_8tbs": round(achieved / NOMINAL_HBM_GBS, 4),
-                     "w_only_gbs": round(w_bytes / (kern_us * 1e-6) / 1e9, 1),
-                     "kernel_us_p10_p50_p90": [round(float(np.percentile(kern_ms, q)) * 1e3, 2)
+                     "w_only_gbs": round(w_bytes / (mean_us * 1e-6) / 1e9, 1),
+                     "kernel_us_p10_p50_p90": [round(float(np.percentile(kern_us, q)), 2)
                                                for q in (10, 50, 90)]},
-        "e2e": {"value": round(whole_job_us_per_step(e2e_us, world), 3), "unit": UNIT, "h2d_bytes_per_step": b * shape.d * 4,
-                "d2h_bytes_per_step": b * k * 8, "api": "vie_head_topk_host (pinned host h read and "
-                "top-k written in place by the kernels over NVLink-C2C, synchronised)",
+        "e2e": {"value": round(whole_job_us_per_step(e2e_us, world), 3), "unit": UNIT,
+                "h2d_bytes_per_step": b * shape.d * 4, "d2h_bytes_per_step": b * k * 8,
+                "api": "vie_head_topk_host (pinned host h read and top-k written in place by the "
+                       "kernels over NVLink-C2C, synchronised)",
                 "clock": "host wall clock over the steps"},
         "gpu_launches": K * launches_per_step,
         **({"sampling": sample_info} if sample_info else {}),
@@ -601,47 +782,37 @@ def main(argv=None):
         "clocks": ClockSampler.summarize(clocks, t_wall0, t_wall1),
     }
     if plan.path == 1:
-        # the tensor-core path against its tensor roofline as well: algorithmic
-        # flops 2*V*d*b; the MMAs issue 2*V*d_pad*(columns per query: hi and lo
-        # bf16 halves of h, or four e4m3 pieces) over the padded query group.
-        # The e4m3 peak is the measured bf16 peak times the nominal fp8 / bf16
-        # ratio of 2.
-        cols = 4 if e4m3 else 2
-        alg_flops = 2.0 * shape.V * shape.d * b
-        per_group = -(-b // plan.groups)
-        nq_tile = max(4 if e4m3 else 8, 1 << (per_group - 1).bit_length())  # the tile the library picked
-        issued = 2.0 * shape.V * props.d_pad * cols * nq_tile * plan.groups
-        tf = alg_flops / (kern_us * 1e-6) / 1e12
-        tpeak = peaks["bf16_tflops"] * (2.0 if e4m3 else 1.0)
-        line["roofline_tensor"] = {
-            "bound": "tensor", "achieved": round(tf, 2), "peak": round(tpeak, 1),
-            "unit": "TFLOP/s", "frac": round(tf / tpeak, 5),
-            "issued_mma_tflops": round(issued / (kern_us * 1e-6) / 1e12, 2),
-            "peak_source": peak_src + (" (bf16 x 2 for e4m3)" if e4m3 else ""),
-            "operands": "e4m3 x e4m3 (kind::f8f6f4)" if e4m3 else "bf16 x bf16 (kind::f16)"}
+        line["roofline_tensor"] = tensor_roofline(shape, props, b, plan, mean_us, peaks, peak_src, e4m3)
+    if world == 1:
+        # every timed step's top-k against the oracle (the queries it used)
+        ok, n_checked, first = check_steps(W, h, starts, b, k, idx_h, val_h, args.storage)
+        line["parity"] = {"ok": bool(ok), "steps_checked": n_checked,
+                          "distinct_queries": len({starts[i % nq] for i in range(K)}) * b,
+                          **({"first_failure": first} if first else {})}
     if not args.no_cpu_baseline and world == 1:
-        us, n, threads, results = cpu_oracle_sample(W, h, k, args.cpu_seconds, b, args.storage)
+        us, n, threads, _ = cpu_oracle_sample(W, h, k, args.cpu_seconds, b, args.storage)
         us1, n1 = cpu_oracle_single_thread(W, h, k, b, args.storage)
         line["cpu_baseline"] = {"value": round(us, 1), "unit": UNIT, "cores": threads, "kind": "oracle",
                                 "sample": f"{n} decode steps (batch {b}) of the same workload in "
                                           f"{args.cpu_seconds:.0f} s: fp64 projection, full sort, "
                                           "sparse tensor",
                                 "single_core": {"value": round(us1, 1), "unit": UNIT, "steps": n1}}
-        # two of the sampled steps double as a parity check of the device path
-        sys.path.insert(0, os.path.join(ROOT, "tests"))
-        import oracle
-        from acceptance import check_topk
-        ok = True
-        logits = oracle_head(W, args.storage)[1]
-        for q0 in list(results)[:2]:
-            gi, gv = head.topk(hd[q0:q0 + b], k)
-            torch.cuda.synchronize()
-            z = logits(h[q0:q0 + b])
-            for q in range(b):
-                ok &= not check_topk(gi.cpu().numpy()[q], gv.cpu().numpy()[q], z[q], k)
-        line["parity_sample_ok"] = bool(ok)
+    del hd, idx_steps, val_steps, sparse
+    if world == 1 and not args.no_per_config and args.storage == "bf16" and not args.sample:
+        t_pc = time.time()
+        # the headline's head (same seed, same weights) serves its workload's entries
+        cache = {"name": args.workload, "W": W, "meta": meta, "head": head} if args.seed == 0 else {}
+        if not cache:
+            head.close()
+        line["per_config"] = per_config_sweep(args, torch, vie, dev, stream, flush, peaks, peak_src,
+                                              cache)
+        line["per_config_note"] = (
+            "each entry: its own seeded head, steps timed like the headline (L2 flushed, CUDA events "
+            "around each launch, identical warm-up), every step's top-k checked against the oracle; "
+            f"sweep took {time.time() - t_pc:.0f} s")
+    else:
+        head.close()
     print(json.dumps(line), flush=True)
-    head.close()
     if world > 1:
         torch.distributed.destroy_process_group()
     return 0

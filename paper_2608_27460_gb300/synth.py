@@ -80,13 +80,25 @@ def make_weights(V: int, d: int, seed: int, dup_frac: float = 0.0,
     variant (empty arrays otherwise)."""
     rng = rng_for(seed)
     W = np.empty((V, d), dtype=np.uint16)
+    # chunk buffers are reused (fresh arrays per chunk cost more in page
+    # faults than the drawing itself); the values are those of
+    # f32_to_bf16_bits on each chunk, bit for bit
+    g_buf = np.empty((min(row_chunk, V), d), dtype=np.float32)
+    t_buf = np.empty((min(row_chunk, V), d), dtype=np.uint32)
     for r0 in range(0, V, row_chunk):
         n = min(row_chunk, V - r0)
-        g = rng.standard_normal((n, d), dtype=np.float32)
+        g = g_buf[:n]
+        rng.standard_normal(out=g, dtype=np.float32)
         g *= np.float32(0.02)
         s = np.exp(rng.normal(0.0, 0.3, size=(n, 1))).astype(np.float32)
         g *= s
-        W[r0:r0 + n] = f32_to_bf16_bits(g)
+        u, t = g.view(np.uint32), t_buf[:n]
+        np.right_shift(u, np.uint32(16), out=t)  # round to nearest even: + 0x7FFF + lsb
+        t &= np.uint32(1)
+        t += np.uint32(0x7FFF)
+        t += u
+        t >>= np.uint32(16)
+        W[r0:r0 + n] = t
     dst = np.zeros(0, dtype=np.int64)
     src = np.zeros(0, dtype=np.int64)
     n_dup = int(np.floor(dup_frac * V))

@@ -25,6 +25,22 @@ def oracle_order(z_row: np.ndarray) -> np.ndarray:
     return np.lexsort((np.arange(len(z_row)), -z_row))
 
 
+def oracle_order_top(z_row: np.ndarray, k: int) -> np.ndarray:
+    """The first min(k + 1, V) entries of oracle_order(z_row), without sorting
+    all V rows: t = the (k+1)-th largest value; every row above t, then the
+    rows equal to t by ascending index, ordered by (z desc, index asc).
+    Exact, ties included (the partition is by value only)."""
+    V = len(z_row)
+    m = min(k + 1, V)
+    if m >= V:
+        return oracle_order(z_row)
+    t = np.partition(z_row, V - m)[V - m]  # the m-th largest value
+    above = np.flatnonzero(z_row > t)
+    at = np.flatnonzero(z_row == t)[: m - len(above)]  # ascending index
+    cand = np.concatenate([above, at])
+    return cand[np.lexsort((cand, -z_row[cand]))]
+
+
 def check_topk(idx, val, z_row, k, order=None):
     """Returns a list of failure messages (empty when the result is accepted)."""
     idx = np.asarray(idx).astype(np.int64).reshape(-1)

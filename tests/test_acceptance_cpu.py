@@ -71,3 +71,18 @@ def test_equal_values_need_ascending_index():
     z = np.array([1.0, 3.0, 3.0, 0.0])
     assert check_topk([1, 2], [3.0, 3.0], z, 2) == []
     assert check_topk([2, 1], [3.0, 3.0], z, 2)
+
+
+def test_partial_order_equals_full_order():
+    """oracle_order_top is the prefix of the full (z desc, index asc) order,
+    with exact ties at and around rank k, k = 1, k = V - 1 and k >= V."""
+    import numpy as np
+    from acceptance import oracle_order, oracle_order_top
+    rng = np.random.default_rng(5)
+    for trial in range(200):
+        V = int(rng.integers(1, 300))
+        z = rng.integers(-6, 6, size=V).astype(np.float64) if trial % 2 else rng.normal(size=V)
+        full = oracle_order(z)
+        for k in sorted({1, max(1, V // 3), max(1, V - 1), V, V + 2}):
+            got = oracle_order_top(z, k)
+            np.testing.assert_array_equal(got, full[:min(k + 1, V)])
