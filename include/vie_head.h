@@ -169,7 +169,11 @@ typedef enum {
                                       half-warp: 1 on, 0 off, -1 automatic       (-1)  */
     VIE_OPT_HOST_H_DIRECT = 7,     /* vie_head_topk_host reads page-locked
                                       queries in place: 1, or copies them: 0     (1)   */
-    VIE_OPT_COUNT = 8
+    VIE_OPT_EARLY_MERGE = 8,       /* single-query streaming launches with
+                                      k <= 64: one CTA merges the per-CTA lists
+                                      while the others still stream: 1, or the
+                                      last CTA to finish merges them all: 0      (1)   */
+    VIE_OPT_COUNT = 9
 } vie_launch_option;
 
 #define VIE_OPT_DEFAULT INT32_MIN /* value that restores an option's default */
@@ -371,7 +375,7 @@ vie_status vie_scatter_sparse_logits(const int32_t *idx, const float *logits, in
  * Scratch: one 1 MiB array per device (every GPU that loads the library keeps
  * it until the process exits), of which the first 256 bytes hold counters.
  * A call needs
- *   8 * (round_up_even(slots * ctas * k) + slots * ctas * 4)
+ *   8 * (round_up_even(slots * ctas * k) + slots * ctas * 8)
  * bytes of the rest, where ctas = min(SM count, ceil(V / 64), 1024) and
  * slots = the batch rounded up to a power of two, at most cap; larger
  * requests return VIE_ERR_UNSUPPORTED with the sizes in the message.  Groups

@@ -43,7 +43,8 @@ VIE_OPT_TC_KPS = 4
 VIE_OPT_TC_MIN_BATCH_E4M3 = 5
 VIE_OPT_HALF_ROWS = 6
 VIE_OPT_HOST_H_DIRECT = 7
-VIE_OPT_COUNT = 8
+VIE_OPT_EARLY_MERGE = 8
+VIE_OPT_COUNT = 9
 VIE_OPT_DEFAULT = -(2 ** 31)
 
 STATUS_NAMES = {0: "VIE_OK", 1: "VIE_ERR_INVALID_ARG", 2: "VIE_ERR_UNSUPPORTED",

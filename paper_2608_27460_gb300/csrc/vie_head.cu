@@ -47,6 +47,12 @@ constexpr int kMaxNB = 8;
 static_assert(vie::kTcListKeys + (vie::kTcHRows / 2) * vie::kTcMergeE <= kMaxNB * VIE_K_MAX,
               "tensor-core lists must fit the candidate scratch");
 constexpr int kMaxHBytes = 64 * 1024;  // shared-memory budget for staged queries
+// Scratch words of a handle: [0] completion ticket, [1] device flag word,
+// [2] chunk / tile pool counter, [3] merging CTAs done (tensor-core path),
+// [4] launch epoch (early merge), [8 ..] one publication word per CTA.
+constexpr int kEpochWord = 4;
+constexpr int kFlagWords = 8;
+constexpr int kNumWords = kFlagWords + vie::kMaxLists;
 
 }  // namespace
 
@@ -59,8 +65,7 @@ struct vie_head {
     uint16_t *W;        // [V, d_pad] bf16 bits, or e4m3 codes (bytes) when scale is set
     float *scale;       // e4m3 heads: fp32 scale per row [V]; nullptr for bf16 heads
     uint64_t *cand;     // [kMaxNB][G][VIE_K_MAX] ranking keys, then [kMaxNB][G][kFastE] heads
-    uint32_t *words;    // [0] completion ticket, [1] device flag word, [2] chunk pool counter,
-                        // [3] merging CTAs done (tensor-core path)
+    uint32_t *words;    // kNumWords scratch words (see kEpochWord, kFlagWords)
     int64_t scratch_bytes;
     // tensor-core path (batches): hi/lo bf16 query matrix and TMA descriptors
     void *hB;             // [kTcHRows][d_pad] bf16, or e4m3 query pieces [4 NQ][d_pad]
@@ -195,11 +200,13 @@ constexpr OptionSpec kOptionSpec[VIE_OPT_COUNT] = {
     {1, 1, INT32_MAX}, // VIE_OPT_TC_MIN_BATCH_E4M3
     {-1, -1, 1},       // VIE_OPT_HALF_ROWS
     {1, 0, 1},         // VIE_OPT_HOST_H_DIRECT
+    {1, 0, 1},         // VIE_OPT_EARLY_MERGE
 };
 std::atomic<int> g_options[VIE_OPT_COUNT] = {
     {kOptionSpec[0].dflt}, {kOptionSpec[1].dflt}, {kOptionSpec[2].dflt}, {kOptionSpec[3].dflt},
-    {kOptionSpec[4].dflt}, {kOptionSpec[5].dflt}, {kOptionSpec[6].dflt}, {kOptionSpec[7].dflt}};
-static_assert(VIE_OPT_COUNT == 8, "one default per option");
+    {kOptionSpec[4].dflt}, {kOptionSpec[5].dflt}, {kOptionSpec[6].dflt}, {kOptionSpec[7].dflt},
+    {kOptionSpec[8].dflt}};
+static_assert(VIE_OPT_COUNT == 9, "one default per option");
 
 int opt(vie_launch_option o) { return g_options[o].load(std::memory_order_relaxed); }
 
@@ -380,17 +387,17 @@ static vie_status create_head(const void *W_out, int64_t V, int32_t d, vie_dtype
     const size_t wbytes = static_cast<size_t>(V) * hd->d_pad * (e4m3 ? 1 : 2);
     const size_t cbytes =
         static_cast<size_t>(kMaxNB) * hd->G * (VIE_K_MAX + vie::kFastE) * sizeof(uint64_t);
-    hd->scratch_bytes = static_cast<int64_t>(cbytes + 4 * sizeof(uint32_t));
+    hd->scratch_bytes = static_cast<int64_t>(cbytes + kNumWords * sizeof(uint32_t));
     e = cudaMalloc(&hd->W, wbytes);
     if (e == cudaSuccess && e4m3) e = cudaMalloc(&hd->scale, static_cast<size_t>(V) * sizeof(float));
     if (e == cudaSuccess) e = cudaMalloc(&hd->cand, cbytes);
     if (e == cudaSuccess) e = cudaMemset(hd->cand, 0, cbytes);  // empty lists until written
-    if (e == cudaSuccess) e = cudaMalloc(&hd->words, 4 * sizeof(uint32_t));
+    if (e == cudaSuccess) e = cudaMalloc(&hd->words, kNumWords * sizeof(uint32_t));
     if (e == cudaSuccess)
         e = cudaMalloc(&hd->hB, static_cast<size_t>(vie::kTcHRows) * hd->d_pad * 2);
     if (e == cudaSuccess) e = cudaMemset(hd->hB, 0, static_cast<size_t>(vie::kTcHRows) * hd->d_pad * 2);
     if (e == cudaSuccess && e4m3) e = cudaMalloc(&hd->qscale, 32 * vie::kQ8Pieces * sizeof(float));
-    if (e == cudaSuccess) e = cudaMemset(hd->words, 0, 4 * sizeof(uint32_t));
+    if (e == cudaSuccess) e = cudaMemset(hd->words, 0, kNumWords * sizeof(uint32_t));
     if (e == cudaSuccess && e4m3) {
         int64_t blocks = (V + 7) / 8;  // 8 rows (warps) per block
         if (blocks > 64LL * sms) blocks = 64LL * sms;
@@ -646,6 +653,16 @@ static vie_status run_topk(const char *fn, vie_head *head, const float *h, int32
         p.ticket = head->words;
         p.err = head->words + 1;
         p.next_chunk = head->words + 2;
+        // one query, k <= 64: CTA 0 merges the lists as they arrive (its
+        // merge buffers and every list's first keys in the ring's shared memory)
+        const vie::SmemLayout L(nb, head->d_pad, shp.rs, shp.stages,
+                                head->d_pad * (head->scale != nullptr ? 1 : 2));
+        const uint32_t early_bytes = vie::SmemLayout::merge_fixed_bytes() + 8u * vie::kFastE * head->G +
+                                     4u * ((head->G + 7) & ~7);
+        p.early = (opt(VIE_OPT_EARLY_MERGE) != 0 && nq == 1 && k <= vie::kFastMaxK && head->G >= 2 &&
+                   2 * head->G <= vie::kThreads && L.total - L.merge >= early_bytes) ? 1 : 0;
+        p.epoch = head->words + kEpochWord;
+        p.flags = head->words + kFlagWords;
         p.out_idx = out_idx + static_cast<int64_t>(q0) * k;
         p.out_logits = out_logits + static_cast<int64_t>(q0) * k;
         p.sparse = sparse != nullptr ? sparse + static_cast<int64_t>(q0) * head->V : nullptr;
@@ -1043,6 +1060,9 @@ extern "C" vie_status vie_head_topk_noalloc(const void *W_out, int64_t V, int32_
         p.ticket = counters;
         p.next_chunk = counters + 2;
         p.err = nd.flag;
+        p.early = 0;  // the last-ticket merge: no per-CTA words in the fixed array
+        p.epoch = nullptr;
+        p.flags = nullptr;
         p.out_idx = out_idx + static_cast<int64_t>(q0) * k;
         p.out_logits = out_logits + static_cast<int64_t>(q0) * k;
         p.sparse = nullptr;

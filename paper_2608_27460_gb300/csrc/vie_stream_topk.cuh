@@ -31,9 +31,16 @@
 //   2. every list contributes its prefix of keys >= tau*;
 //   3. exact top-k of those candidates (rank counting, or radix select when
 //      there are many), written best first.
+// Single-query launches with k <= 64 merge early instead: CTA 0 streams only
+// its round-robin chunks (never the pool), so it finishes first, and then
+// merges the other CTAs' lists as they are published (a release store of the
+// launch's epoch per CTA, polled with acquire loads), gathering their first
+// keys in shared memory as they come; after the last list only one poll, one
+// load and the fast merge over those keys remain.
 // With a sparse output, every CTA first fills a fixed slice of each output
-// row with -inf; the merging CTA writes the k logits after the last ticket,
-// so each fill happens before the value at the same position.
+// row with -inf; the merging CTA writes the k logits after every CTA has
+// finished (the last ticket, or the last published list), so each fill
+// happens before the value at the same position.
 #pragma once
 
 #include <cuda_fp16.h>
@@ -54,7 +61,7 @@ constexpr int kMergePrefixCap = 2048;  // keys: first-J prefixes of all lists
 constexpr int kMergeCandCap = 2048;    // keys: gathered candidates
 constexpr int kRankCountMax = 640;     // rank counting below this many keys
 constexpr int kMaxLists = 1024;        // G <= 1024 CTAs
-constexpr int kFastE = 4;              // fast merge: entries read per list (even)
+constexpr int kFastE = 8;              // fast merge: entries read per list (even)
 constexpr int kFastMaxK = 64;          // fast merge: largest k
 
 struct StreamTopkParams {
@@ -75,6 +82,9 @@ struct StreamTopkParams {
     uint32_t *ticket;        // CTA completion counter (self-resetting)
     uint32_t *next_chunk;    // pool counter (self-resetting)
     uint32_t *err;           // device flag word
+    int32_t early;           // 1: CTA 0 merges the lists as they are published (nq == 1)
+    uint32_t *epoch;         // launch counter word (early merge; advanced by CTA 0)
+    uint32_t *flags;         // [G] publication words (early merge)
     int32_t *out_idx;        // [nq, k]
     float *out_logits;       // [nq, k]
     float *sparse;           // [nq, V] fp32 or nullptr
@@ -111,6 +121,7 @@ struct MiscSmem {
     unsigned long long prefix;
     unsigned int tau_v;
     int overflow;
+    uint32_t epoch;
     int chunk_w[kMaxStages];     // first row of each weight stage (-1: end)
     int chunk_s[kScoreStages];   // first row of each score stage (-1: end)
 };
@@ -584,6 +595,75 @@ __device__ inline void merge_queries(const uint64_t *cand, const uint64_t *heads
 }
 
 // --------------------------------------------------------------------------
+// Early merge of one query (CTA 0, every thread, after its own list and
+// heads are written and a bar.sync).  List c (c = 1 .. G-1) is published by
+// CTA c with a release store of `target` into flags[c]; thread c polls that
+// word with acquire loads and, one iteration after it sees the value (so the
+// load overlaps the next polls), copies the list's first kFastE keys from
+// the heads area into shared memory, where the fast merge of merge_queries
+// finds them.  When every list is in, the fast merge settles the query, or
+// (a list that may hold more than kFastE of the top k, or fewer than k real
+// heads) the lists are merged in full.  Every wait is bounded; a list that
+// never arrives is reported through the device flag and counted as empty.
+__device__ inline void early_merge_query(const StreamTopkParams &p, int G, uint32_t target,
+                                         unsigned char *ws, MiscSmem *ms) {
+    const int tid = threadIdx.x;
+    const int k = p.k;
+    MergeBufs mb;
+    mb.pref = reinterpret_cast<uint64_t *>(ws);
+    mb.cands = mb.pref + kMergePrefixCap;
+    mb.win = mb.cands + kMergeCandCap;
+    mb.counts = reinterpret_cast<int *>(mb.win + 1024);
+    mb.offsets = mb.counts + kMaxLists;
+    mb.hist = reinterpret_cast<uint32_t *>(mb.offsets + kMaxLists);
+    const int G8 = (G + 7) & ~7;
+    uint64_t *fe = reinterpret_cast<uint64_t *>(ws + SmemLayout::merge_fixed_bytes());  // [G][kFastE]
+    uint32_t *hv = reinterpret_cast<uint32_t *>(fe + G * kFastE);                     // [G8]
+    const ulonglong2 *heads2 = reinterpret_cast<const ulonglong2 *>(p.heads);
+
+    // empty lists until they arrive; CTA 0's own heads; the fast merge's counters
+    for (int i = tid; i < G * kFastE; i += static_cast<int>(blockDim.x))
+        fe[i] = i < kFastE ? __ldcg(reinterpret_cast<const unsigned long long *>(p.heads) + i) : 0ull;
+    for (int i = tid; i < G8; i += static_cast<int>(blockDim.x))
+        hv[i] = i == 0 ? static_cast<uint32_t>(__ldcg(reinterpret_cast<const unsigned long long *>(p.heads)) >> 32)
+                       : 0u;
+    merge_fast_reset(mb.counts, ms);
+    bool pending = tid >= 1 && tid < G;  // thread c watches list c
+    bool have = false;                   // list c seen, its heads not copied yet
+    const uint64_t t0 = global_timer_ns();
+    for (;;) {
+        const bool load_now = have;
+        ulonglong2 e[kFastE / 2];
+        if (load_now) {
+#pragma unroll
+            for (int j = 0; j < kFastE / 2; ++j) e[j] = __ldcg(heads2 + static_cast<size_t>(tid) * (kFastE / 2) + j);
+            have = false;
+        }
+        if (pending) {
+            if (ld_acquire_gpu(p.flags + tid) == target) {
+                pending = false;
+                have = true;
+            } else if (global_timer_ns() - t0 > kWaitLimitNs) {
+                pending = false;
+                atomicOr(p.err, kErrWaitTimeout);
+            }
+        }
+        if (load_now) {
+            ulonglong2 *dst = reinterpret_cast<ulonglong2 *>(fe + tid * kFastE);
+#pragma unroll
+            for (int j = 0; j < kFastE / 2; ++j) dst[j] = e[j];
+            hv[tid] = static_cast<uint32_t>(e[0].x >> 32);
+        }
+        if (__syncthreads_count((pending || have) ? 1 : 0) == 0) break;
+    }
+    // every list is in: the barrier above ordered each thread's acquire (and
+    // the fast merge's reset) before what follows
+    const bool fast_ok = k <= G && 2 * G <= static_cast<int>(blockDim.x);
+    if (!(fast_ok && merge_fast_query(fe, hv, G, k, mb.cands, mb.counts, ms, p.out_idx, p.out_logits, p.sparse)))
+        merge_lists(GlobalKeys{p.cand}, G, k, mb, ms, p.out_idx, p.out_logits, p.sparse);
+}
+
+// --------------------------------------------------------------------------
 // Rows of the stage that starts at row0: whole chunks (RS rows) in the
 // round-robin part, pool pieces (RSH rows) behind it, and never past the
 // vocabulary.
@@ -649,6 +729,7 @@ __global__ void __launch_bounds__(kThreads, 1) stream_topk_kernel(const StreamTo
         }
         ms->abort = 0;
         ms->is_last = 0;
+        if (p.early) ms->epoch = *reinterpret_cast<volatile uint32_t *>(p.epoch);
         fence_mbar_init();
         griddep_launch_dependents();  // a kernel launched after this one may be scheduled now
     }
@@ -675,17 +756,21 @@ __global__ void __launch_bounds__(kThreads, 1) stream_topk_kernel(const StreamTo
             const uint64_t pol = l2_evict_first_policy();
             const unsigned char *W = reinterpret_cast<const unsigned char *>(p.W);
             const int Ns = p.static_chunks;
+            // the early merger (CTA 0) streams its round-robin chunks only
+            const bool pool = !(p.early && cta == 0);
             // first draw from the pool, issued early so its latency is hidden
-            uint32_t draw = (Ns == 0) ? atomic_add_relaxed_gpu(p.next_chunk, 1u) : 0u;
+            uint32_t draw = (Ns == 0 && pool) ? atomic_add_relaxed_gpu(p.next_chunk, 1u) : 0u;
             int issued = 0;
             bool ok = true;
             for (int t = 0;; ++t) {
                 int64_t row0;
                 if (t < Ns) {
                     row0 = static_cast<int64_t>(t * G + cta) * RS;
-                } else {
+                } else if (pool) {
                     row0 = pool_row0 + static_cast<int64_t>(draw) * RSH;
                     if (row0 >= p.V) row0 = -1;
+                } else {
+                    row0 = -1;
                 }
                 const int s = t % S, u = t / S;
                 if (t >= S && !mbar_wait(&empty[s], (u - 1) & 1, abort_flag)) {
@@ -702,7 +787,7 @@ __global__ void __launch_bounds__(kThreads, 1) stream_topk_kernel(const StreamTo
                 mbar_arrive_expect_tx(&full[s], bytes);
                 bulk_g2s(ring + s * stage_bytes, W + row0 * row_bytes, bytes, &full[s], pol);
                 issued = t + 1;
-                if (t + 1 >= Ns) draw = atomic_add_relaxed_gpu(p.next_chunk, 1u);
+                if (t + 1 >= Ns && pool) draw = atomic_add_relaxed_gpu(p.next_chunk, 1u);
             }
             if (!ok) {
                 atomicOr(p.err, kErrWaitTimeout);
@@ -926,6 +1011,27 @@ __global__ void __launch_bounds__(kThreads, 1) stream_topk_kernel(const StreamTo
                 }
             }
         }
+    }
+
+    // ---------------- early merge (one query, k <= 64) ----------------
+    // bar.sync orders every thread's writes (list, heads, sparse fill) before
+    // thread 0's release store of this launch's epoch + 1; CTA 0 acquires each
+    // word before it reads that CTA's list, and a bar.sync orders all of
+    // those acquires before its output writes.  Words left by earlier
+    // launches hold older epochs, so nothing needs clearing.
+    if (p.early) {
+        __syncthreads();
+        const uint32_t target = ms->epoch + 1u;
+        if (cta != 0) {
+            if (tid == 0) st_release_gpu(p.flags + cta, target);
+            return;
+        }
+        early_merge_query(p, G, target, smem + L.merge, ms);
+        if (tid == 0) {
+            *p.next_chunk = 0;  // re-arm the pool for the next launch
+            *reinterpret_cast<volatile uint32_t *>(p.epoch) = target;
+        }
+        return;
     }
 
     // ---------------- completion ticket ----------------

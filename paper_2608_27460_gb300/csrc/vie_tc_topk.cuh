@@ -59,7 +59,7 @@ constexpr int kTcHRows = 128;      // rows of the hi/lo query matrix (N <= 128)
 constexpr int kTcMaxK = 128;       // largest k of this path
 constexpr int kTcListKeys = 4096;  // keys of the per-CTA lists per CTA: NQ * k <= this
 constexpr int kTcMaxKPS = 4;       // K-blocks per stage, at most
-constexpr int kTcMergeE = 4;       // merge: keys per list in the heads area
+constexpr int kTcMergeE = 8;       // merge: keys per list in the heads area
 constexpr int kQ8Pieces = 4;       // e4m3 columns per query on the Q8 path
 constexpr int kTcMaxMergers = 64;  // CTAs that merge, at most (one per query)
 
@@ -164,12 +164,6 @@ __device__ __forceinline__ uint8_t e4m3_code(float x) {
 }
 __device__ __forceinline__ float e4m3_value(uint8_t c) {
     return __half2float(__half(__nv_cvt_fp8_to_halfraw(static_cast<__nv_fp8_storage_t>(c), __NV_E4M3)));
-}
-
-__device__ __forceinline__ uint64_t shfl_xor_u64(uint64_t v, int m) {
-    const uint32_t lo = __shfl_xor_sync(0xFFFFFFFFu, static_cast<uint32_t>(v), m);
-    const uint32_t hi = __shfl_xor_sync(0xFFFFFFFFu, static_cast<uint32_t>(v >> 32), m);
-    return (static_cast<uint64_t>(hi) << 32) | lo;
 }
 
 // Bitonic sort, descending, of the 32 * PER keys a warp holds (lane l holds

@@ -143,7 +143,7 @@ def test_launch_options_hook(lib):
     library reads no environment variable."""
     defaults = {vie.VIE_OPT_STAGE_MIN_KB: 48, vie.VIE_OPT_STATIC_PCT: 85, vie.VIE_OPT_POOL_DIV: 1,
                 vie.VIE_OPT_TC_MIN_BATCH: 2, vie.VIE_OPT_TC_KPS: 4, vie.VIE_OPT_TC_MIN_BATCH_E4M3: 1,
-                vie.VIE_OPT_HALF_ROWS: -1, vie.VIE_OPT_HOST_H_DIRECT: 1}
+                vie.VIE_OPT_HALF_ROWS: -1, vie.VIE_OPT_HOST_H_DIRECT: 1, vie.VIE_OPT_EARLY_MERGE: 1}
     assert len(defaults) == vie.VIE_OPT_COUNT
     for o, v in defaults.items():
         assert vie.vie_get_launch_option(o) == (vie.VIE_OK, v)

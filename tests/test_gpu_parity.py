@@ -270,3 +270,43 @@ def test_parity_full_size(vie, name, batch, k, n):
             want, ok = oracle.scatter(idx, val, V)
             assert ok and np.array_equal(want.view(np.uint32), sparse.view(np.uint32))
         assert head.device_status() == vie.VIE_OK, vie.vie_last_error()
+
+
+@pytest.mark.parametrize("early", [0, 1])
+def test_batch1_merge_modes(vie, early):
+    """Single-query launches merged early (CTA 0 streams only its round-robin
+    chunks, then takes the other CTAs' lists as they are published) or by
+    the last CTA to finish: the same parity, the sparse tensor equal to the
+    oracle's scatter of the returned top-k, and many back-to-back calls on
+    one handle (the early merge keys each launch's publications by an epoch
+    that advances every launch).  Covered: vocabularies so small that CTA 0
+    streams nothing (V = 200, 2 CTAs at V = 128), k = 1 and k = 64 (the
+    largest early-merged k), duplicate rows, and the full Gemma-3-1B shape."""
+    import torch
+    with vie.launch_options({vie.VIE_OPT_EARLY_MERGE: early}):
+        for V, d, k, dup in [(151936, 1024, 50, 0.0), (20011, 640, 64, 0.05), (9000, 256, 1, 0.0),
+                             (4099, 100, 50, 0.0), (200, 64, 50, 0.0), (128, 16, 64, 0.0),
+                             (262144, 1152, 50, 0.05)]:
+            n = 4
+            W, h = workload(V, d, n, seed=V + d + k, dup_frac=dup, planted=0.5 if dup else 0.0)
+            z = oracle.logits(W, h)
+            hd = torch.from_numpy(h).cuda()
+            with vie.Head(to_device_bits(W)) as head:
+                assert head.plan(1, k).path == 0
+                first = None
+                for rep in range(3):
+                    for q in range(n):
+                        idx, val, sp = head.topk_sparse(hd[q:q + 1], k)
+                        torch.cuda.synchronize()
+                        idx, val, sp = idx.cpu().numpy(), val.cpu().numpy(), sp.cpu().numpy()
+                        errs = check_topk(idx[0], val[0], z[q], k)
+                        assert not errs, (V, d, k, early, rep, q, errs)
+                        want, ok = oracle.scatter(idx, val, V)
+                        assert ok and np.array_equal(want.view(np.uint32), sp.view(np.uint32))
+                        if q == 0:
+                            if first is None:
+                                first = (idx, val)
+                            else:  # a repeated call returns the same bits
+                                assert np.array_equal(first[0], idx)
+                                assert np.array_equal(first[1].view(np.uint32), val.view(np.uint32))
+                assert head.device_status() == vie.VIE_OK, vie.vie_last_error()
