@@ -48,8 +48,8 @@ static_assert(vie::kTcListKeys + (vie::kTcHRows / 2) * vie::kTcMergeE <= kMaxNB 
               "tensor-core lists must fit the candidate scratch");
 constexpr int kMaxHBytes = 64 * 1024;  // shared-memory budget for staged queries
 // Scratch words of a handle: [0] completion ticket, [1] device flag word,
-// [2] chunk / tile pool counter, [3] merging CTAs done (tensor-core path),
-// [4] launch epoch (early merge), [8 ..] one publication word per CTA.
+// [2] chunk / tile pool counter, [4] launch epoch, [8 ..] one publication
+// word per CTA (a CTA's lists are ready once its word holds the epoch + 1).
 constexpr int kEpochWord = 4;
 constexpr int kFlagWords = 8;
 constexpr int kNumWords = kFlagWords + vie::kMaxLists;
@@ -563,7 +563,8 @@ static vie_status run_topk_tc(const char *fn, vie_head *head, const float *h, in
         if (vie::tc_shape(nqt, q8, c, hres_bytes, &stages, &slots, &smem)) kps = c;
     }
     if (kps == 0) return fail(VIE_ERR_UNSUPPORTED, "%s: no tensor-core layout", fn);
-    const int n_tiles = static_cast<int>((head->V + vie::kTcTile - 1) / vie::kTcTile);
+    const int tile_rows = vie::tc_tile_rows(nqt, q8);
+    const int n_tiles = static_cast<int>((head->V + tile_rows - 1) / tile_rows);
     const int pct = opt(VIE_OPT_STATIC_PCT);
     const int n_h = (q8 ? vie::kQ8Pieces : 2) * nqt;  // query rows: boxes of 16 / 32 / 64 / 128
     const CUtensorMap &mapH = head->mapH[n_h == 16 ? 0 : (n_h == 32 ? 1 : (n_h == 64 ? 2 : 3))];
@@ -588,8 +589,9 @@ static vie_status run_topk_tc(const char *fn, vie_head *head, const float *h, in
         p.heads = head->cand + static_cast<size_t>(vie::kTcListKeys) * head->G;
         p.ticket = head->words;
         p.next_tile = head->words + 2;
-        p.merged = head->words + 3;
         p.err = head->words + 1;
+        p.epoch = head->words + kEpochWord;
+        p.flags = head->words + kFlagWords;
         p.out_idx = out_idx + static_cast<int64_t>(q0) * k;
         p.out_logits = out_logits + static_cast<int64_t>(q0) * k;
         p.sparse = sparse != nullptr ? sparse + static_cast<int64_t>(q0) * head->V : nullptr;

@@ -48,6 +48,8 @@ cudaError_t launch_sample_topk(const int32_t *idx, const float *logits, int batc
 // Largest k the tensor-core kernel with nq_tmpl query slots handles (q8: on
 // e4m3 rows).
 int tc_max_k(int nq_tmpl, bool q8 = false);
+// Rows of W per tile of that kernel (128, or 256 for the 64-query bf16 tile).
+int tc_tile_rows(int nq_tmpl, bool q8 = false);
 // Ring depth, score-ring depth and dynamic shared memory for query groups of
 // nq_tmpl (8, 16, 32 or 64; 4, 8, 16 or 32 on e4m3 rows), kps K-blocks per
 // stage and hres_bytes of query operand built in shared memory; false if

@@ -33,10 +33,10 @@
 //      there are many), written best first.
 // Single-query launches with k <= 64 merge early instead: CTA 0 streams only
 // its round-robin chunks (never the pool), so it finishes first, and then
-// merges the other CTAs' lists as they are published (a release store of the
-// launch's epoch per CTA, polled with acquire loads), gathering their first
-// keys in shared memory as they come; after the last list only one poll, one
-// load and the fast merge over those keys remain.
+// merges the CTAs' lists as they are published (merge_published: a release
+// store of the launch's epoch per CTA, polled with acquire loads, the lists'
+// first keys gathered in shared memory as they come); after the last list
+// only one poll, one load and the fast merge over those keys remain.
 // With a sparse output, every CTA first fills a fixed slice of each output
 // row with -inf; the merging CTA writes the k logits after every CTA has
 // finished (the last ticket, or the last published list), so each fill
@@ -595,20 +595,23 @@ __device__ inline void merge_queries(const uint64_t *cand, const uint64_t *heads
 }
 
 // --------------------------------------------------------------------------
-// Early merge of one query (CTA 0, every thread, after its own list and
-// heads are written and a bar.sync).  List c (c = 1 .. G-1) is published by
-// CTA c with a release store of `target` into flags[c]; thread c polls that
-// word with acquire loads and, one iteration after it sees the value (so the
-// load overlaps the next polls), copies the list's first kFastE keys from
-// the heads area into shared memory, where the fast merge of merge_queries
-// finds them.  When every list is in, the fast merge settles the query, or
-// (a list that may hold more than kFastE of the top k, or fewer than k real
-// heads) the lists are merged in full.  Every wait is bounded; a list that
-// never arrives is reported through the device flag and counted as empty.
-__device__ inline void early_merge_query(const StreamTopkParams &p, int G, uint32_t target,
-                                         unsigned char *ws, MiscSmem *ms) {
+// Merge of one query from published lists (every thread of the merging CTA).
+// CTA c publishes its lists with a release store of `target` (the launch's
+// epoch + 1) into flags[c] once they and its sparse fill are written; words
+// left by earlier launches hold older epochs.  Thread c polls flags[c] with
+// acquire loads and, one iteration after it sees the value (so that load
+// overlaps the next polls), copies list c's first kFastE keys (heads_q + c *
+// kFastE) into fe, where the fast merge finds them.  When every list is in,
+// the fast merge settles the query, or (a list that may hold more than
+// kFastE of the top k, or fewer than k real heads) the lists (lists_q, G x k
+// keys) are merged in full.  ws holds the merge buffers (merge_fixed_bytes);
+// fe holds G * kFastE keys and then ceil(G/8)*8 head words.  Every wait is
+// bounded; a list that never arrives is reported in *err and counted empty.
+__device__ inline void merge_published(const uint32_t *flags, uint32_t target, const uint64_t *heads_q,
+                                       const uint64_t *lists_q, int G, int k, unsigned char *ws,
+                                       uint64_t *fe, MiscSmem *ms, uint32_t *err, int32_t *oi, float *ol,
+                                       float *sp) {
     const int tid = threadIdx.x;
-    const int k = p.k;
     MergeBufs mb;
     mb.pref = reinterpret_cast<uint64_t *>(ws);
     mb.cands = mb.pref + kMergePrefixCap;
@@ -617,19 +620,15 @@ __device__ inline void early_merge_query(const StreamTopkParams &p, int G, uint3
     mb.offsets = mb.counts + kMaxLists;
     mb.hist = reinterpret_cast<uint32_t *>(mb.offsets + kMaxLists);
     const int G8 = (G + 7) & ~7;
-    uint64_t *fe = reinterpret_cast<uint64_t *>(ws + SmemLayout::merge_fixed_bytes());  // [G][kFastE]
-    uint32_t *hv = reinterpret_cast<uint32_t *>(fe + G * kFastE);                     // [G8]
-    const ulonglong2 *heads2 = reinterpret_cast<const ulonglong2 *>(p.heads);
+    uint32_t *hv = reinterpret_cast<uint32_t *>(fe + G * kFastE);  // [G8]
+    const ulonglong2 *heads2 = reinterpret_cast<const ulonglong2 *>(heads_q);
 
-    // empty lists until they arrive; CTA 0's own heads; the fast merge's counters
-    for (int i = tid; i < G * kFastE; i += static_cast<int>(blockDim.x))
-        fe[i] = i < kFastE ? __ldcg(reinterpret_cast<const unsigned long long *>(p.heads) + i) : 0ull;
-    for (int i = tid; i < G8; i += static_cast<int>(blockDim.x))
-        hv[i] = i == 0 ? static_cast<uint32_t>(__ldcg(reinterpret_cast<const unsigned long long *>(p.heads)) >> 32)
-                       : 0u;
+    // empty lists until they arrive; the fast merge's counters
+    for (int i = tid; i < G * kFastE; i += static_cast<int>(blockDim.x)) fe[i] = 0ull;
+    for (int i = tid; i < G8; i += static_cast<int>(blockDim.x)) hv[i] = 0u;
     merge_fast_reset(mb.counts, ms);
-    bool pending = tid >= 1 && tid < G;  // thread c watches list c
-    bool have = false;                   // list c seen, its heads not copied yet
+    bool pending = tid < G;  // thread c watches list c
+    bool have = false;       // list c seen, its heads not copied yet
     const uint64_t t0 = global_timer_ns();
     for (;;) {
         const bool load_now = have;
@@ -640,12 +639,12 @@ __device__ inline void early_merge_query(const StreamTopkParams &p, int G, uint3
             have = false;
         }
         if (pending) {
-            if (ld_acquire_gpu(p.flags + tid) == target) {
+            if (ld_acquire_gpu(flags + tid) == target) {
                 pending = false;
                 have = true;
             } else if (global_timer_ns() - t0 > kWaitLimitNs) {
                 pending = false;
-                atomicOr(p.err, kErrWaitTimeout);
+                atomicOr(err, kErrWaitTimeout);
             }
         }
         if (load_now) {
@@ -659,8 +658,8 @@ __device__ inline void early_merge_query(const StreamTopkParams &p, int G, uint3
     // every list is in: the barrier above ordered each thread's acquire (and
     // the fast merge's reset) before what follows
     const bool fast_ok = k <= G && 2 * G <= static_cast<int>(blockDim.x);
-    if (!(fast_ok && merge_fast_query(fe, hv, G, k, mb.cands, mb.counts, ms, p.out_idx, p.out_logits, p.sparse)))
-        merge_lists(GlobalKeys{p.cand}, G, k, mb, ms, p.out_idx, p.out_logits, p.sparse);
+    if (!(fast_ok && merge_fast_query(fe, hv, G, k, mb.cands, mb.counts, ms, oi, ol, sp)))
+        merge_lists(GlobalKeys{lists_q}, G, k, mb, ms, oi, ol, sp);
 }
 
 // --------------------------------------------------------------------------
@@ -798,6 +797,9 @@ __global__ void __launch_bounds__(kThreads, 1) stream_topk_kernel(const StreamTo
                     mbar_wait(&full[t2 % S], (t2 / S) & 1, const_cast<volatile int *>(&never));
             }
         }
+        // the other lanes wait for the producer lane here, so the whole warp
+        // reaches the CTA barrier below together (bar.sync counts warps)
+        __syncwarp();
     } else {
         // fused sparse output: a fixed slice of every query row = -inf
         if (p.sparse != nullptr) {
@@ -1022,11 +1024,12 @@ __global__ void __launch_bounds__(kThreads, 1) stream_topk_kernel(const StreamTo
     if (p.early) {
         __syncthreads();
         const uint32_t target = ms->epoch + 1u;
-        if (cta != 0) {
-            if (tid == 0) st_release_gpu(p.flags + cta, target);
-            return;
-        }
-        early_merge_query(p, G, target, smem + L.merge, ms);
+        if (tid == 0) st_release_gpu(p.flags + cta, target);
+        if (cta != 0) return;
+        unsigned char *ws = smem + L.merge;
+        merge_published(p.flags, target, p.heads, p.cand, G, p.k, ws,
+                        reinterpret_cast<uint64_t *>(ws + SmemLayout::merge_fixed_bytes()), ms, p.err,
+                        p.out_idx, p.out_logits, p.sparse);
         if (tid == 0) {
             *p.next_chunk = 0;  // re-arm the pool for the next launch
             *reinterpret_cast<volatile uint32_t *>(p.epoch) = target;

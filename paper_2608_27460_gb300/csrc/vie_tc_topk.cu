@@ -77,6 +77,20 @@ bool tc_shape(int nq_tmpl, bool q8, int kps, int hres_bytes, int *stages, int *s
     return false;
 }
 
+int tc_tile_rows(int nq_tmpl, bool q8) {
+    switch (q8 ? -nq_tmpl : nq_tmpl) {
+        case 8: return TcShape<8>::kTileRows;
+        case 16: return TcShape<16>::kTileRows;
+        case 32: return TcShape<32>::kTileRows;
+        case 64: return TcShape<64>::kTileRows;
+        case -4: return TcShape<4, true>::kTileRows;
+        case -8: return TcShape<8, true>::kTileRows;
+        case -16: return TcShape<16, true>::kTileRows;
+        case -32: return TcShape<32, true>::kTileRows;
+        default: return 0;
+    }
+}
+
 int tc_max_k(int nq_tmpl, bool q8) {
     switch (q8 ? -nq_tmpl : nq_tmpl) {
         case 8: return TcShape<8>::kMaxK;

@@ -76,7 +76,8 @@ struct TcParams {
     uint64_t *heads;         // [NQ][G][kTcMergeE]: the first keys of each list
     uint32_t *ticket;        // CTA completion counter (self-resetting)
     uint32_t *next_tile;     // pool counter (self-resetting)
-    uint32_t *merged;        // merging CTAs done (self-resetting)
+    uint32_t *epoch;         // launch counter word (advanced by the last CTA to finish)
+    uint32_t *flags;         // [G] publication words: flags[c] = epoch + 1 once CTA c's lists are written
     uint32_t *err;           // device flag word
     int32_t *out_idx;        // [nq, k]
     float *out_logits;       // [nq, k]
@@ -97,10 +98,20 @@ struct TcShape {
     static constexpr int kSelWarps = NQ / kQPW;
     static constexpr int kWarps = 6 + kSelWarps;
     static constexpr int kThreads = 32 * kWarps;
-    static constexpr int kStageA = kTcTile * 128;  // 16 KB per K-block of W (128 B per row)
+    // 128-row halves per tile (two M = 128 MMAs into two accumulators per
+    // K-block: a query box rides with twice the weight bytes).  Measured: at
+    // 256 rows the 64-query tile finishes later, its coarser tiles leaving the
+    // CTAs up to a tile apart at the end (~30 us at d = 3072), so every tile
+    // is 128 rows.
+    static constexpr int kMH = 1;
+    static constexpr int kTileRows = kTcTile * kMH;
+    static constexpr int kHalfA = kTcTile * 128;   // 16 KB: one 128-row box of a K-block of W
+    static constexpr int kStageA = kMH * kHalfA;   // W bytes per K-block (128 B per row)
     static constexpr int kStageB = N * 128;        // N x 128 B per K-block of H
     static constexpr int kStageBytes = kStageA + kStageB;    // per K-block; a multiple of 1024
-    static constexpr int kTmemCols = (2 * N <= 32) ? 32 : (2 * N <= 64 ? 64 : (2 * N <= 128 ? 128 : 256));
+    static constexpr int kAccCols = kMH * N;  // accumulator columns of one tile
+    static constexpr int kTmemCols = (2 * kAccCols <= 32) ? 32 : (2 * kAccCols <= 64 ? 64 :
+                                     (2 * kAccCols <= 128 ? 128 : (2 * kAccCols <= 256 ? 256 : 512)));
     // score ring depth (e4m3 tiles: 2, leaving shared memory to the weight ring)
     static constexpr int kMinSlots = NQ >= 64 ? 1 : 2;     // score ring depth, at least
     static constexpr int kSlotBytes = NQ * kTcTile * 4;    // one tile's logits, [query][row]
@@ -128,8 +139,9 @@ struct TcMisc {
     int abort;
     int stage_tile[kTcMaxStages];  // tile of a stage that starts a tile (-1: end)
     int buf_tile[2];               // tile held by each TMEM accumulator
-    int slot_tile[kTcScoreSlots];  // tile of each score slot
+    int slot_tile[kTcScoreSlots];  // 128-row block (row / 128) of each score slot (-1: end)
     int merger;                    // m >= 0: this CTA merges queries m, m + X, ...
+    uint32_t epoch;                // the launch counter, read after the previous kernel finished
 };
 
 // The ring (1024-byte aligned at run time) starts with the resident query
@@ -340,7 +352,9 @@ __global__ void __launch_bounds__(TcShape<NQ, Q8>::kThreads, 1)
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int G = gridDim.x, cta = blockIdx.x;
     const int n_st = (n_kb + KPS - 1) / KPS;  // stages per tile
-    const int n_tiles = static_cast<int>((p.V + kTcTile - 1) / kTcTile);
+    constexpr int MH = Sh::kMH;
+    constexpr int TR = Sh::kTileRows;
+    const int n_tiles = static_cast<int>((p.V + TR - 1) / TR);
 
     if (tid == 0) {
         for (int s = 0; s < S; ++s) {
@@ -487,8 +501,10 @@ __global__ void __launch_bounds__(TcShape<NQ, Q8>::kThreads, 1)
                     mbar_arrive_expect_tx(&full[s], nin * kb_bytes);
                     unsigned char *st = ring + s * stage_bytes;
                     for (int i = 0; i < nin; ++i)
-                        tma_load_2d(st + i * Sh::kStageA, &mapW, (kb0 + i) * KB, tile * kTcTile,
-                                    &full[s], pol);
+#pragma unroll
+                        for (int h = 0; h < MH; ++h)
+                            tma_load_2d(st + i * Sh::kStageA + h * Sh::kHalfA, &mapW, (kb0 + i) * KB,
+                                        tile * TR + h * kTcTile, &full[s], pol);
                     if (!hres) {
                         if (it == 0) griddep_wait();  // the query matrix comes from the prep kernel
                         for (int i = 0; i < nin; ++i)
@@ -507,6 +523,9 @@ __global__ void __launch_bounds__(TcShape<NQ, Q8>::kThreads, 1)
                     mbar_wait(&full[t2 % S], (t2 / S) & 1, const_cast<volatile int *>(&never));
             }
         }
+        // the other lanes wait for the producer lane here, so the whole warp
+        // reaches the CTA barrier below together (bar.sync counts warps)
+        __syncwarp();
     } else if (warp == 1) {
         // ---------------- MMA issuer ----------------
         if (lane == 0) {
@@ -533,7 +552,7 @@ __global__ void __launch_bounds__(TcShape<NQ, Q8>::kThreads, 1)
                     break;
                 }
                 mc->buf_tile[b] = tile;
-                const uint32_t d = tmem + static_cast<uint32_t>(b * N);
+                const uint32_t d = tmem + static_cast<uint32_t>(b * Sh::kAccCols);
                 for (int st_i = 0; st_i < n_st; ++st_i, ++it) {
                     const int s = it % S, u = it / S;
                     if (st_i > 0 && !mbar_wait(&full[s], u & 1, abort_flag)) {
@@ -549,10 +568,15 @@ __global__ void __launch_bounds__(TcShape<NQ, Q8>::kThreads, 1)
                             hres ? hq_res + (kb0 + i) * Sh::kStageB : st + KPS * Sh::kStageA + i * Sh::kStageB);
 #pragma unroll
                         for (int k4 = 0; k4 < 4; ++k4) {  // +32 bytes per MMA (K = 16 bf16 or 32 e4m3)
-                            if constexpr (Q8)
-                                umma_e4m3(d, ad + 2 * k4, bd + 2 * k4, idesc, ((kb0 + i) | k4) != 0 ? 1u : 0u);
-                            else
-                                umma_bf16(d, ad + 2 * k4, bd + 2 * k4, idesc, ((kb0 + i) | k4) != 0 ? 1u : 0u);
+#pragma unroll
+                            for (int h = 0; h < MH; ++h) {  // rows h*128.. of the tile: accumulator h
+                                const uint64_t adh = ad + static_cast<uint64_t>(h * (Sh::kHalfA >> 4));
+                                const uint32_t acc = ((kb0 + i) | k4) != 0 ? 1u : 0u;
+                                if constexpr (Q8)
+                                    umma_e4m3(d + h * N, adh + 2 * k4, bd + 2 * k4, idesc, acc);
+                                else
+                                    umma_bf16(d + h * N, adh + 2 * k4, bd + 2 * k4, idesc, acc);
+                            }
                         }
                     }
                     umma_commit(&empty[s]);
@@ -570,6 +594,7 @@ __global__ void __launch_bounds__(TcShape<NQ, Q8>::kThreads, 1)
             const int never = 0;
             mbar_wait(final_bar, 0, const_cast<volatile int *>(&never));
         }
+        __syncwarp();  // the whole warp reaches the CTA barrier together
     } else if (warp < 6) {
         // ---------------- epilogue: TMEM -> logits ----------------
         const int qw = warp & 3;  // TMEM lane quarter this warp may access
@@ -595,54 +620,65 @@ __global__ void __launch_bounds__(TcShape<NQ, Q8>::kThreads, 1)
             // Q8: this row's scale, loaded under the accumulator reads
             float rsc = 1.0f;
             if constexpr (Q8) {
-                const int64_t gr = static_cast<int64_t>(tile) * kTcTile + row;
+                const int64_t gr = static_cast<int64_t>(tile) * TR + row;  // MH == 1 on e4m3 rows
                 if (tile >= 0 && gr < p.V) rsc = __ldg(p.row_scale + gr);
             }
             if constexpr (N > 64) {
-                // wide tiles: wait for the score slot first, then drain the
-                // accumulator 32 columns (16 queries) at a time
-                if (ti >= SL && !mbar_wait(&sempty[ss], (su - 1) & 1, abort_flag)) {
-                    if (lane == 0) {
-                        atomicOr(p.err, kErrWaitTimeout);
-                        mc->abort = 1;
+                // wide tiles: per 128-row half, wait for a score slot first,
+                // then drain that half's accumulator 32 columns (16 queries)
+                // at a time; the TMEM buffer is handed back after the last half
+                bool failed = false;
+#pragma unroll 1
+                for (int h = 0; h < MH; ++h) {
+                    const int si = ti * MH + h, ssh = si % SL, suh = si / SL;
+                    if (si >= SL && !mbar_wait(&sempty[ssh], (suh - 1) & 1, abort_flag)) {
+                        if (lane == 0) {
+                            atomicOr(p.err, kErrWaitTimeout);
+                            mc->abort = 1;
+                        }
+                        failed = true;
+                        break;
                     }
-                    break;
-                }
-                if (tile >= 0) {
-                    const uint32_t tb = tmem + (static_cast<uint32_t>(32 * qw) << 16) + b * N;
-                    float *sc = scores + ss * NQ * kTcTile;
-                    constexpr int QC = 32 / Sh::kCols;  // queries per 32 accumulator columns
+                    if (tile >= 0) {
+                        const uint32_t tb = tmem + (static_cast<uint32_t>(32 * qw) << 16) + b * Sh::kAccCols + h * N;
+                        float *sc = scores + ssh * NQ * kTcTile;
+                        constexpr int QC = 32 / Sh::kCols;  // queries per 32 accumulator columns
 #pragma unroll
-                    for (int c = 0; c < N / 16; c += 2) {
-                        uint32_t r[2][16];
-                        tmem_ld_32x32b_x16(tb + 16 * c, r[0]);
-                        tmem_ld_32x32b_x16(tb + 16 * (c + 1), r[1]);
-                        tmem_wait_ld();
+                        for (int c = 0; c < N / 16; c += 2) {
+                            uint32_t r[2][16];
+                            tmem_ld_32x32b_x16(tb + 16 * c, r[0]);
+                            tmem_ld_32x32b_x16(tb + 16 * (c + 1), r[1]);
+                            tmem_wait_ld();
 #pragma unroll
-                        for (int qq = 0; qq < QC; ++qq) {
-                            const int q = QC * (c / 2) + qq, c0 = Sh::kCols * qq;
-                            float z;
-                            if constexpr (Q8) {
-                                z = 0.0f;
+                            for (int qq = 0; qq < QC; ++qq) {
+                                const int q = QC * (c / 2) + qq, c0 = Sh::kCols * qq;
+                                float z;
+                                if constexpr (Q8) {
+                                    z = 0.0f;
 #pragma unroll
-                                for (int pc = 0; pc < kQ8Pieces; ++pc)
-                                    z = fmaf(qs[kQ8Pieces * q + pc],
-                                             __uint_as_float(r[(c0 + pc) / 16][(c0 + pc) % 16]), z);
-                                z *= rsc;
-                            } else {
-                                z = __uint_as_float(r[c0 / 16][c0 % 16]) + __uint_as_float(r[c0 / 16][c0 % 16 + 1]);
+                                    for (int pc = 0; pc < kQ8Pieces; ++pc)
+                                        z = fmaf(qs[kQ8Pieces * q + pc],
+                                                 __uint_as_float(r[(c0 + pc) / 16][(c0 + pc) % 16]), z);
+                                    z *= rsc;
+                                } else {
+                                    z = __uint_as_float(r[c0 / 16][c0 % 16]) +
+                                        __uint_as_float(r[c0 / 16][c0 % 16 + 1]);
+                                }
+                                sc[q * kTcTile + row] = z;
                             }
-                            sc[q * kTcTile + row] = z;
                         }
                     }
+                    if (h == MH - 1 || tile < 0) {
+                        tc_fence_before_sync();
+                        __syncwarp();
+                        if (lane == 0) mbar_arrive(&tempty[b]);
+                    }
+                    if (warp == 2 && lane == 0) mc->slot_tile[ssh] = tile >= 0 ? tile * MH + h : -1;
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(&sfull[ssh]);
+                    if (tile < 0) break;
                 }
-                tc_fence_before_sync();
-                __syncwarp();
-                if (lane == 0) mbar_arrive(&tempty[b]);
-                if (warp == 2 && lane == 0) mc->slot_tile[ss] = tile;
-                __syncwarp();
-                if (lane == 0) mbar_arrive(&sfull[ss]);
-                if (tile < 0) break;
+                if (failed || tile < 0) break;
                 continue;
             }
             float lg[NQ];
@@ -681,7 +717,7 @@ __global__ void __launch_bounds__(TcShape<NQ, Q8>::kThreads, 1)
 #pragma unroll
                 for (int q = 0; q < NQ; ++q) sc[q * kTcTile + row] = lg[q];
             }
-            if (warp == 2 && lane == 0) mc->slot_tile[ss] = tile;
+            if (warp == 2 && lane == 0) mc->slot_tile[ss] = tile;  // MH == 1: the tile is the row block
             __syncwarp();
             if (lane == 0) mbar_arrive(&sfull[ss]);
             if (tile < 0) break;
@@ -690,6 +726,9 @@ __global__ void __launch_bounds__(TcShape<NQ, Q8>::kThreads, 1)
         // ---------------- selectors ----------------
         const int sel = warp - 6;
         griddep_wait();  // writes below must follow the previous kernel on the stream
+        // the launch counter, now that the kernel before this one has finished
+        // (it may have advanced it)
+        if (sel == 0 && lane == 0) mc->epoch = *reinterpret_cast<volatile uint32_t *>(p.epoch);
         if (p.sparse != nullptr) {
             // this CTA's fixed slice of every sparse row = -inf (values come later)
             const float ninf = __uint_as_float(0xFF800000u);
@@ -725,9 +764,9 @@ __global__ void __launch_bounds__(TcShape<NQ, Q8>::kThreads, 1)
                     }
                     break;
                 }
-                const int tile = mc->slot_tile[ss];
-                if (tile < 0) break;
-                const int64_t row0 = static_cast<int64_t>(tile) * kTcTile;
+                const int rblk = mc->slot_tile[ss];
+                if (rblk < 0) break;
+                const int64_t row0 = static_cast<int64_t>(rblk) * kTcTile;
                 const int rows = static_cast<int>(min(static_cast<int64_t>(kTcTile), p.V - row0));
                 const float *sc = scores + ss * NQ * kTcTile;
 #pragma unroll 1
@@ -792,9 +831,9 @@ __global__ void __launch_bounds__(TcShape<NQ, Q8>::kThreads, 1)
                     }
                     break;
                 }
-                const int tile = mc->slot_tile[ss];
-                if (tile < 0) break;
-                const int64_t row0 = static_cast<int64_t>(tile) * kTcTile;
+                const int rblk = mc->slot_tile[ss];
+                if (rblk < 0) break;
+                const int64_t row0 = static_cast<int64_t>(rblk) * kTcTile;
                 const int rows = static_cast<int>(min(static_cast<int64_t>(kTcTile), p.V - row0));
                 const float *sc = scores + ss * NQ * kTcTile;
 #pragma unroll
@@ -849,80 +888,50 @@ __global__ void __launch_bounds__(TcShape<NQ, Q8>::kThreads, 1)
         tmem_dealloc(tmem, Sh::kTmemCols);
     }
 
-    // ---------------- completion ticket ----------------
-    // bar.sync orders every thread's writes (lists, heads, sparse fill)
-    // before thread 0's release.  The last X CTAs to take a ticket merge: each
-    // waits until every CTA has taken one (an acquire of the final count,
-    // which follows every release), then merges queries m, m + X, ... with the
-    // whole CTA; the last of them to finish re-arms the counters.
+    // ---------------- publication, then the merge (first X CTAs) ----------------
+    // bar.sync orders every thread's writes (lists, heads, sparse fill) before
+    // thread 0's release store of epoch + 1 into this CTA's publication word.
+    // A relaxed ticket then ranks the CTAs by finishing order: the first X
+    // merge (queries m, m + X, ...), taking each CTA's lists as they are
+    // published, while the others still stream; the last re-arms the tile
+    // pool and the ticket and advances the epoch (every CTA has drawn its
+    // last tile and taken its ticket by then).
     const int X = min(p.nq, min(G, kTcMaxMergers));
+    const uint32_t target = mc->epoch + 1u;
     if (tid == 0) {
-        const uint32_t ticket = atomic_add_acq_rel_gpu(p.ticket, 1u);
-        const int m = static_cast<int>(ticket) - (G - X);
-        mc->merger = m;
-        if (m >= 0) {
-            const uint64_t t0 = global_timer_ns();
-            while (ld_acquire_gpu(p.ticket) < static_cast<uint32_t>(G)) {
-                if (global_timer_ns() - t0 > kWaitLimitNs) {
-                    atomicOr(p.err, kErrWaitTimeout);
-                    break;
-                }
-                __nanosleep(32);
-            }
+        st_release_gpu(p.flags + cta, target);
+        const uint32_t ticket = atomic_add_relaxed_gpu(p.ticket, 1u);
+        if (ticket == static_cast<uint32_t>(G - 1)) {
+            *p.next_tile = 0;
+            *p.ticket = 0;
+            *reinterpret_cast<volatile uint32_t *>(p.epoch) = target;
         }
+        mc->merger = ticket < static_cast<uint32_t>(X) ? static_cast<int>(ticket) : -1;
     }
     __syncthreads();
     const int m = mc->merger;
     if (m < 0) return;
 
-    // ---------------- global merge (last X CTAs) ----------------
+    // ---------------- merge ----------------
     // Scores, buffers and ring are free now.  Per query: the first kFastE keys
-    // of every list (the heads area) go to shared memory, the fast merge
-    // settles the query from them, or the full merge reads the lists.
-    // (every CTA wrote full lists and heads, valid keys or zeros, even if it
-    // gave up on a wait: the merge stays in bounds, the flag reports the call)
+    // of every list (the heads area) go to shared memory as the lists are
+    // published, the fast merge settles the query from them, or the full
+    // merge reads the lists.  (Every CTA wrote full lists and heads, valid
+    // keys or zeros, even if it gave up on a wait: the merge stays in bounds,
+    // the flag reports the call.)
     {
         static_assert(kTcMergeE == kFastE, "the heads area feeds the fast merge");
         unsigned char *ws = smem + L.scores;
-        MergeBufs mb;
-        mb.pref = reinterpret_cast<uint64_t *>(ws);
-        mb.cands = mb.pref + kMergePrefixCap;
-        mb.win = mb.cands + kMergeCandCap;
-        mb.counts = reinterpret_cast<int *>(mb.win + 1024);
-        mb.offsets = mb.counts + kMaxLists;
-        mb.hist = reinterpret_cast<uint32_t *>(mb.offsets + kMaxLists);
         const uint32_t ms_off = (SmemLayout::merge_fixed_bytes() + 15u) & ~15u;
         MiscSmem *ms = reinterpret_cast<MiscSmem *>(ws + ms_off);
         uint64_t *fe = reinterpret_cast<uint64_t *>(ws + ms_off + ((sizeof(MiscSmem) + 15u) & ~15u));
-        const int G8 = (G + 7) & ~7;
-        uint32_t *hv = reinterpret_cast<uint32_t *>(fe + G * kFastE);
-        const bool fast_ok = p.k <= G && 2 * G <= kThreads;
         for (int q = m; q < p.nq; q += X) {
-            const unsigned long long *hq =
-                reinterpret_cast<const unsigned long long *>(p.heads) + static_cast<size_t>(q) * G * kFastE;
-            for (int i = tid; i < G8 * kFastE; i += Sh::kThreads) {
-                const uint64_t x = i < G * kFastE ? __ldcg(hq + i) : 0ull;
-                if (i == tid) merge_fast_reset(mb.counts, ms);  // while the first loads are in flight
-                if (i < G * kFastE) fe[i] = x;
-                if ((i & (kFastE - 1)) == 0) hv[i / kFastE] = static_cast<uint32_t>(x >> 32);
-            }
-            if (tid >= G8 * kFastE) merge_fast_reset(mb.counts, ms);
-            __syncthreads();
             int32_t *oi = p.out_idx + static_cast<size_t>(q) * p.k;
             float *ol = p.out_logits + static_cast<size_t>(q) * p.k;
             float *sp = p.sparse != nullptr ? p.sparse + static_cast<int64_t>(q) * p.V : nullptr;
-            if (!(fast_ok && merge_fast_query(fe, hv, G, p.k, mb.cands, mb.counts, ms, oi, ol, sp)))
-                merge_lists(GlobalKeys{p.cand + static_cast<size_t>(q) * G * p.k}, G, p.k, mb, ms, oi,
-                            ol, sp);
+            merge_published(p.flags, target, p.heads + static_cast<size_t>(q) * G * kFastE,
+                            p.cand + static_cast<size_t>(q) * G * p.k, G, p.k, ws, fe, ms, p.err, oi, ol, sp);
             __syncthreads();
-        }
-    }
-    if (tid == 0) {
-        const uint32_t done = atomic_add_acq_rel_gpu(p.merged, 1u);
-        if (done == static_cast<uint32_t>(X - 1)) {
-            *p.ticket = 0;  // re-arm the counters for the next launch
-            *p.next_tile = 0;
-            *p.merged = 0;
         }
     }
 }
