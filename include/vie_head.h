@@ -370,8 +370,9 @@ vie_status vie_scatter_sparse_logits(const int32_t *idx, const float *logits, in
  *
  * Every batch runs on the streaming CUDA-core kernel, in query groups of up
  * to `cap` queries, one launch per group:
- *   cap = 8 for k <= 64, 4 for k <= 256, 1 above, then halved (not below 1)
- *         while cap * d * 4 > 65536.
+ *   cap = 8, halved (not below 1) while cap * d * 4 > 65536 or, for k > 64,
+ *         while cap * c * 8 > 32768, where c = max(256, 2k rounded up to a
+ *         multiple of 64) is the candidate buffer of one query.
  * Scratch: one 1 MiB array per device (every GPU that loads the library keeps
  * it until the process exits), of which the first 256 bytes hold counters.
  * A call needs

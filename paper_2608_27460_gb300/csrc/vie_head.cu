@@ -47,6 +47,7 @@ constexpr int kMaxNB = 8;
 static_assert(vie::kTcListKeys + (vie::kTcHRows / 2) * vie::kTcMergeE <= kMaxNB * VIE_K_MAX,
               "tensor-core lists must fit the candidate scratch");
 constexpr int kMaxHBytes = 64 * 1024;  // shared-memory budget for staged queries
+constexpr int kMaxSelBytes = 32 * 1024;  // ... and for the wide lists' candidate buffers
 // Scratch words of a handle: [0] completion ticket, [1] device flag word,
 // [2] chunk / tile pool counter, [4] launch epoch, [8 ..] one publication
 // word per CTA (a CTA's lists are ready once its word holds the epoch + 1).
@@ -175,13 +176,23 @@ __global__ void scatter_sparse_kernel(const int32_t *__restrict__ idx,
 // ---------------------------------------------------------------------------
 namespace {
 
-int pick_mm(int k) { return k <= 64 ? 2 : (k <= 256 ? 8 : 32); }
+// Selector of the streaming kernel: register lists of 2 keys per lane for
+// k <= 64, else (0) the shared-memory candidate buffers of the wide lists.
+int pick_mm(int k) { return k <= vie::kFastMaxK ? 2 : 0; }
 
-// Widest query group for a row width and list width: the staged queries
-// must fit their shared-memory budget and the selector's lists its registers.
-int nb_cap_for(int d_pad, int mm) {
-    int nb = mm >= 32 ? 1 : (mm >= 8 ? 4 : kMaxNB);
-    while (nb > 1 && nb * d_pad * 4 > kMaxHBytes) nb >>= 1;
+// Keys per query of a launch's candidate buffers (wide lists): one query
+// gets 2048 (no cut-back while a CTA streams up to ~2000 rows), groups the
+// least size for k.
+int sel_cap_launch(int nb, int k) {
+    const int c = vie::sel_cap_for(k);
+    return (nb == 1 && c > 0 && c < 2048) ? 2048 : c;
+}
+
+// Widest query group for a row width and k: the staged queries and the wide
+// lists' candidate buffers must fit their shared-memory budgets.
+int nb_cap_for(int d_pad, int k) {
+    int nb = kMaxNB;
+    while (nb > 1 && (nb * d_pad * 4 > kMaxHBytes || nb * vie::sel_cap_for(k) * 8 > kMaxSelBytes)) nb >>= 1;
     return nb;
 }
 
@@ -236,13 +247,13 @@ struct LaunchShape {
 
 // Rows per warp per stage (R), stage rows (8*R, fewer for very wide rows),
 // and ring depth (deepest that fits) for one launch.
-bool pick_shape(int nb, int d_pad, int row_bytes, LaunchShape *out) {
+bool pick_shape(int nb, int d_pad, int row_bytes, int sel_cap, LaunchShape *out) {
     const int r_max = nb == 1 ? 8 : 4;  // 8 rows per warp only for single-query launches
     int r = 1;
     while (r < r_max && 8 * r * row_bytes < opt(VIE_OPT_STAGE_MIN_KB) * 1024) r <<= 1;
     for (int rs = 8 * r; rs >= 1; --rs) {
         for (int s = vie::kMaxStages; s >= 2; --s) {
-            const vie::SmemLayout L(nb, d_pad, rs, s, row_bytes);
+            const vie::SmemLayout L(nb, d_pad, rs, s, row_bytes, sel_cap);
             if (L.total <= static_cast<uint32_t>(kMaxSmem)) {
                 out->r = r;
                 out->rs = rs;
@@ -536,7 +547,7 @@ static vie_topk_plan make_plan(const vie_head *head, int32_t batch, int32_t k) {
         // projection, per-CTA top-k and merge in one launch
         pl.launches = (tc_hres(head, nqt) > 0 ? 1 : 2) * pl.groups;
     } else {
-        const int cap = nb_cap_for(head->d_pad, pick_mm(k));
+        const int cap = nb_cap_for(head->d_pad, k);
         pl.path = 0;
         pl.groups = (batch + cap - 1) / cap;
         pl.launches = pl.groups;
@@ -626,13 +637,14 @@ static vie_status run_topk(const char *fn, vie_head *head, const float *h, int32
     const int mm = pick_mm(k);
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     if (use_tc(head, batch, k)) return run_topk_tc(fn, head, h, batch, k, out_idx, out_logits, sparse, s);
-    const int cap = nb_cap_for(head->d_pad, mm);
+    const int cap = nb_cap_for(head->d_pad, k);
     for (int q0 = 0; q0 < batch; q0 += cap) {
         const int nq = batch - q0 < cap ? batch - q0 : cap;
         int nb = 1;
         while (nb < nq) nb <<= 1;
         LaunchShape shp;
-        if (!pick_shape(nb, head->d_pad, head->d_pad * (head->scale != nullptr ? 1 : 2), &shp))
+        if (!pick_shape(nb, head->d_pad, head->d_pad * (head->scale != nullptr ? 1 : 2), sel_cap_launch(nb, k),
+                        &shp))
             return fail(VIE_ERR_UNSUPPORTED, "%s: no shared-memory layout for d=%d", fn, head->d);
         vie::StreamTopkParams p;
         p.W = head->W;
@@ -650,6 +662,7 @@ static vie_status run_topk(const char *fn, vie_head *head, const float *h, int32
         p.static_chunks = static_cast<int32_t>(n_chunks * pct / 100 / head->G);
         p.pool_rows = pool_rows_for(shp.rs);
         p.half_rows = half_rows_for(shp.r, head->d_pad / (head->scale != nullptr ? 16 : 8));
+        p.sel_cap = sel_cap_launch(nb, k);
         p.cand = head->cand;
         p.heads = head->cand + static_cast<size_t>(kMaxNB) * head->G * VIE_K_MAX;
         p.ticket = head->words;
@@ -658,11 +671,13 @@ static vie_status run_topk(const char *fn, vie_head *head, const float *h, int32
         // one query, k <= 64: CTA 0 merges the lists as they arrive (its
         // merge buffers and every list's first keys in the ring's shared memory)
         const vie::SmemLayout L(nb, head->d_pad, shp.rs, shp.stages,
-                                head->d_pad * (head->scale != nullptr ? 1 : 2));
+                                head->d_pad * (head->scale != nullptr ? 1 : 2), p.sel_cap);
         const uint32_t early_bytes = vie::SmemLayout::merge_fixed_bytes() + 8u * vie::kFastE * head->G +
                                      4u * ((head->G + 7) & ~7);
         p.early = (opt(VIE_OPT_EARLY_MERGE) != 0 && nq == 1 && k <= vie::kFastMaxK && head->G >= 2 &&
                    2 * head->G <= vie::kThreads && L.total - L.merge >= early_bytes) ? 1 : 0;
+        // several queries: the first CTAs to finish merge them in parallel
+        p.pmerge = (nq > 1 && head->G <= vie::kThreads && L.total - L.merge >= early_bytes) ? 1 : 0;
         p.epoch = head->words + kEpochWord;
         p.flags = head->words + kFlagWords;
         p.out_idx = out_idx + static_cast<int64_t>(q0) * k;
@@ -1009,7 +1024,7 @@ extern "C" vie_status vie_head_topk_noalloc(const void *W_out, int64_t V, int32_
     if (g > vie::kMaxLists) g = vie::kMaxLists;
     const int G = static_cast<int>(g < 1 ? 1 : g);
     const int mm = pick_mm(k);
-    const int cap = nb_cap_for(d, mm);
+    const int cap = nb_cap_for(d, k);
     int nb_max = 1;
     while (nb_max < cap && nb_max < batch) nb_max <<= 1;
     // lists [nb_max][G][k], then the heads [nb_max][G][kFastE], which the
@@ -1039,7 +1054,7 @@ extern "C" vie_status vie_head_topk_noalloc(const void *W_out, int64_t V, int32_
         int nb = 1;
         while (nb < nq) nb <<= 1;
         LaunchShape shp;
-        if (!pick_shape(nb, d, d * 2, &shp))
+        if (!pick_shape(nb, d, d * 2, sel_cap_launch(nb, k), &shp))
             return fail(VIE_ERR_UNSUPPORTED, "%s: no shared-memory layout for d=%d", fn, d);
         vie::StreamTopkParams p;
         p.W = static_cast<const uint16_t *>(W_out);
@@ -1057,12 +1072,14 @@ extern "C" vie_status vie_head_topk_noalloc(const void *W_out, int64_t V, int32_
         p.static_chunks = static_cast<int32_t>(n_chunks * pct / 100 / G);
         p.pool_rows = pool_rows_for(shp.rs);
         p.half_rows = half_rows_for(shp.r, d / 8);
+        p.sel_cap = sel_cap_launch(nb, k);
         p.cand = cand;
         p.heads = heads;
         p.ticket = counters;
         p.next_chunk = counters + 2;
         p.err = nd.flag;
         p.early = 0;  // the last-ticket merge: no per-CTA words in the fixed array
+        p.pmerge = 0;
         p.epoch = nullptr;
         p.flags = nullptr;
         p.out_idx = out_idx + static_cast<int64_t>(q0) * k;

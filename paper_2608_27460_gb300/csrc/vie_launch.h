@@ -10,7 +10,7 @@
 namespace vie {
 
 // Launches stream_topk_kernel<nb, mm, r> on `grid` CTAs; nb in {1,2,4,8},
-// mm in {2,8,32}, r in {1,2,4}.  Returns the launch error
+// mm in {2 (register lists), 0 (candidate buffers)}, r in {1,2,4,8}.  Returns the launch error
 // (cudaErrorInvalidValue for an unsupported combination).
 cudaError_t launch_stream_topk(int nb, int mm, int r, const StreamTopkParams &p, int grid,
                                uint32_t smem, cudaStream_t stream);

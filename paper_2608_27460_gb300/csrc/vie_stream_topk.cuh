@@ -22,6 +22,13 @@
 //   warp 1     selector: keeps the best keys seen so far as a sorted list
 //              spread over the warp's registers; a row enters only if it
 //              beats the current k-th key.  It never holds a weight stage.
+//              Wide lists (k > 64): every key above the bound tau goes into
+//              a shared-memory buffer of the query (ballot and append); a
+//              full buffer is cut back to its best k by a bisection on the
+//              keys, which raises tau to the k-th of them.  After the stream
+//              the whole CTA turns each buffer into the sorted list (radix
+//              select of the best k, sorted runs of 128 keys in registers,
+//              then each key's place from binary searches in the other runs).
 // The full logit vector never leaves the chip.  Afterwards each CTA writes
 // its sorted top-k list to scratch and takes a ticket (an acq_rel atomic, no
 // full fences); the CTA that draws the last ticket copies every list into
@@ -37,6 +44,8 @@
 // store of the launch's epoch per CTA, polled with acquire loads, the lists'
 // first keys gathered in shared memory as they come); after the last list
 // only one poll, one load and the fast merge over those keys remain.
+// Launches of several queries publish their lists the same way; the first
+// CTAs to finish (one per query, round robin) merge them as they arrive.
 // With a sparse output, every CTA first fills a fixed slice of each output
 // row with -inf; the merging CTA writes the k logits after every CTA has
 // finished (the last ticket, or the last published list), so each fill
@@ -63,6 +72,17 @@ constexpr int kRankCountMax = 640;     // rank counting below this many keys
 constexpr int kMaxLists = 1024;        // G <= 1024 CTAs
 constexpr int kFastE = 8;              // fast merge: entries read per list (even)
 constexpr int kFastMaxK = 64;          // fast merge: largest k
+constexpr int kSelRun = 128;           // keys of one sorted run (a warp's registers)
+constexpr int kRankRunsMin = 256;      // ranking by sorted runs above this many keys
+
+// Keys per query of the shared-memory candidate buffer of the wide lists
+// (k > kFastMaxK): room for k keys and as many again, so a cut-back keeps k
+// and frees at least k; 0 for the register lists.
+__host__ __device__ inline int sel_cap_for(int k) {
+    if (k <= kFastMaxK) return 0;
+    const int c = (2 * k + 63) & ~63;
+    return c < 256 ? 256 : c;
+}
 
 struct StreamTopkParams {
     const uint16_t *W;   // padded [V, d_pad] bf16 bits, or [V, d_pad] e4m3 codes (bytes)
@@ -77,14 +97,17 @@ struct StreamTopkParams {
     int32_t static_chunks;   // chunks each CTA owns before drawing from the pool
     int32_t pool_rows;       // rows of a pool piece (<= rows_per_stage)
     int32_t half_rows;       // 1: each half-warp projects its own row (R >= 2)
+    int32_t sel_cap;         // wide lists: buffer keys per query (sel_cap_for(k)); else 0
     uint64_t *cand;          // [NB][G][k] keys
     uint64_t *heads;         // [NB][G][kFastE]: the first keys of each list
     uint32_t *ticket;        // CTA completion counter (self-resetting)
     uint32_t *next_chunk;    // pool counter (self-resetting)
     uint32_t *err;           // device flag word
     int32_t early;           // 1: CTA 0 merges the lists as they are published (nq == 1)
-    uint32_t *epoch;         // launch counter word (early merge; advanced by CTA 0)
-    uint32_t *flags;         // [G] publication words (early merge)
+    int32_t pmerge;          // 1: the first min(nq, G) CTAs to finish merge the queries,
+                             //    each taking the lists as they are published (nq > 1)
+    uint32_t *epoch;         // launch counter word (early merge or pmerge)
+    uint32_t *flags;         // [G] publication words (early merge or pmerge)
     int32_t *out_idx;        // [nq, k]
     float *out_logits;       // [nq, k]
     float *sparse;           // [nq, V] fp32 or nullptr
@@ -92,14 +115,15 @@ struct StreamTopkParams {
 
 // Shared-memory carve-up; all offsets are multiples of 128 bytes.
 struct SmemLayout {
-    uint32_t bars, misc, h, scores, ring, merge, total;
+    uint32_t bars, misc, h, scores, sel, ring, merge, total;
     __host__ __device__ static uint32_t align128(uint32_t x) { return (x + 127u) & ~127u; }
-    __host__ __device__ SmemLayout(int nb, int d_pad, int rs, int stages, int row_bytes) {
+    __host__ __device__ SmemLayout(int nb, int d_pad, int rs, int stages, int row_bytes, int sel_cap) {
         bars = 0;
         misc = align128(bars + 8u * (2 * kMaxStages + 2 * kScoreStages));
         h = align128(misc + 256u);
         scores = align128(h + 4u * nb * d_pad);
-        ring = align128(scores + 4u * kScoreStages * rs * nb);
+        sel = align128(scores + 4u * kScoreStages * rs * nb);  // wide lists: [nb][sel_cap] keys
+        ring = align128(sel + 8u * nb * sel_cap);
         merge = ring;  // the merge reuses the ring once the stream is drained
         uint32_t ring_end = ring + static_cast<uint32_t>(stages) * rs * row_bytes;
         uint32_t merge_end = merge + merge_fixed_bytes();
@@ -122,9 +146,12 @@ struct MiscSmem {
     unsigned int tau_v;
     int overflow;
     uint32_t epoch;
+    int merger;                  // pmerge: m >= 0 merges queries m, m + X, ...
+    int sel_cnt[8];              // wide lists: keys in each query's buffer
     int chunk_w[kMaxStages];     // first row of each weight stage (-1: end)
     int chunk_s[kScoreStages];   // first row of each score stage (-1: end)
 };
+static_assert(sizeof(MiscSmem) <= 256, "MiscSmem fits its 256-byte slot");
 
 __device__ __forceinline__ uint32_t atomic_add_acq_rel_gpu(uint32_t *p, uint32_t v) {
     uint32_t old;
@@ -176,6 +203,43 @@ struct WarpList {
     }
 };
 
+// Bitonic sort, descending, of the 32 * PER keys a warp holds (lane l holds
+// elements l*PER .. l*PER + PER - 1).  Steps with a stride below PER swap
+// registers; wider steps exchange with lane ^ (stride / PER).
+template <int PER>
+__device__ __forceinline__ void warp_sort_desc(uint64_t (&v)[PER], int lane) {
+#pragma unroll
+    for (int size = 2; size <= 32 * PER; size <<= 1) {
+#pragma unroll
+        for (int stride = size >> 1; stride > 0; stride >>= 1) {
+            if (stride < PER) {
+#pragma unroll
+                for (int j = 0; j < PER; ++j) {
+                    const int pj = j ^ stride;
+                    if (pj > j) {
+                        const bool desc = ((lane * PER + j) & size) == 0;
+                        const uint64_t a = v[j], b = v[pj];
+                        if (desc ? (a < b) : (a > b)) {
+                            v[j] = b;
+                            v[pj] = a;
+                        }
+                    }
+                }
+            } else {
+                const int ls = stride / PER;
+                const bool lower = (lane & ls) == 0;
+#pragma unroll
+                for (int j = 0; j < PER; ++j) {
+                    const uint64_t o = shfl_xor_u64(v[j], ls);
+                    const bool desc = ((lane * PER + j) & size) == 0;
+                    const bool keep_max = lower == desc;
+                    v[j] = keep_max ? (v[j] > o ? v[j] : o) : (v[j] < o ? v[j] : o);
+                }
+            }
+        }
+    }
+}
+
 // --------------------------------------------------------------------------
 // Block-wide helpers for the merge: every thread of the CTA calls them, for
 // any block size of at least 32 threads (merge_queries: at least kThreads).
@@ -194,20 +258,26 @@ struct GlobalKeys {
 // Threshold T such that exactly k of the keys with key >= lo (lo >= 1) are
 // >= T (keys are unique apart from 0, which is never counted).  MSB-first
 // radix select over 8-bit digits, stopping early once the selected bin
-// holds exactly the keys still needed.
+// holds exactly the keys still needed.  The lanes of a warp that hit the
+// same bin add their count with one atomic (the keys of a top-k share their
+// leading digits, so a bin can draw most of the block's increments).  The
+// block size is a multiple of 32.
 template <class Keys>
 __device__ uint64_t block_radix_threshold(Keys keys, int n, int k, uint64_t lo, uint32_t *hist,
                                           MiscSmem *ms) {
-    const int tid = threadIdx.x;
+    const int tid = threadIdx.x, lane = tid & 31;
     uint64_t prefix = 0, mask = 0;
     int remaining = k;
     for (int shift = 56; shift >= 0; shift -= 8) {
         for (int i = tid; i < 256; i += static_cast<int>(blockDim.x)) hist[i] = 0;
         __syncthreads();
-        for (int i = tid; i < n; i += static_cast<int>(blockDim.x)) {
-            const uint64_t x = keys[i];
-            if (x >= lo && x != 0 && (x & mask) == prefix)
-                atomicAdd(&hist[(x >> shift) & 255u], 1u);
+        for (int i0 = tid - lane; i0 < n; i0 += static_cast<int>(blockDim.x)) {
+            const int i = i0 + lane;
+            const uint64_t x = i < n ? keys[i] : 0ull;
+            const bool in = x >= lo && x != 0 && (x & mask) == prefix;
+            const unsigned bin = in ? static_cast<unsigned>((x >> shift) & 255u) : 256u;
+            const unsigned peers = __match_any_sync(0xFFFFFFFFu, bin);
+            if (in && (__ffs(peers) - 1) == lane) atomicAdd(&hist[bin], static_cast<unsigned>(__popc(peers)));
         }
         __syncthreads();
         if (tid < 32) {
@@ -268,15 +338,64 @@ __device__ __forceinline__ int rank_among(const uint64_t *keys, int n, uint64_t 
     return r0 + r1;
 }
 
+// Descending ranks of the m unique nonzero keys a[0..m) (shared memory):
+// runs of kSelRun keys are each sorted by one warp in its registers (a is
+// rewritten run by run), then a key's rank is its place in its own run plus,
+// per other run, the number of that run's keys above it (binary search).
+// emit(rank, key) is called once per key.  Every thread of the CTA calls it;
+// it ends with a barrier.
+template <class Emit>
+__device__ inline void block_rank_by_runs(uint64_t *a, int m, Emit emit) {
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int nthr = static_cast<int>(blockDim.x), nw = nthr >> 5;
+    const int nruns = (m + kSelRun - 1) / kSelRun;
+    constexpr int PER = kSelRun / 32;
+    for (int r = warp; r < nruns; r += nw) {
+        uint64_t v[PER];
+#pragma unroll
+        for (int j = 0; j < PER; ++j) {
+            const int e = r * kSelRun + lane * PER + j;
+            v[j] = e < m ? a[e] : 0ull;
+        }
+        warp_sort_desc<PER>(v, lane);
+#pragma unroll
+        for (int j = 0; j < PER; ++j) {
+            const int e = r * kSelRun + lane * PER + j;
+            if (e < m) a[e] = v[j];  // zeros sort last: the real keys fill the run's front
+        }
+    }
+    __syncthreads();
+    for (int i = tid; i < m; i += nthr) {
+        const uint64_t x = a[i];
+        const int r = i / kSelRun;
+        int rank = i - r * kSelRun;
+        for (int r2 = 0; r2 < nruns; ++r2) {
+            if (r2 == r) continue;
+            const uint64_t *run = a + r2 * kSelRun;
+            int lo = 0, hi = min(kSelRun, m - r2 * kSelRun);
+            while (lo < hi) {
+                const int mid = (lo + hi) >> 1;
+                if (run[mid] > x)
+                    lo = mid + 1;
+                else
+                    hi = mid;
+            }
+            rank += lo;
+        }
+        emit(rank, x);
+    }
+    __syncthreads();
+}
+
 // Exact top-k of n unique nonzero keys in shared memory, written best first
 // to out_idx / out_logits (and into the sparse row, if any).  Rank counting
 // for small n, otherwise a radix-select threshold and rank counting of the
 // k winners.
-__device__ inline void block_topk_to_output(const uint64_t *keys, int n, int k, uint64_t *win,
+__device__ inline void block_topk_to_output(uint64_t *keys, int n, int k, uint64_t *win,
                                             uint32_t *hist, MiscSmem *ms, int32_t *out_idx,
                                             float *out_logits, float *sparse_row) {
     const int tid = threadIdx.x;
-    const uint64_t *src = keys;
+    uint64_t *src = keys;
     int m = n;
     if (n > kRankCountMax && n > k) {
         const uint64_t T = block_radix_threshold(SmemKeys{keys}, n, k, 1, hist, ms);
@@ -290,6 +409,17 @@ __device__ inline void block_topk_to_output(const uint64_t *keys, int n, int k, 
         src = win;
         m = k;
     }
+    if (m > kRankRunsMin) {
+        // many keys: sorted runs and binary searches (rank counting is m^2)
+        block_rank_by_runs(src, m, [&](int rank, uint64_t x) {
+            if (rank < k) {
+                out_idx[rank] = key_index(x);
+                out_logits[rank] = key_value(x);
+                if (sparse_row != nullptr) sparse_row[key_index(x)] = key_value(x);
+            }
+        });
+        return;
+    }
     for (int i = tid; i < m; i += static_cast<int>(blockDim.x)) {
         const uint64_t x = src[i];
         const int rank = rank_among(src, m, x);
@@ -300,6 +430,108 @@ __device__ inline void block_topk_to_output(const uint64_t *keys, int n, int k, 
         }
     }
     __syncthreads();
+}
+
+// Wide lists: cuts the cnt (> k) unique nonzero keys of buf back to its best
+// k, moved to buf[0..k), and returns the k-th largest key (the new entry
+// bound).  One warp.  The k-th key is found one digit at a time: two bits of
+// the high word (the ordered logit) per step, from three independent counts
+// of keys at or above the candidates; then, when several keys share that
+// logit, two bits per step of the low word (the inverted row) among them.
+// Each step reads the buffer from shared memory.
+static __device__ __noinline__ uint64_t warp_cut_to_best(uint64_t *buf, int cnt, int k, int lane) {
+    __syncwarp();
+    const uint32_t *w32 = reinterpret_cast<const uint32_t *>(buf);
+    uint32_t th = 0;
+#pragma unroll 1
+    for (int bit = 30; bit >= 0; bit -= 2) {
+        const uint32_t c1 = th | (1u << bit), c2 = th | (2u << bit), c3 = th | (3u << bit);
+        int n1 = 0, n2 = 0, n3 = 0;
+        for (int e = lane; e < cnt; e += 32) {
+            const uint32_t hi = w32[2 * e + 1];
+            n1 += hi >= c1 ? 1 : 0;
+            n2 += hi >= c2 ? 1 : 0;
+            n3 += hi >= c3 ? 1 : 0;
+        }
+        n1 = static_cast<int>(__reduce_add_sync(0xFFFFFFFFu, n1));
+        n2 = static_cast<int>(__reduce_add_sync(0xFFFFFFFFu, n2));
+        n3 = static_cast<int>(__reduce_add_sync(0xFFFFFFFFu, n3));
+        th = n3 >= k ? c3 : (n2 >= k ? c2 : (n1 >= k ? c1 : th));
+    }
+    int n_gt = 0, n_ge = 0;
+    for (int e = lane; e < cnt; e += 32) {
+        const uint32_t hi = w32[2 * e + 1];
+        n_gt += hi > th ? 1 : 0;
+        n_ge += hi >= th ? 1 : 0;
+    }
+    n_gt = static_cast<int>(__reduce_add_sync(0xFFFFFFFFu, n_gt));
+    n_ge = static_cast<int>(__reduce_add_sync(0xFFFFFFFFu, n_ge));
+    uint32_t tl = 0;
+    if (n_ge > k) {
+        const int need = k - n_gt;  // keys still needed among those with logit th
+#pragma unroll 1
+        for (int bit = 30; bit >= 0; bit -= 2) {
+            const uint32_t c1 = tl | (1u << bit), c2 = tl | (2u << bit), c3 = tl | (3u << bit);
+            int n1 = 0, n2 = 0, n3 = 0;
+            for (int e = lane; e < cnt; e += 32) {
+                if (w32[2 * e + 1] != th) continue;
+                const uint32_t lo = w32[2 * e];
+                n1 += lo >= c1 ? 1 : 0;
+                n2 += lo >= c2 ? 1 : 0;
+                n3 += lo >= c3 ? 1 : 0;
+            }
+            n1 = static_cast<int>(__reduce_add_sync(0xFFFFFFFFu, n1));
+            n2 = static_cast<int>(__reduce_add_sync(0xFFFFFFFFu, n2));
+            n3 = static_cast<int>(__reduce_add_sync(0xFFFFFFFFu, n3));
+            tl = n3 >= need ? c3 : (n2 >= need ? c2 : (n1 >= need ? c1 : tl));
+        }
+    }
+    const uint64_t T = (static_cast<uint64_t>(th) << 32) | tl;
+    // in place: every write lands at or below the position it was read from
+    // in this pass, after the whole warp has read that block of 32
+    const unsigned lt_mask = (1u << lane) - 1u;
+    int base = 0;
+    for (int e0 = 0; e0 < cnt; e0 += 32) {
+        const int e = e0 + lane;
+        const uint64_t v = e < cnt ? buf[e] : 0ull;
+        const bool in = v >= T && v != 0;
+        const unsigned m = __ballot_sync(0xFFFFFFFFu, in);
+        if (in) buf[base + __popc(m & lt_mask)] = v;
+        base += __popc(m);
+    }
+    __syncwarp();
+    return T;
+}
+
+// Wide lists, after the stream: the sorted list of one query's buffer (cnt
+// unique nonzero keys; cnt may exceed k) written best first to dst[0..k)
+// (zeros after the real keys) and its first kFastE keys to head.  Every
+// thread of the CTA calls it.  win (k keys) and hist (256 words) are free
+// shared memory; buf is sorted in place when it holds at most k keys.
+__device__ inline void write_cta_list(uint64_t *buf, int cnt, int k, uint32_t *hist, uint64_t *win,
+                                      MiscSmem *ms, uint64_t *dst, uint64_t *head) {
+    const int tid = threadIdx.x, nthr = static_cast<int>(blockDim.x);
+    uint64_t *a = buf;
+    int m = cnt;
+    if (cnt > k) {
+        // exactly k keys are >= T (keys are unique)
+        const uint64_t T = block_radix_threshold(SmemKeys{buf}, cnt, k, 1, hist, ms);
+        if (tid == 0) ms->n_win = 0;
+        __syncthreads();
+        for (int i = tid; i < cnt; i += nthr) {
+            const uint64_t x = buf[i];
+            if (x >= T) win[atomicAdd(&ms->n_win, 1)] = x;
+        }
+        a = win;
+        m = k;
+    }
+    __syncthreads();
+    block_rank_by_runs(a, m, [&](int rank, uint64_t x) {
+        dst[rank] = x;
+        if (rank < kFastE) head[rank] = x;
+    });
+    for (int i = m + tid; i < k; i += nthr) dst[i] = 0ull;
+    for (int i = m + tid; i < kFastE; i += nthr) head[i] = 0ull;
 }
 
 // Shared-memory buffers of the merge.
@@ -696,7 +928,7 @@ __global__ void __launch_bounds__(kThreads, 1) stream_topk_kernel(const StreamTo
     const int S = p.stages;
     const int row_bytes = Q8 ? p.d_pad : p.d_pad * 2;
     constexpr int kEPC = Q8 ? 16 : 8;  // weights per 16-byte chunk
-    const SmemLayout L(NB, p.d_pad, RS, S, row_bytes);
+    const SmemLayout L(NB, p.d_pad, RS, S, row_bytes, MM == 0 ? p.sel_cap : 0);
     uint64_t *full = reinterpret_cast<uint64_t *>(smem + L.bars);
     uint64_t *empty = full + kMaxStages;
     uint64_t *sfull = empty + kMaxStages;
@@ -728,7 +960,7 @@ __global__ void __launch_bounds__(kThreads, 1) stream_topk_kernel(const StreamTo
         }
         ms->abort = 0;
         ms->is_last = 0;
-        if (p.early) ms->epoch = *reinterpret_cast<volatile uint32_t *>(p.epoch);
+        if (p.early || p.pmerge) ms->epoch = *reinterpret_cast<volatile uint32_t *>(p.epoch);
         fence_mbar_init();
         griddep_launch_dependents();  // a kernel launched after this one may be scheduled now
     }
@@ -815,60 +1047,113 @@ __global__ void __launch_bounds__(kThreads, 1) stream_topk_kernel(const StreamTo
         cp_async_wait_all();
         named_barrier_sync(1, kThreads - 32);  // h in shared memory for warps 1..
         if (warp == 1) {
-            // ---------------- selector ----------------
-            WarpList<MM> list[NB];
-            uint64_t tau[NB];
-#pragma unroll
-            for (int nb = 0; nb < NB; ++nb) {
-                list[nb].clear();
-                tau[nb] = 0;
-            }
-            for (int t = 0;; ++t) {
-                const int s = t % kScoreStages, u = t / kScoreStages;
-                if (!mbar_wait(&sfull[s], u & 1, abort_flag)) {
-                    if (lane == 0) {
-                        atomicOr(p.err, kErrWaitTimeout);
-                        ms->abort = 1;
-                    }
-                    break;
-                }
-                const int chunk = ms->chunk_s[s];
-                if (chunk < 0) break;
-                const int64_t row0 = chunk;
-                const int rows = stage_rows(row0, pool_row0, RS, RSH, p.V);
-                const float *sc = scores + s * RS * NB;
+            if constexpr (MM == 0) {
+                // ---------------- selector (wide lists) ----------------
+                uint64_t *sbuf = reinterpret_cast<uint64_t *>(smem + L.sel);
+                const int cap = p.sel_cap;
+                const unsigned lt_mask = (1u << lane) - 1u;
+                int cnt[NB];
+                uint64_t tau[NB];
 #pragma unroll
                 for (int nb = 0; nb < NB; ++nb) {
-                    if (nb >= p.nq) break;
-                    for (int rb = 0; rb < rows; rb += 32) {
-                        const int r = rb + lane;
-                        const uint64_t key =
-                            (r < rows) ? make_key(sc[r * NB + nb], static_cast<uint32_t>(row0 + r)) : 0;
-                        unsigned m = __ballot_sync(0xFFFFFFFFu, key > tau[nb]);
-                        while (m) {
-                            const int srcl = __ffs(m) - 1;
-                            m &= m - 1;
-                            const uint64_t x = shfl_u64(key, srcl);
-                            if (x > tau[nb]) {
-                                list[nb].insert(x, lane);
-                                tau[nb] = list[nb].at(p.k - 1);
+                    cnt[nb] = 0;
+                    tau[nb] = 0;
+                }
+                for (int t = 0;; ++t) {
+                    const int s = t % kScoreStages, u = t / kScoreStages;
+                    if (!mbar_wait(&sfull[s], u & 1, abort_flag)) {
+                        if (lane == 0) {
+                            atomicOr(p.err, kErrWaitTimeout);
+                            ms->abort = 1;
+                        }
+                        break;
+                    }
+                    const int chunk = ms->chunk_s[s];
+                    if (chunk < 0) break;
+                    const int64_t row0 = chunk;
+                    const int rows = stage_rows(row0, pool_row0, RS, RSH, p.V);
+                    const float *sc = scores + s * RS * NB;
+#pragma unroll
+                    for (int nb = 0; nb < NB; ++nb) {
+                        if (nb >= p.nq) break;
+                        uint64_t *buf = sbuf + nb * cap;
+                        for (int rb = 0; rb < rows; rb += 32) {
+                            if (cnt[nb] > cap - 32) {  // no room for another 32 keys: keep the best k
+                                tau[nb] = warp_cut_to_best(buf, cnt[nb], p.k, lane);
+                                cnt[nb] = p.k;
+                            }
+                            const int r = rb + lane;
+                            const uint64_t key =
+                                (r < rows) ? make_key(sc[r * NB + nb], static_cast<uint32_t>(row0 + r)) : 0;
+                            const bool in = key > tau[nb];
+                            const unsigned m = __ballot_sync(0xFFFFFFFFu, in);
+                            if (in) buf[cnt[nb] + __popc(m & lt_mask)] = key;
+                            cnt[nb] += __popc(m);
+                        }
+                    }
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(&sempty[s]);
+                }
+                if (lane == 0) {
+#pragma unroll
+                    for (int nb = 0; nb < NB; ++nb) ms->sel_cnt[nb] = nb < p.nq ? cnt[nb] : 0;
+                }
+            } else {
+                // ---------------- selector ----------------
+                WarpList<MM> list[NB];
+                uint64_t tau[NB];
+#pragma unroll
+                for (int nb = 0; nb < NB; ++nb) {
+                    list[nb].clear();
+                    tau[nb] = 0;
+                }
+                for (int t = 0;; ++t) {
+                    const int s = t % kScoreStages, u = t / kScoreStages;
+                    if (!mbar_wait(&sfull[s], u & 1, abort_flag)) {
+                        if (lane == 0) {
+                            atomicOr(p.err, kErrWaitTimeout);
+                            ms->abort = 1;
+                        }
+                        break;
+                    }
+                    const int chunk = ms->chunk_s[s];
+                    if (chunk < 0) break;
+                    const int64_t row0 = chunk;
+                    const int rows = stage_rows(row0, pool_row0, RS, RSH, p.V);
+                    const float *sc = scores + s * RS * NB;
+#pragma unroll
+                    for (int nb = 0; nb < NB; ++nb) {
+                        if (nb >= p.nq) break;
+                        for (int rb = 0; rb < rows; rb += 32) {
+                            const int r = rb + lane;
+                            const uint64_t key =
+                                (r < rows) ? make_key(sc[r * NB + nb], static_cast<uint32_t>(row0 + r)) : 0;
+                            unsigned m = __ballot_sync(0xFFFFFFFFu, key > tau[nb]);
+                            while (m) {
+                                const int srcl = __ffs(m) - 1;
+                                m &= m - 1;
+                                const uint64_t x = shfl_u64(key, srcl);
+                                if (x > tau[nb]) {
+                                    list[nb].insert(x, lane);
+                                    tau[nb] = list[nb].at(p.k - 1);
+                                }
                             }
                         }
                     }
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(&sempty[s]);
                 }
-                __syncwarp();
-                if (lane == 0) mbar_arrive(&sempty[s]);
-            }
-            // this CTA's sorted top-k per query -> scratch
+                // this CTA's sorted top-k per query -> scratch
 #pragma unroll
-            for (int nb = 0; nb < NB; ++nb) {
-                uint64_t *dst = p.cand + (static_cast<size_t>(nb) * G + cta) * p.k;
-                uint64_t *head = p.heads + (static_cast<size_t>(nb) * G + cta) * kFastE;
+                for (int nb = 0; nb < NB; ++nb) {
+                    uint64_t *dst = p.cand + (static_cast<size_t>(nb) * G + cta) * p.k;
+                    uint64_t *head = p.heads + (static_cast<size_t>(nb) * G + cta) * kFastE;
 #pragma unroll
-                for (int s = 0; s < MM; ++s) {
-                    const int pos = lane * MM + s;
-                    if (pos < p.k) dst[pos] = list[nb].v[s];
-                    if (pos < kFastE) head[pos] = pos < p.k ? list[nb].v[s] : 0ull;
+                    for (int s = 0; s < MM; ++s) {
+                        const int pos = lane * MM + s;
+                        if (pos < p.k) dst[pos] = list[nb].v[s];
+                        if (pos < kFastE) head[pos] = pos < p.k ? list[nb].v[s] : 0ull;
+                    }
                 }
             }
         } else {
@@ -1015,6 +1300,19 @@ __global__ void __launch_bounds__(kThreads, 1) stream_topk_kernel(const StreamTo
         }
     }
 
+    // ---------------- wide lists: buffers -> sorted lists ----------------
+    // (the ring is free: every stage was consumed before its role ended)
+    if constexpr (MM == 0) {
+        __syncthreads();
+        uint32_t *hist = reinterpret_cast<uint32_t *>(smem + L.ring);
+        uint64_t *win = reinterpret_cast<uint64_t *>(smem + L.ring + 1024);
+        uint64_t *sbuf = reinterpret_cast<uint64_t *>(smem + L.sel);
+        for (int nb = 0; nb < p.nq; ++nb)
+            write_cta_list(sbuf + nb * p.sel_cap, ms->sel_cnt[nb], p.k, hist, win, ms,
+                           p.cand + (static_cast<size_t>(nb) * G + cta) * p.k,
+                           p.heads + (static_cast<size_t>(nb) * G + cta) * kFastE);
+    }
+
     // ---------------- early merge (one query, k <= 64) ----------------
     // bar.sync orders every thread's writes (list, heads, sparse fill) before
     // thread 0's release store of this launch's epoch + 1; CTA 0 acquires each
@@ -1033,6 +1331,41 @@ __global__ void __launch_bounds__(kThreads, 1) stream_topk_kernel(const StreamTo
         if (tid == 0) {
             *p.next_chunk = 0;  // re-arm the pool for the next launch
             *reinterpret_cast<volatile uint32_t *>(p.epoch) = target;
+        }
+        return;
+    }
+
+    // ---------------- publication, then the merge (first X CTAs) ----------------
+    // Several queries: the release store and the epoch as in the early merge;
+    // a relaxed ticket ranks the CTAs by finishing order, the first X merge
+    // (queries m, m + X, ...) while the others still stream, and the last
+    // re-arms the pool and the ticket and advances the epoch (every CTA has
+    // drawn its last chunk and taken its ticket by then).
+    if (p.pmerge) {
+        __syncthreads();
+        const int X = min(p.nq, G);
+        const uint32_t target = ms->epoch + 1u;
+        if (tid == 0) {
+            st_release_gpu(p.flags + cta, target);
+            const uint32_t ticket = atomic_add_relaxed_gpu(p.ticket, 1u);
+            if (ticket == static_cast<uint32_t>(G - 1)) {
+                *p.next_chunk = 0;
+                *p.ticket = 0;
+                *reinterpret_cast<volatile uint32_t *>(p.epoch) = target;
+            }
+            ms->merger = ticket < static_cast<uint32_t>(X) ? static_cast<int>(ticket) : -1;
+        }
+        __syncthreads();
+        const int mg = ms->merger;
+        if (mg < 0) return;
+        unsigned char *ws = smem + L.merge;
+        uint64_t *fe = reinterpret_cast<uint64_t *>(ws + SmemLayout::merge_fixed_bytes());
+        for (int q = mg; q < p.nq; q += X) {
+            merge_published(p.flags, target, p.heads + static_cast<size_t>(q) * G * kFastE,
+                            p.cand + static_cast<size_t>(q) * G * p.k, G, p.k, ws, fe, ms, p.err,
+                            p.out_idx + static_cast<size_t>(q) * p.k, p.out_logits + static_cast<size_t>(q) * p.k,
+                            p.sparse != nullptr ? p.sparse + static_cast<int64_t>(q) * p.V : nullptr);
+            __syncthreads();
         }
         return;
     }

@@ -26,15 +26,10 @@ cudaError_t launch_one(const StreamTopkParams &p, int grid, uint32_t smem, cudaS
 template <int NB, int R, bool Q8>
 cudaError_t launch_rows(int mm, const StreamTopkParams &p, int grid, uint32_t smem,
                         cudaStream_t stream) {
-    // Wide lists are only built for narrow query groups (register budget).
+    // 2: register lists (k <= 64); 0: shared-memory candidate buffers
     switch (mm) {
         case 2: return launch_one<NB, 2, R, Q8>(p, grid, smem, stream);
-        case 8:
-            if constexpr (NB <= 4) return launch_one<NB, 8, R, Q8>(p, grid, smem, stream);
-            return cudaErrorInvalidValue;
-        case 32:
-            if constexpr (NB == 1) return launch_one<NB, 32, R, Q8>(p, grid, smem, stream);
-            return cudaErrorInvalidValue;
+        case 0: return launch_one<NB, 0, R, Q8>(p, grid, smem, stream);
         default: return cudaErrorInvalidValue;
     }
 }

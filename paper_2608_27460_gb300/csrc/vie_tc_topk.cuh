@@ -178,43 +178,6 @@ __device__ __forceinline__ float e4m3_value(uint8_t c) {
     return __half2float(__half(__nv_cvt_fp8_to_halfraw(static_cast<__nv_fp8_storage_t>(c), __NV_E4M3)));
 }
 
-// Bitonic sort, descending, of the 32 * PER keys a warp holds (lane l holds
-// elements l*PER .. l*PER + PER - 1).  Steps with a stride below PER swap
-// registers; wider steps exchange with lane ^ (stride / PER).
-template <int PER>
-__device__ __forceinline__ void warp_sort_desc(uint64_t (&v)[PER], int lane) {
-#pragma unroll
-    for (int size = 2; size <= 32 * PER; size <<= 1) {
-#pragma unroll
-        for (int stride = size >> 1; stride > 0; stride >>= 1) {
-            if (stride < PER) {
-#pragma unroll
-                for (int j = 0; j < PER; ++j) {
-                    const int pj = j ^ stride;
-                    if (pj > j) {
-                        const bool desc = ((lane * PER + j) & size) == 0;
-                        const uint64_t a = v[j], b = v[pj];
-                        if (desc ? (a < b) : (a > b)) {
-                            v[j] = b;
-                            v[pj] = a;
-                        }
-                    }
-                }
-            } else {
-                const int ls = stride / PER;
-                const bool lower = (lane & ls) == 0;
-#pragma unroll
-                for (int j = 0; j < PER; ++j) {
-                    const uint64_t o = shfl_xor_u64(v[j], ls);
-                    const bool desc = ((lane * PER + j) & size) == 0;
-                    const bool keep_max = lower == desc;
-                    v[j] = keep_max ? (v[j] > o ? v[j] : o) : (v[j] < o ? v[j] : o);
-                }
-            }
-        }
-    }
-}
-
 // Keeps the k largest of the cnt (k < cnt <= 32 * PER) nonzero keys in buf, unsorted at
 // buf[0..k), and returns k; *tau becomes a bound T <= the k-th key such that
 // exactly k keys are >= T.  T is found by bisection: first on the high words

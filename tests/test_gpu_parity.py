@@ -31,9 +31,9 @@ def test_hand_worked_case_exact(vie):
     (20011, 640, 1, 50),     # ragged CTA slices and stages
     (20011, 640, 3, 1),      # greedy, odd batch
     (33333, 1024, 2, 64),    # largest short-list k
-    (33333, 1152, 4, 65),    # first k of the middle list width
+    (33333, 1152, 4, 65),    # k = 65 on the tensor cores (batch 4)
     (9973, 256, 5, 256),
-    (9973, 256, 1, 257),     # first k of the widest list
+    (9973, 256, 1, 257),     # streaming wide lists, a 576-key buffer
     (70001, 512, 8, 50),     # widest query group
     (70001, 512, 13, 50),    # two query groups
     (5000, 2048, 1, 1024),   # largest k

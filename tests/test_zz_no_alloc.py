@@ -29,6 +29,8 @@ pytestmark = pytest.mark.gpu
     (5000, 64, 1, 1),        # 79 CTAs x k = 1: an odd number of list keys
     (5000, 64, 1, 3),        # 79 x 3 keys: odd again
     (5000, 64, 3, 3),        # 4 slots x 79 x 3: even, three queries
+    (30011, 64, 3, 150),     # wide lists: 320-key candidate buffers, 4 slots
+    (30011, 64, 1, 600),     # wide lists, one 1216-key buffer
 ])
 def test_noalloc_matches_oracle_and_head_topk_twice(vie, V, d, batch, k):
     import torch
