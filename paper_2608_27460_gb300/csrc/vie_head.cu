@@ -180,12 +180,15 @@ namespace {
 // k <= 64, else (0) the shared-memory candidate buffers of the wide lists.
 int pick_mm(int k) { return k <= vie::kFastMaxK ? 2 : 0; }
 
-// Keys per query of a launch's candidate buffers (wide lists): one query
-// gets 2048 (no cut-back while a CTA streams up to ~2000 rows), groups the
-// least size for k.
+// Keys per query of a launch's candidate buffers (wide lists): a single
+// query gets about 4k (its first cut-back comes early in the stream, where it
+// is hidden, and usually stays the only one; the CTA's final selection then
+// sorts a few k keys, not every row it streamed), groups the least size for k.
 int sel_cap_launch(int nb, int k) {
     const int c = vie::sel_cap_for(k);
-    return (nb == 1 && c > 0 && c < 2048) ? 2048 : c;
+    if (nb != 1 || c == 0) return c;
+    const int c4 = (4 * k + 63) & ~63;
+    return c4 > kMaxSelBytes / 8 ? kMaxSelBytes / 8 : c4;
 }
 
 // Widest query group for a row width and k: the staged queries and the wide

@@ -12,23 +12,25 @@
 //              shared-memory stages (mbarrier transaction counts, L2
 //              evict-first); the chunk id travels with the stage; an id of
 //              -1 closes the stream;
-//   warps 2-9  projection: warp w owns rows w, w+8, .. (at most R) of each
-//              stage and every lane a strided set of 16-byte column chunks;
-//              bf16 -> fp32 widening, fp32 FMA against h (staged in shared
-//              memory, one load per chunk reused for the warp's rows).  The
-//              stage is released as soon as its last shared-memory read
-//              retires; the warp-shuffle sums then go to a separate, deeper
-//              score ring;
-//   warp 1     selector: keeps the best keys seen so far as a sorted list
-//              spread over the warp's registers; a row enters only if it
-//              beats the current k-th key.  It never holds a weight stage.
-//              Wide lists (k > 64): every key above the bound tau goes into
-//              a shared-memory buffer of the query (ballot and append); a
-//              full buffer is cut back to its best k by a bisection on the
-//              keys, which raises tau to the k-th of them.  After the stream
-//              the whole CTA turns each buffer into the sorted list (radix
-//              select of the best k, sorted runs of 128 keys in registers,
-//              then each key's place from binary searches in the other runs).
+//   warps 1..NS  selectors, NS = one per query up to four (selector s takes
+//              query slots s, s + NS, ..): per query, the best keys seen so
+//              far as a sorted list spread over the warp's registers; a row
+//              enters only if it beats the current k-th key.  They never
+//              hold a weight stage.  Wide lists (k > 64): every key above
+//              the bound tau goes into a shared-memory buffer of the query
+//              (ballot and append); a full buffer is cut back to a set
+//              holding its best k by a bisection on the keys, which raises
+//              tau.  After the stream the whole CTA turns each buffer into
+//              the sorted list (radix select of the best k, then a bitonic
+//              sort: runs of 128 keys in registers, merged through shared
+//              memory);
+//   the next 8 warps  projection: warp w owns rows w, w+8, .. (at most R) of
+//              each stage and every lane a strided set of 16-byte column
+//              chunks; bf16 -> fp32 widening, fp32 FMA against h (staged in
+//              shared memory, one load per chunk reused for the warp's
+//              rows).  The stage is released as soon as its last
+//              shared-memory read retires; the warp-shuffle sums then go to
+//              a separate, deeper score ring.
 // The full logit vector never leaves the chip.  Afterwards each CTA writes
 // its sorted top-k list to scratch and takes a ticket (an acq_rel atomic, no
 // full fences); the CTA that draws the last ticket copies every list into
@@ -63,7 +65,14 @@
 namespace vie {
 
 constexpr int kDotWarps = 8;
-constexpr int kThreads = 32 * (2 + kDotWarps);
+constexpr int kThreads = 32 * (2 + kDotWarps);  // single-query launches (the fewest threads)
+
+// Selector warps of a launch with NB query slots, one per query up to four
+// (selector s takes slots s, s + NS, ...), and the launch's thread count.
+template <int NB>
+__host__ __device__ constexpr int sel_warps() { return NB < 4 ? NB : 4; }
+template <int NB>
+__host__ __device__ constexpr int threads_for() { return 32 * (1 + sel_warps<NB>() + kDotWarps); }
 constexpr int kMaxStages = 16;         // weight ring depth limit
 constexpr int kScoreStages = 16;       // score ring depth
 constexpr int kMergePrefixCap = 2048;  // keys: first-J prefixes of all lists
@@ -73,7 +82,7 @@ constexpr int kMaxLists = 1024;        // G <= 1024 CTAs
 constexpr int kFastE = 8;              // fast merge: entries read per list (even)
 constexpr int kFastMaxK = 64;          // fast merge: largest k
 constexpr int kSelRun = 128;           // keys of one sorted run (a warp's registers)
-constexpr int kRankRunsMin = 256;      // ranking by sorted runs above this many keys
+constexpr int kRankRunsMin = 256;      // merge output: a bitonic sort above this many keys
 
 // Keys per query of the shared-memory candidate buffer of the wide lists
 // (k > kFastMaxK): room for k keys and as many again, so a cut-back keeps k
@@ -338,51 +347,91 @@ __device__ __forceinline__ int rank_among(const uint64_t *keys, int n, uint64_t 
     return r0 + r1;
 }
 
-// Descending ranks of the m unique nonzero keys a[0..m) (shared memory):
-// runs of kSelRun keys are each sorted by one warp in its registers (a is
-// rewritten run by run), then a key's rank is its place in its own run plus,
-// per other run, the number of that run's keys above it (binary search).
-// emit(rank, key) is called once per key.  Every thread of the CTA calls it;
-// it ends with a barrier.
-template <class Emit>
-__device__ inline void block_rank_by_runs(uint64_t *a, int m, Emit emit) {
+// The last merge of a warp's sort network: the 32 * PER keys it holds
+// (bitonic) sorted descending by half-cleaners of strides 16 * PER .. 1.
+template <int PER>
+__device__ __forceinline__ void warp_merge_desc(uint64_t (&v)[PER], int lane) {
+#pragma unroll
+    for (int stride = 16 * PER; stride > 0; stride >>= 1) {
+        if (stride < PER) {
+#pragma unroll
+            for (int j = 0; j < PER; ++j) {
+                const int pj = j ^ stride;
+                if (pj > j && v[j] < v[pj]) {
+                    const uint64_t a = v[j];
+                    v[j] = v[pj];
+                    v[pj] = a;
+                }
+            }
+        } else {
+            const int ls = stride / PER;
+            const bool lower = (lane & ls) == 0;
+#pragma unroll
+            for (int j = 0; j < PER; ++j) {
+                const uint64_t o = shfl_xor_u64(v[j], ls);
+                v[j] = lower ? (v[j] > o ? v[j] : o) : (v[j] < o ? v[j] : o);
+            }
+        }
+    }
+}
+
+// Sorts the m unique nonzero keys a[0..m) (shared memory) descending in
+// place.  a must have room for P keys, P the power of two >= max(m,
+// kSelRun); a[m..P) is zero-filled (zeros sort last).  Bitonic: runs of
+// kSelRun keys sorted in registers (a warp each), then per doubling of the
+// sorted length a mirror compare-exchange between the two runs of each pair
+// and half-cleaners of strides >= kSelRun in shared memory, and the strides
+// below kSelRun in registers.  Every thread of the CTA calls it; it ends
+// with a barrier.
+__device__ inline void block_sort_desc(uint64_t *a, int m) {
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int nthr = static_cast<int>(blockDim.x), nw = nthr >> 5;
-    const int nruns = (m + kSelRun - 1) / kSelRun;
     constexpr int PER = kSelRun / 32;
+    int P = kSelRun;
+    while (P < m) P <<= 1;
+    for (int i = m + tid; i < P; i += nthr) a[i] = 0ull;
+    __syncthreads();
+    const int nruns = P / kSelRun;
     for (int r = warp; r < nruns; r += nw) {
         uint64_t v[PER];
 #pragma unroll
-        for (int j = 0; j < PER; ++j) {
-            const int e = r * kSelRun + lane * PER + j;
-            v[j] = e < m ? a[e] : 0ull;
-        }
+        for (int j = 0; j < PER; ++j) v[j] = a[r * kSelRun + lane * PER + j];
         warp_sort_desc<PER>(v, lane);
 #pragma unroll
-        for (int j = 0; j < PER; ++j) {
-            const int e = r * kSelRun + lane * PER + j;
-            if (e < m) a[e] = v[j];  // zeros sort last: the real keys fill the run's front
-        }
+        for (int j = 0; j < PER; ++j) a[r * kSelRun + lane * PER + j] = v[j];
     }
-    __syncthreads();
-    for (int i = tid; i < m; i += nthr) {
-        const uint64_t x = a[i];
-        const int r = i / kSelRun;
-        int rank = i - r * kSelRun;
-        for (int r2 = 0; r2 < nruns; ++r2) {
-            if (r2 == r) continue;
-            const uint64_t *run = a + r2 * kSelRun;
-            int lo = 0, hi = min(kSelRun, m - r2 * kSelRun);
-            while (lo < hi) {
-                const int mid = (lo + hi) >> 1;
-                if (run[mid] > x)
-                    lo = mid + 1;
-                else
-                    hi = mid;
+    for (int size = 2 * kSelRun; size <= P; size <<= 1) {
+        const int half = size >> 1;
+        __syncthreads();
+        for (int i = tid; i < (P >> 1); i += nthr) {
+            const int blk = i / half, j = i - blk * half;
+            const int lo = blk * size + j, hi = blk * size + size - 1 - j;
+            const uint64_t x = a[lo], y = a[hi];
+            if (x < y) {
+                a[lo] = y;
+                a[hi] = x;
             }
-            rank += lo;
         }
-        emit(rank, x);
+        for (int stride = half >> 1; stride >= kSelRun; stride >>= 1) {
+            __syncthreads();
+            for (int i = tid; i < (P >> 1); i += nthr) {
+                const int lo = (i / stride) * 2 * stride + (i % stride), hi = lo + stride;
+                const uint64_t x = a[lo], y = a[hi];
+                if (x < y) {
+                    a[lo] = y;
+                    a[hi] = x;
+                }
+            }
+        }
+        __syncthreads();
+        for (int r = warp; r < nruns; r += nw) {
+            uint64_t v[PER];
+#pragma unroll
+            for (int j = 0; j < PER; ++j) v[j] = a[r * kSelRun + lane * PER + j];
+            warp_merge_desc<PER>(v, lane);
+#pragma unroll
+            for (int j = 0; j < PER; ++j) a[r * kSelRun + lane * PER + j] = v[j];
+        }
     }
     __syncthreads();
 }
@@ -410,14 +459,16 @@ __device__ inline void block_topk_to_output(uint64_t *keys, int n, int k, uint64
         m = k;
     }
     if (m > kRankRunsMin) {
-        // many keys: sorted runs and binary searches (rank counting is m^2)
-        block_rank_by_runs(src, m, [&](int rank, uint64_t x) {
-            if (rank < k) {
-                out_idx[rank] = key_index(x);
-                out_logits[rank] = key_value(x);
-                if (sparse_row != nullptr) sparse_row[key_index(x)] = key_value(x);
-            }
-        });
+        // many keys: a bitonic sort (rank counting is m^2); src has room for
+        // the sort's power of two (at most 1024 keys here)
+        block_sort_desc(src, m);
+        for (int i = tid; i < min(m, k); i += static_cast<int>(blockDim.x)) {
+            const uint64_t x = src[i];
+            out_idx[i] = key_index(x);
+            out_logits[i] = key_value(x);
+            if (sparse_row != nullptr) sparse_row[key_index(x)] = key_value(x);
+        }
+        __syncthreads();
         return;
     }
     for (int i = tid; i < m; i += static_cast<int>(blockDim.x)) {
@@ -432,21 +483,26 @@ __device__ inline void block_topk_to_output(uint64_t *keys, int n, int k, uint64
     __syncthreads();
 }
 
-// Wide lists: cuts the cnt (> k) unique nonzero keys of buf back to its best
-// k, moved to buf[0..k), and returns the k-th largest key (the new entry
-// bound).  One warp.  The k-th key is found one digit at a time: two bits of
-// the high word (the ordered logit) per step, from three independent counts
-// of keys at or above the candidates; then, when several keys share that
-// logit, two bits per step of the low word (the inverted row) among them.
-// Each step reads the buffer from shared memory.
-static __device__ __noinline__ uint64_t warp_cut_to_best(uint64_t *buf, int cnt, int k, int lane) {
+// Wide lists: cuts the cnt (> k) unique nonzero keys of buf back to a set
+// that holds its best k, moved to buf[0..), and returns its size and the new
+// entry bound (a later key enters only if it is above the bound).
+// One warp.  The cut is found one digit at a time, two bits per step from
+// three independent counts, each step reading the buffer from shared
+// memory: first the top 16 bits of the high word (the ordered logit); if
+// the keys at or above that coarse threshold are at most `room`, they are
+// kept (at least k of them).  Otherwise the rest of the high word and then,
+// when several keys share the k-th logit, the low word (the inverted row)
+// give the exact k-th key, and exactly k keys are kept.
+struct CutBack {
+    int n;
+    uint64_t bound;
+};
+static __device__ __noinline__ CutBack warp_cut_back(uint64_t *buf, int cnt, int k, int room, int lane) {
     __syncwarp();
     const uint32_t *w32 = reinterpret_cast<const uint32_t *>(buf);
-    uint32_t th = 0;
-#pragma unroll 1
-    for (int bit = 30; bit >= 0; bit -= 2) {
-        const uint32_t c1 = th | (1u << bit), c2 = th | (2u << bit), c3 = th | (3u << bit);
-        int n1 = 0, n2 = 0, n3 = 0;
+    auto count3 = [&](uint32_t c1, uint32_t c2, uint32_t c3, int &n1, int &n2, int &n3) {
+        n1 = n2 = n3 = 0;
+#pragma unroll 4
         for (int e = lane; e < cnt; e += 32) {
             const uint32_t hi = w32[2 * e + 1];
             n1 += hi >= c1 ? 1 : 0;
@@ -456,37 +512,59 @@ static __device__ __noinline__ uint64_t warp_cut_to_best(uint64_t *buf, int cnt,
         n1 = static_cast<int>(__reduce_add_sync(0xFFFFFFFFu, n1));
         n2 = static_cast<int>(__reduce_add_sync(0xFFFFFFFFu, n2));
         n3 = static_cast<int>(__reduce_add_sync(0xFFFFFFFFu, n3));
+    };
+    uint32_t th = 0;
+    int n1, n2, n3;
+#pragma unroll 1
+    for (int bit = 30; bit >= 16; bit -= 2) {
+        const uint32_t c1 = th | (1u << bit), c2 = th | (2u << bit), c3 = th | (3u << bit);
+        count3(c1, c2, c3, n1, n2, n3);
         th = n3 >= k ? c3 : (n2 >= k ? c2 : (n1 >= k ? c1 : th));
     }
-    int n_gt = 0, n_ge = 0;
-    for (int e = lane; e < cnt; e += 32) {
-        const uint32_t hi = w32[2 * e + 1];
-        n_gt += hi > th ? 1 : 0;
-        n_ge += hi >= th ? 1 : 0;
-    }
-    n_gt = static_cast<int>(__reduce_add_sync(0xFFFFFFFFu, n_gt));
+    int n_ge = 0;
+    for (int e = lane; e < cnt; e += 32) n_ge += w32[2 * e + 1] >= th ? 1 : 0;
     n_ge = static_cast<int>(__reduce_add_sync(0xFFFFFFFFu, n_ge));
-    uint32_t tl = 0;
-    if (n_ge > k) {
-        const int need = k - n_gt;  // keys still needed among those with logit th
+    uint64_t T;
+    if (th != 0 && n_ge <= room) {
+        T = static_cast<uint64_t>(th) << 32;  // keys >= T: n_ge of them, at least k
+    } else {
 #pragma unroll 1
-        for (int bit = 30; bit >= 0; bit -= 2) {
-            const uint32_t c1 = tl | (1u << bit), c2 = tl | (2u << bit), c3 = tl | (3u << bit);
-            int n1 = 0, n2 = 0, n3 = 0;
-            for (int e = lane; e < cnt; e += 32) {
-                if (w32[2 * e + 1] != th) continue;
-                const uint32_t lo = w32[2 * e];
-                n1 += lo >= c1 ? 1 : 0;
-                n2 += lo >= c2 ? 1 : 0;
-                n3 += lo >= c3 ? 1 : 0;
-            }
-            n1 = static_cast<int>(__reduce_add_sync(0xFFFFFFFFu, n1));
-            n2 = static_cast<int>(__reduce_add_sync(0xFFFFFFFFu, n2));
-            n3 = static_cast<int>(__reduce_add_sync(0xFFFFFFFFu, n3));
-            tl = n3 >= need ? c3 : (n2 >= need ? c2 : (n1 >= need ? c1 : tl));
+        for (int bit = 14; bit >= 0; bit -= 2) {
+            const uint32_t c1 = th | (1u << bit), c2 = th | (2u << bit), c3 = th | (3u << bit);
+            count3(c1, c2, c3, n1, n2, n3);
+            th = n3 >= k ? c3 : (n2 >= k ? c2 : (n1 >= k ? c1 : th));
         }
+        int n_gt = 0;
+        n_ge = 0;
+        for (int e = lane; e < cnt; e += 32) {
+            const uint32_t hi = w32[2 * e + 1];
+            n_gt += hi > th ? 1 : 0;
+            n_ge += hi >= th ? 1 : 0;
+        }
+        n_gt = static_cast<int>(__reduce_add_sync(0xFFFFFFFFu, n_gt));
+        n_ge = static_cast<int>(__reduce_add_sync(0xFFFFFFFFu, n_ge));
+        uint32_t tl = 0;
+        if (n_ge > k) {
+            const int need = k - n_gt;  // keys still needed among those with logit th
+#pragma unroll 1
+            for (int bit = 30; bit >= 0; bit -= 2) {
+                const uint32_t c1 = tl | (1u << bit), c2 = tl | (2u << bit), c3 = tl | (3u << bit);
+                int m1 = 0, m2 = 0, m3 = 0;
+                for (int e = lane; e < cnt; e += 32) {
+                    if (w32[2 * e + 1] != th) continue;
+                    const uint32_t lo = w32[2 * e];
+                    m1 += lo >= c1 ? 1 : 0;
+                    m2 += lo >= c2 ? 1 : 0;
+                    m3 += lo >= c3 ? 1 : 0;
+                }
+                m1 = static_cast<int>(__reduce_add_sync(0xFFFFFFFFu, m1));
+                m2 = static_cast<int>(__reduce_add_sync(0xFFFFFFFFu, m2));
+                m3 = static_cast<int>(__reduce_add_sync(0xFFFFFFFFu, m3));
+                tl = m3 >= need ? c3 : (m2 >= need ? c2 : (m1 >= need ? c1 : tl));
+            }
+        }
+        T = (static_cast<uint64_t>(th) << 32) | tl;  // the k-th key: exactly k keys >= T
     }
-    const uint64_t T = (static_cast<uint64_t>(th) << 32) | tl;
     // in place: every write lands at or below the position it was read from
     // in this pass, after the whole warp has read that block of 32
     const unsigned lt_mask = (1u << lane) - 1u;
@@ -500,14 +578,16 @@ static __device__ __noinline__ uint64_t warp_cut_to_best(uint64_t *buf, int cnt,
         base += __popc(m);
     }
     __syncwarp();
-    return T;
+    // entry bound: a key enters if > bound, i.e. >= T (keys are never equal)
+    return CutBack{base, T - 1};
 }
 
 // Wide lists, after the stream: the sorted list of one query's buffer (cnt
 // unique nonzero keys; cnt may exceed k) written best first to dst[0..k)
 // (zeros after the real keys) and its first kFastE keys to head.  Every
-// thread of the CTA calls it.  win (k keys) and hist (256 words) are free
-// shared memory; buf is sorted in place when it holds at most k keys.
+// thread of the CTA calls it.  win (room for the power of two >= k, at least
+// kSelRun keys) and hist (256 words) are free shared memory; buf (room for
+// 2k keys) is sorted in place when it holds at most k keys.
 __device__ inline void write_cta_list(uint64_t *buf, int cnt, int k, uint32_t *hist, uint64_t *win,
                                       MiscSmem *ms, uint64_t *dst, uint64_t *head) {
     const int tid = threadIdx.x, nthr = static_cast<int>(blockDim.x);
@@ -526,10 +606,11 @@ __device__ inline void write_cta_list(uint64_t *buf, int cnt, int k, uint32_t *h
         m = k;
     }
     __syncthreads();
-    block_rank_by_runs(a, m, [&](int rank, uint64_t x) {
-        dst[rank] = x;
-        if (rank < kFastE) head[rank] = x;
-    });
+    block_sort_desc(a, m);  // room: win holds k keys; buf at least 2k when cnt <= k
+    for (int i = tid; i < m; i += nthr) {
+        dst[i] = a[i];
+        if (i < kFastE) head[i] = a[i];
+    }
     for (int i = m + tid; i < k; i += nthr) dst[i] = 0ull;
     for (int i = m + tid; i < kFastE; i += nthr) head[i] = 0ull;
 }
@@ -922,7 +1003,8 @@ __device__ __forceinline__ float fma_e4m3x4(uint32_t w, float4 h, float a) {
 // Q8: rows of e4m3 codes (16 per 16-byte chunk) with one fp32 scale per row,
 // logit = scale * sum; otherwise bf16 rows (8 per chunk).
 template <int NB, int MM, int R, bool Q8>
-__global__ void __launch_bounds__(kThreads, 1) stream_topk_kernel(const StreamTopkParams p) {
+__global__ void __launch_bounds__(threads_for<NB>(), 1) stream_topk_kernel(const StreamTopkParams p) {
+    constexpr int NS = sel_warps<NB>(), T = threads_for<NB>(), QPS = NB / NS;
     extern __shared__ __align__(128) unsigned char smem[];
     const int RS = p.rows_per_stage;  // <= 8 * R
     const int S = p.stages;
@@ -956,7 +1038,7 @@ __global__ void __launch_bounds__(kThreads, 1) stream_topk_kernel(const StreamTo
         }
         for (int s = 0; s < kScoreStages; ++s) {
             mbar_init(&sfull[s], kDotWarps);
-            mbar_init(&sempty[s], 1);
+            mbar_init(&sempty[s], NS);
         }
         ms->abort = 0;
         ms->is_last = 0;
@@ -970,7 +1052,7 @@ __global__ void __launch_bounds__(kThreads, 1) stream_topk_kernel(const StreamTo
     // starts, so h is ahead of the weight stream in the memory queues; those
     // warps wait for them after the barrier (bar.sync 1 below).
     if (warp > 0) {
-        for (int i = tid - 32; i < NB * p.d_pad; i += kThreads - 32) {
+        for (int i = tid - 32; i < NB * p.d_pad; i += T - 32) {
             const int nb = i / p.d_pad, j = i - nb * p.d_pad;
             const bool real = nb < p.nq && j < p.d;
             const float *src = real ? p.h + static_cast<int64_t>(nb) * p.d + j : p.h;
@@ -1041,23 +1123,24 @@ __global__ void __launch_bounds__(kThreads, 1) stream_topk_kernel(const StreamTo
             const int64_t fn = base + (cta < rem ? 1 : 0);
             for (int q = 0; q < p.nq; ++q) {
                 float *row = p.sparse + static_cast<int64_t>(q) * p.V + f0;
-                for (int64_t i = tid - 32; i < fn; i += kThreads - 32) row[i] = ninf;
+                for (int64_t i = tid - 32; i < fn; i += T - 32) row[i] = ninf;
             }
         }
         cp_async_wait_all();
-        named_barrier_sync(1, kThreads - 32);  // h in shared memory for warps 1..
-        if (warp == 1) {
+        named_barrier_sync(1, T - 32);  // h in shared memory for warps 1..
+        if (warp <= NS) {
+            const int sw = NS == 1 ? 0 : warp - 1;  // this selector's query slots: sw, sw + NS, ...
             if constexpr (MM == 0) {
                 // ---------------- selector (wide lists) ----------------
                 uint64_t *sbuf = reinterpret_cast<uint64_t *>(smem + L.sel);
                 const int cap = p.sel_cap;
                 const unsigned lt_mask = (1u << lane) - 1u;
-                int cnt[NB];
-                uint64_t tau[NB];
+                int cnt[QPS];
+                uint64_t tau[QPS];
 #pragma unroll
-                for (int nb = 0; nb < NB; ++nb) {
-                    cnt[nb] = 0;
-                    tau[nb] = 0;
+                for (int j = 0; j < QPS; ++j) {
+                    cnt[j] = 0;
+                    tau[j] = 0;
                 }
                 for (int t = 0;; ++t) {
                     const int s = t % kScoreStages, u = t / kScoreStages;
@@ -1074,21 +1157,23 @@ __global__ void __launch_bounds__(kThreads, 1) stream_topk_kernel(const StreamTo
                     const int rows = stage_rows(row0, pool_row0, RS, RSH, p.V);
                     const float *sc = scores + s * RS * NB;
 #pragma unroll
-                    for (int nb = 0; nb < NB; ++nb) {
+                    for (int j = 0; j < QPS; ++j) {
+                        const int nb = sw + j * NS;
                         if (nb >= p.nq) break;
                         uint64_t *buf = sbuf + nb * cap;
                         for (int rb = 0; rb < rows; rb += 32) {
-                            if (cnt[nb] > cap - 32) {  // no room for another 32 keys: keep the best k
-                                tau[nb] = warp_cut_to_best(buf, cnt[nb], p.k, lane);
-                                cnt[nb] = p.k;
+                            if (cnt[j] > cap - 32) {  // no room for another 32 keys: cut back
+                                const CutBack cb = warp_cut_back(buf, cnt[j], p.k, (cap + p.k) / 2, lane);
+                                cnt[j] = cb.n;
+                                tau[j] = cb.bound;
                             }
                             const int r = rb + lane;
                             const uint64_t key =
                                 (r < rows) ? make_key(sc[r * NB + nb], static_cast<uint32_t>(row0 + r)) : 0;
-                            const bool in = key > tau[nb];
+                            const bool in = key > tau[j];
                             const unsigned m = __ballot_sync(0xFFFFFFFFu, in);
-                            if (in) buf[cnt[nb] + __popc(m & lt_mask)] = key;
-                            cnt[nb] += __popc(m);
+                            if (in) buf[cnt[j] + __popc(m & lt_mask)] = key;
+                            cnt[j] += __popc(m);
                         }
                     }
                     __syncwarp();
@@ -1096,16 +1181,16 @@ __global__ void __launch_bounds__(kThreads, 1) stream_topk_kernel(const StreamTo
                 }
                 if (lane == 0) {
 #pragma unroll
-                    for (int nb = 0; nb < NB; ++nb) ms->sel_cnt[nb] = nb < p.nq ? cnt[nb] : 0;
+                    for (int j = 0; j < QPS; ++j) ms->sel_cnt[sw + j * NS] = sw + j * NS < p.nq ? cnt[j] : 0;
                 }
             } else {
                 // ---------------- selector ----------------
-                WarpList<MM> list[NB];
-                uint64_t tau[NB];
+                WarpList<MM> list[QPS];
+                uint64_t tau[QPS];
 #pragma unroll
-                for (int nb = 0; nb < NB; ++nb) {
-                    list[nb].clear();
-                    tau[nb] = 0;
+                for (int j = 0; j < QPS; ++j) {
+                    list[j].clear();
+                    tau[j] = 0;
                 }
                 for (int t = 0;; ++t) {
                     const int s = t % kScoreStages, u = t / kScoreStages;
@@ -1122,20 +1207,21 @@ __global__ void __launch_bounds__(kThreads, 1) stream_topk_kernel(const StreamTo
                     const int rows = stage_rows(row0, pool_row0, RS, RSH, p.V);
                     const float *sc = scores + s * RS * NB;
 #pragma unroll
-                    for (int nb = 0; nb < NB; ++nb) {
+                    for (int j = 0; j < QPS; ++j) {
+                        const int nb = sw + j * NS;
                         if (nb >= p.nq) break;
                         for (int rb = 0; rb < rows; rb += 32) {
                             const int r = rb + lane;
                             const uint64_t key =
                                 (r < rows) ? make_key(sc[r * NB + nb], static_cast<uint32_t>(row0 + r)) : 0;
-                            unsigned m = __ballot_sync(0xFFFFFFFFu, key > tau[nb]);
+                            unsigned m = __ballot_sync(0xFFFFFFFFu, key > tau[j]);
                             while (m) {
                                 const int srcl = __ffs(m) - 1;
                                 m &= m - 1;
                                 const uint64_t x = shfl_u64(key, srcl);
-                                if (x > tau[nb]) {
-                                    list[nb].insert(x, lane);
-                                    tau[nb] = list[nb].at(p.k - 1);
+                                if (x > tau[j]) {
+                                    list[j].insert(x, lane);
+                                    tau[j] = list[j].at(p.k - 1);
                                 }
                             }
                         }
@@ -1143,22 +1229,24 @@ __global__ void __launch_bounds__(kThreads, 1) stream_topk_kernel(const StreamTo
                     __syncwarp();
                     if (lane == 0) mbar_arrive(&sempty[s]);
                 }
-                // this CTA's sorted top-k per query -> scratch
+                // this CTA's sorted top-k per query -> scratch (every slot,
+                // zeros for the unused ones)
 #pragma unroll
-                for (int nb = 0; nb < NB; ++nb) {
+                for (int j = 0; j < QPS; ++j) {
+                    const int nb = sw + j * NS;
                     uint64_t *dst = p.cand + (static_cast<size_t>(nb) * G + cta) * p.k;
                     uint64_t *head = p.heads + (static_cast<size_t>(nb) * G + cta) * kFastE;
 #pragma unroll
                     for (int s = 0; s < MM; ++s) {
                         const int pos = lane * MM + s;
-                        if (pos < p.k) dst[pos] = list[nb].v[s];
-                        if (pos < kFastE) head[pos] = pos < p.k ? list[nb].v[s] : 0ull;
+                        if (pos < p.k) dst[pos] = list[j].v[s];
+                        if (pos < kFastE) head[pos] = pos < p.k ? list[j].v[s] : 0ull;
                     }
                 }
             }
         } else {
             // ---------------- projection ----------------
-            const int w = warp - 2;
+            const int w = warp - 1 - NS;
             int t = 0;
             for (;; ++t) {
                 const int s = t % S, u = t / S;

@@ -19,7 +19,7 @@ cudaError_t launch_one(const StreamTopkParams &p, int grid, uint32_t smem, cudaS
         if (e != cudaSuccess) return e;
         configured[dev] = true;
     }
-    stream_topk_kernel<NB, MM, kR, Q8><<<grid, kThreads, smem, stream>>>(p);
+    stream_topk_kernel<NB, MM, kR, Q8><<<grid, threads_for<NB>(), smem, stream>>>(p);
     return cudaGetLastError();
 }
 
