@@ -82,7 +82,7 @@ constexpr int kMaxLists = 1024;        // G <= 1024 CTAs
 constexpr int kFastE = 8;              // fast merge: entries read per list (even)
 constexpr int kFastMaxK = 64;          // fast merge: largest k
 constexpr int kSelRun = 128;           // keys of one sorted run (a warp's registers)
-constexpr int kRankRunsMin = 256;      // merge output: a bitonic sort above this many keys
+constexpr int kRankRunsMin = kRankCountMax;  // merge output: a bitonic sort above this many keys
 
 // Keys per query of the shared-memory candidate buffer of the wide lists
 // (k > kFastMaxK): room for k keys and as many again, so a cut-back keeps k
