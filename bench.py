@@ -68,6 +68,8 @@ def parse_args(argv=None):
                     help="skip the per_config sweep over every workload, batch and k")
     ap.add_argument("--config-steps", type=int, default=50,
                     help="timed steps of each per_config entry (each parity-checked)")
+    ap.add_argument("--config-warmup", type=int, default=10,
+                    help="warm-up steps of each per_config entry (run like the timed ones)")
     ap.add_argument("--long-parity-steps", type=int, default=1000,
                     help="distinct decode steps of the Qwen3-0.6B-shaped b = 1 entry, every one "
                          "timed and checked against the oracle")
@@ -599,8 +601,8 @@ def per_config_sweep(args, torch, vie, dev, stream, flush, peaks, peak_src, cach
         steps, nb = args.config_steps, (8 if b < 4 else (4 if b < 16 else 2))
         if name == "qwen3-0.6b" and b == 1 and args.long_parity_steps > 0:
             steps = nb = args.long_parity_steps  # the 1000-step config: every step a new query
-        out.append(config_entry(torch, vie, dev, stream, flush, name, b, k, steps, 10, nb, peaks,
-                                peak_src, cache, args.seed))
+        out.append(config_entry(torch, vie, dev, stream, flush, name, b, k, steps, args.config_warmup, nb,
+                                peaks, peak_src, cache, args.seed))
     if cache.get("head") is not None:
         cache["head"].close()
     return out
