@@ -354,9 +354,10 @@ vie_status vie_scatter_sparse_logits(const int32_t *idx, const float *logits, in
  * vie_head_topk_noalloc - vie_head_topk for callers that cannot allocate
  * device memory.  The paper has no counterpart: this is a deployment variant.
  *
- * Some callers are not allowed to call cudaMalloc at all: code running while
- * a CUDA graph is being captured, engines whose device memory is carved out
- * of one budget up front, and latency-critical loops that cannot afford the
+ * Some callers are not allowed to call cudaMalloc at all: serving engines
+ * whose device memory is carved out of one budget up front (a further
+ * allocation could fail mid-request or take memory another model was
+ * promised), and latency-critical decode loops that cannot afford the
  * implicit device synchronisation an allocation may bring.  A vie_head
  * allocates its padded weight copy and scratch in vie_head_create, so those
  * callers cannot make one.  This entry point takes the weights as they are

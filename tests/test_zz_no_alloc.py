@@ -1,7 +1,6 @@
 """vie_head_topk_noalloc: top-k for callers that must not allocate device
-memory -- code that runs while a CUDA graph is being captured (where
-cudaMalloc is not allowed), engines that carve all device memory out of one
-budget fixed at start-up, and decode loops that cannot afford the device
+memory -- serving engines that carve all device memory out of one budget
+fixed at start-up, and decode loops that cannot afford the device
 synchronisation an allocation may cause.
 
 Its results must pass the oracle's acceptance rule and agree with
